@@ -1,0 +1,363 @@
+"""Benchmark: quantized MoE layer decode on GB300.
+
+One step = one pass of the whole layer (router logits, group-limited top-k,
+permutation, SwiGLU gate/up, down + weighted combine + shared expert) over
+one batch of synthetic tokens, through the C ABI (moe_quant_forward).
+Default workload: one DeepSeek-V3-shaped layer (hidden 7168, expert
+intermediate 2048, 192 surviving experts of 256, 8 groups / 4 kept, top-8,
+shared expert), decode batch of 1 token, gate/up Q2_K-style, down
+Q3_K-style, shared expert Q8_0.  Packed weights are drawn on the device;
+every step gets a fresh token and the L2 is flushed (256 MB write) before it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+
+With N > 1 (torchrun, one rank per GPU) every rank runs an independent
+replica of the layer (weak scaling; no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tokens/s and achieved HBM GB/s (% of peak) for quantized MoE layer decode, 1 GB300"
+WORKLOAD = "v3_decode_t1"
+FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                c = [s.strip() for s in line.split(",")]
+                if len(c) < 9:
+                    continue
+                try:
+                    sm.append(float(c[1])); smax.append(float(c[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, c[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def step_bytes(spec, fmts, idx_steps):
+    """Algorithmic bytes per step for each kernel (packed bytes of the tensors
+    each kernel must read, plus activations)."""
+    from workloads.configs import packed_bytes
+    H, I, E, T, K = spec.hidden, spec.inter, spec.n_experts, spec.tokens, spec.top_k
+    gu = lambda e: packed_bytes(int(fmts[e, 0]), I, H) + packed_bytes(int(fmts[e, 1]), I, H)
+    dn = lambda e: packed_bytes(int(fmts[e, 2]), H, I)
+    sh = E if spec.has_shared else None
+    out = []
+    for idx in idx_steps:
+        touched = sorted(set(int(e) for e in idx.reshape(-1)))
+        b_gu = sum(gu(e) for e in touched) + (gu(sh) if sh is not None else 0) + T * H * 2 + (T * K + T) * I * 4
+        b_dn = sum(dn(e) for e in touched) + (dn(sh) if sh is not None else 0) + (T * K + T) * I * 4 + T * H * 4
+        b_rt = E * H * 4 + T * H * 2 + T * E * 4
+        quant = sum(gu(e) + dn(e) for e in touched) + ((gu(sh) + dn(sh)) if sh is not None else 0)
+        out.append({"gateup": b_gu, "down": b_dn, "router_logits": b_rt, "quantized": quant,
+                    "total": b_gu + b_dn + b_rt})
+    return out
+
+
+def cpu_baseline(host_layer, x_steps, budget_s=15.0, max_tokens=8):
+    """The oracle (plain single-threaded C) on a bounded sample of tokens."""
+    import oracle
+    oracle.build()
+    done, t_used = 0, 0.0
+    for i in range(min(max_tokens, len(x_steps))):
+        t_used += host_layer.timed_forward(oracle, x_steps[i])
+        done += x_steps[i].shape[0]
+        if t_used > budget_s:
+            break
+    return {"value": done / t_used, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"{done} decode token(s) of a V3 layer of the same recipe (fresh token each), full layer "
+                      f"per token: routing + 8 routed experts + shared expert, fp64 FFN; {t_used:.1f} s"}
+
+
+class HostOracleLayer:
+    """Host-only layer for the oracle: same seeded recipe as the device layer;
+    packed tensors are drawn on the host for the experts a token touches."""
+
+    def __init__(self, spec, seed):
+        from workloads.synth import draw_formats, draw_router
+        self.spec, self.seed = spec, seed
+        self.fmts = draw_formats(spec, seed)
+        self.router_w, self.bias = draw_router(spec, seed)
+        self.cache = {}
+
+    def timed_forward(self, orc, x_bits):
+        from workloads.synth import draw_packed_layer_host
+        spec = self.spec
+        layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
+                               spec.top_k, spec.routed_scale, spec.has_shared)
+        idx, _, _, _ = orc.route(layer, x_bits, self.router_w, self.bias)
+        n = spec.n_experts + (1 if spec.has_shared else 0)
+        used = set(int(e) for e in idx.reshape(-1)) | set(range(spec.n_experts, n))
+        for e in used:
+            if e not in self.cache:
+                self.cache[e] = draw_packed_layer_host(spec, self.seed, self.fmts, experts=[e])[e]
+        dummy = np.zeros(16, np.uint8)
+        g = [self.cache[e][0] if e in used else dummy for e in range(n)]
+        u = [self.cache[e][1] if e in used else dummy for e in range(n)]
+        d = [self.cache[e][2] if e in used else dummy for e in range(n)]
+        t0 = time.perf_counter()
+        orc.moe_forward(layer, x_bits, self.router_w, self.bias, g, u, d, self.fmts)
+        return time.perf_counter() - t0
+
+
+class BenchLayer:
+    def __init__(self, spec, seed):
+        import torch
+        import paper_2509_25689_gb300 as mq
+        from workloads.synth import draw_formats, draw_router, random_packed_device, tensor_shapes
+        self.mq, self.spec = mq, spec
+        self.fmts = draw_formats(spec, seed)
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(seed * 7919 + 13)
+        shapes = tensor_shapes(spec)
+        n = spec.n_experts + (1 if spec.has_shared else 0)
+        self.tensors = [tuple(random_packed_device(int(self.fmts[e, j]), *shapes[j], gen, "cuda") for j in range(3))
+                        for e in range(n)]
+        self.table = mq.ExpertTable(self.tensors[:spec.n_experts],
+                                    self.tensors[spec.n_experts] if spec.has_shared else None)
+        rw, b = draw_router(spec, seed)
+        self.router_w_host, self.bias_host = rw, b
+        self.router_w, self.bias = torch.from_numpy(rw).cuda(), torch.from_numpy(b).cuda()
+        self.cfg = mq.make_cfg(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
+                               spec.top_k, spec.routed_scale, spec.has_shared)
+        self.wsb = mq.moe_quant_workspace_size(self.cfg, spec.tokens)
+        self.ws = torch.empty(self.wsb, dtype=torch.uint8, device="cuda")
+        self.out = torch.empty((spec.tokens, spec.hidden), dtype=torch.float32, device="cuda")
+        self.wts = torch.empty((spec.tokens, spec.top_k), dtype=torch.float32, device="cuda")
+
+    def forward(self, x, idx_out, out=None):
+        self.mq.moe_quant_forward(self.cfg, self.spec.tokens, x, self.router_w, self.bias, self.table, self.fmts,
+                                  self.out if out is None else out, idx_out, self.wts, self.ws, self.wsb)
+
+
+def run_native(args):
+    import torch
+    import torch.distributed as dist
+    from workloads import get_config
+    from workloads.synth import draw_tokens
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    spec = get_config(args.config)
+    T, K, W = spec.tokens, args.steps, args.warmup
+    layer = BenchLayer(spec, seed=rank)
+    steps = W + K
+    x_host = np.stack([draw_tokens(1000 + rank * 100003 + i, T, spec.hidden) for i in range(steps)])
+    x_dev = torch.from_numpy(x_host.view(np.int16)).cuda()
+    idx_all = torch.empty((steps, T, spec.top_k), dtype=torch.int32, device="cuda")
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device="cuda")
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for i in range(W):
+        flush.fill_(i)
+        layer.forward(x_dev[i], idx_all[i])
+    barrier()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    layer.mq.mq_profile_enable(K * 8)
+    barrier()
+    t_wall0 = time.perf_counter()
+    for i in range(K):
+        flush.fill_(i)
+        evs[i][0].record()
+        layer.forward(x_dev[W + i], idx_all[W + i])
+        evs[i][1].record()
+    barrier()
+    t_wall = time.perf_counter() - t_wall0
+    kstats = layer.mq.mq_profile_collect()
+    clk = clocks.stop()
+    dev_ms = sum(a.elapsed_time(b) for a, b in evs)
+    t = torch.tensor([dev_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dev_ms_max = float(t.item())
+
+    # e2e through the C ABI with host buffers (pinned), copies inside the region
+    x_pin = torch.from_numpy(x_host.view(np.int16)).pin_memory()
+    out_pin = torch.empty((K, T, spec.hidden), dtype=torch.float32).pin_memory()
+    x_step = torch.empty((T, spec.hidden), dtype=torch.int16, device="cuda")
+    e2e_evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    barrier()
+    for i in range(K):
+        flush.fill_(i)
+        e2e_evs[i][0].record()
+        x_step.copy_(x_pin[W + i], non_blocking=True)
+        layer.forward(x_step, idx_all[W + i])
+        out_pin[i].copy_(layer.out, non_blocking=True)
+        e2e_evs[i][1].record()
+    barrier()
+    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_evs)
+    t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e2e_ms_max = float(t.item())
+
+    idx_host = idx_all[W:].cpu().numpy()
+    sb = step_bytes(spec, layer.fmts, idx_host)
+    peak, peak_src = _peaks()
+    quant_bytes = sum(s["quantized"] for s in sb)
+    gbs = quant_bytes / (dev_ms / 1e3) / 1e9
+    result = None
+    if rank == 0:
+        dominant = max(kstats, key=lambda s: s[2]) if kstats else None
+        roof = None
+        if dominant:
+            name, launches, tot_ms = dominant
+            per_launch_bytes = sum(s.get(name, 0) for s in sb) / max(len(sb), 1)
+            avg_s = tot_ms / launches / 1e3
+            achieved = per_launch_bytes / avg_s / 1e9
+            roof = {"bound": "hbm", "kernel": name, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                    "frac": round(achieved / peak, 4), "traffic": None, "peak_source": peak_src,
+                    "algorithmic_bytes_per_launch": int(per_launch_bytes), "avg_launch_us": round(avg_s * 1e6, 2)}
+        result = {
+            "metric": METRIC, "value": round(world * T * K / (dev_ms_max / 1e3), 2), "unit": "tokens/s",
+            "n_gpus": world, "steps": K, "warmup": W, "ms_per_step": round(dev_ms_max / K, 5),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "fp32-acc/q2k-q3k-q8_0",
+            "data": "synthetic (seeded random packed weights on device; fresh N(0,1) bf16 token per step)",
+            "config": {"workload": f"{spec.name}: V3 MoE layer, hidden {spec.hidden}, inter {spec.inter}, "
+                                   f"{spec.n_experts} experts + shared, G={spec.n_groups}/{spec.topk_group}, "
+                                   f"top-{spec.top_k}, T={T}", "l2": "flushed (256 MB write) before every step",
+                       "parallelism": f"replicas x{world}"},
+            "achieved_hbm_gbs": round(gbs, 1), "hbm_frac_of_measured": round(gbs / peak, 4),
+            "hbm_frac_of_8tbs": round(gbs / 8000.0, 4), "quantized_bytes_per_step": int(quant_bytes / K),
+            "roofline": roof,
+            "kernels": [{"name": n, "launches": l, "total_ms": round(ms, 4)} for n, l, ms in kstats],
+            "gpu_launches": int(sum(l for _, l, _ in kstats)),
+            "wall_s_timed_region": round(t_wall, 4),
+            "clocks": clk,
+            "e2e": {"value": round(world * T * K / (e2e_ms_max / 1e3), 2), "unit": "tokens/s",
+                    "h2d_bytes_per_step": int(T * spec.hidden * 2), "d2h_bytes_per_step": int(T * spec.hidden * 4)},
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            xs = [x_host[W + i] for i in range(min(K, 8))]
+            result["cpu_baseline"] = cpu_baseline(HostOracleLayer(spec, seed=0), xs)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    if result is not None:
+        print(json.dumps(result))
+
+
+def run_reference(args):
+    """Reference arm: the oracle as it stands, on the host cores, rank 0."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    from workloads import get_config
+    from workloads.synth import draw_tokens
+    oracle.build()
+    spec = get_config(args.config)
+    host = HostOracleLayer(spec, seed=0)
+    budget_s, done_steps, t_used = 150.0, 0, 0.0
+    for i in range(min(args.warmup, 1)):
+        host.timed_forward(oracle, draw_tokens(1000 + i, spec.tokens, spec.hidden))
+    for i in range(args.steps):
+        t_used += host.timed_forward(oracle, draw_tokens(1000 + args.warmup + i, spec.tokens, spec.hidden))
+        done_steps += 1
+        if t_used > budget_s:
+            break
+    value = done_steps * spec.tokens / t_used
+    line = {"metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": 1, "steps": done_steps,
+            "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t_used / done_steps * 1e3, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{spec.name} (oracle: plain single-threaded C, fp64 FFN)"},
+            "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{done_steps} step(s) of one decode token each (time budget {budget_s} s)"},
+            "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--config", default=WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -9,12 +9,13 @@ from __future__ import annotations
 
 import ctypes
 import os
+import platform
 import subprocess
 
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SO = os.path.join(_HERE, "liboracle.so")
+_SO = os.path.join(_HERE, f"liboracle_{platform.machine()}.so")
 
 Q2_K, Q3_K, Q4_K, Q8_0 = 1, 2, 3, 4
 FORMATS = {"Q2_K": Q2_K, "Q3_K": Q3_K, "Q4_K": Q4_K, "Q8_0": Q8_0}

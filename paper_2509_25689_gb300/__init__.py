@@ -1,0 +1,208 @@
+"""Python binding of libmoeq (quantized MoE expert-FFN layer for GB300).
+
+Argument marshalling only: every function forwards to the C ABI entry point
+of the same name in libmoeq.so (include/moeq.h).  Tensors may be torch
+tensors (device or host) or numpy arrays (host); their data pointers are
+passed through.  Importing this module fails loudly if the CUDA library has
+not been built: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libmoeq.so")
+
+MQ_Q2_K, MQ_Q3_K, MQ_Q4_K, MQ_Q8_0 = 1, 2, 3, 4
+FORMATS = {"Q2_K": MQ_Q2_K, "Q3_K": MQ_Q3_K, "Q4_K": MQ_Q4_K, "Q8_0": MQ_Q8_0}
+MQ_OK = 0
+
+
+class MoeqError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        super().__init__(f"{fn}: {mq_strerror(status)} ({status})")
+        self.status = status
+
+
+class mq_layer_cfg(ctypes.Structure):
+    _fields_ = [
+        ("hidden", ctypes.c_int32), ("inter", ctypes.c_int32), ("n_experts", ctypes.c_int32),
+        ("n_groups", ctypes.c_int32), ("topk_group", ctypes.c_int32), ("top_k", ctypes.c_int32),
+        ("routed_scale", ctypes.c_float), ("has_shared", ctypes.c_int32),
+    ]
+
+
+class mq_expert_weights(ctypes.Structure):
+    _fields_ = [("gate", ctypes.c_void_p), ("up", ctypes.c_void_p), ("down", ctypes.c_void_p)]
+
+
+class mq_expert_table(ctypes.Structure):
+    _fields_ = [("experts", ctypes.POINTER(mq_expert_weights)),
+                ("shared", ctypes.POINTER(mq_expert_weights))]
+
+
+class mq_kernel_stat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int32), ("total_ms", ctypes.c_double)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libmoeq.so not built ({LIB_PATH}); run paper_2509_25689_gb300/build.py")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+    cfgp = ctypes.POINTER(mq_layer_cfg)
+    sig = {
+        "mq_packed_size": (sz, [ctypes.c_int, i64, i64]),
+        "mq_pack": (ctypes.c_int, [ctypes.c_int, vp, i64, i64, vp, sz]),
+        "mq_unpack": (ctypes.c_int, [ctypes.c_int, vp, i64, i64, vp]),
+        "mq_unpack_device": (ctypes.c_int, [ctypes.c_int, vp, i64, i64, vp, vp]),
+        "moe_quant_workspace_size": (sz, [cfgp, i32]),
+        "moe_quant_forward": (ctypes.c_int, [cfgp, i32, vp, vp, vp, ctypes.POINTER(mq_expert_table), vp,
+                                             vp, vp, vp, vp, sz, vp]),
+        "moe_quant_route": (ctypes.c_int, [cfgp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
+        "mq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+        "mq_set_path": (ctypes.c_int, [ctypes.c_int, i32]),
+        "mq_profile_enable": (ctypes.c_int, [i32]),
+        "mq_profile_collect": (ctypes.c_int, [ctypes.POINTER(mq_kernel_stat), i32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype, fn.argtypes = res, args
+    return L
+
+
+_lib = _load()
+EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
+            "moe_quant_forward", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
+            "mq_profile_collect")
+
+
+def _ptr(a):
+    """Data pointer of a torch tensor / numpy array / int / None."""
+    if a is None:
+        return None
+    if isinstance(a, int):
+        return a
+    if hasattr(a, "data_ptr"):
+        return a.data_ptr()
+    return a.ctypes.data
+
+
+def _stream(stream):
+    if stream is None:
+        try:
+            import torch
+            if torch.cuda.is_available():
+                return torch.cuda.current_stream().cuda_stream
+        except ImportError:
+            pass
+        return None
+    return getattr(stream, "cuda_stream", stream)
+
+
+def _check(fn, rc):
+    if rc != MQ_OK:
+        raise MoeqError(fn, rc)
+    return rc
+
+
+def _fmt(f):
+    return FORMATS[f] if isinstance(f, str) else int(f)
+
+
+def mq_strerror(status: int) -> str:
+    return _lib.mq_strerror(status).decode()
+
+
+def mq_packed_size(fmt, rows: int, cols: int) -> int:
+    return int(_lib.mq_packed_size(_fmt(fmt), rows, cols))
+
+
+def mq_pack(fmt, w, dst=None):
+    """Host quantizer. w: float32 [rows, cols] (numpy or CPU tensor).
+    Returns dst (a new numpy uint8 array when dst is None)."""
+    import numpy as np
+    w = np.ascontiguousarray(w if not hasattr(w, "numpy") else w.numpy(), dtype=np.float32)
+    rows, cols = w.shape
+    n = mq_packed_size(fmt, rows, cols)
+    if dst is None:
+        dst = np.empty(n, np.uint8)
+    _check("mq_pack", _lib.mq_pack(_fmt(fmt), w.ctypes.data, rows, cols, _ptr(dst), n))
+    return dst
+
+
+def mq_unpack(fmt, src, rows: int, cols: int):
+    import numpy as np
+    src = np.ascontiguousarray(src, dtype=np.uint8)
+    out = np.empty((rows, cols), np.float32)
+    _check("mq_unpack", _lib.mq_unpack(_fmt(fmt), src.ctypes.data, rows, cols, out.ctypes.data))
+    return out
+
+
+def mq_unpack_device(fmt, src, rows: int, cols: int, dst, stream=None):
+    _check("mq_unpack_device",
+           _lib.mq_unpack_device(_fmt(fmt), _ptr(src), rows, cols, _ptr(dst), _stream(stream)))
+    return dst
+
+
+def make_cfg(hidden, inter, n_experts, n_groups, topk_group, top_k, routed_scale=1.0, has_shared=False):
+    return mq_layer_cfg(hidden, inter, n_experts, n_groups, topk_group, top_k, float(routed_scale),
+                        int(bool(has_shared)))
+
+
+def moe_quant_workspace_size(cfg: mq_layer_cfg, n_tokens: int) -> int:
+    return int(_lib.moe_quant_workspace_size(ctypes.byref(cfg), n_tokens))
+
+
+class ExpertTable:
+    """Holds the ctypes expert table built from per-expert (gate, up, down)
+    device tensors or raw pointers; keeps the ctypes arrays alive."""
+
+    def __init__(self, experts, shared=None):
+        n = len(experts)
+        self._arr = (mq_expert_weights * max(n, 1))()
+        for i, (g, u, d) in enumerate(experts):
+            self._arr[i] = mq_expert_weights(_ptr(g), _ptr(u), _ptr(d))
+        self._shared = None
+        if shared is not None:
+            self._shared = mq_expert_weights(*[_ptr(t) for t in shared])
+        self.table = mq_expert_table(
+            ctypes.cast(self._arr, ctypes.POINTER(mq_expert_weights)),
+            ctypes.pointer(self._shared) if self._shared is not None else None)
+
+
+def moe_quant_forward(cfg, n_tokens, x, router_w, bias, expert_table: ExpertTable, fmt_per_tensor, out,
+                      topk_idx=None, topk_w=None, workspace=None, ws_bytes=None, stream=None):
+    import numpy as np
+    fmt = np.ascontiguousarray(fmt_per_tensor, dtype=np.uint8).reshape(-1)
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = _lib.moe_quant_forward(ctypes.byref(cfg), n_tokens, _ptr(x), _ptr(router_w), _ptr(bias),
+                                ctypes.byref(expert_table.table), fmt.ctypes.data, _ptr(out), _ptr(topk_idx),
+                                _ptr(topk_w), _ptr(workspace), ws_bytes, _stream(stream))
+    return _check("moe_quant_forward", rc)
+
+
+def moe_quant_route(cfg, n_tokens, x, router_w, bias, topk_idx, topk_w, offsets=None, perm=None, inv=None,
+                    workspace=None, ws_bytes=None, stream=None):
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = _lib.moe_quant_route(ctypes.byref(cfg), n_tokens, _ptr(x), _ptr(router_w), _ptr(bias), _ptr(topk_idx),
+                              _ptr(topk_w), _ptr(offsets), _ptr(perm), _ptr(inv), _ptr(workspace), ws_bytes,
+                              _stream(stream))
+    return _check("moe_quant_route", rc)
+
+
+def mq_set_path(mode: int, prefill_threshold: int = 0):
+    return _check("mq_set_path", _lib.mq_set_path(mode, prefill_threshold))
+
+
+def mq_profile_enable(max_launches: int):
+    return _check("mq_profile_enable", _lib.mq_profile_enable(max_launches))
+
+
+def mq_profile_collect(max_entries: int = 64):
+    arr = (mq_kernel_stat * max_entries)()
+    n = _lib.mq_profile_collect(arr, max_entries)
+    return [(arr[i].name.decode(), int(arr[i].launches), float(arr[i].total_ms)) for i in range(n)]

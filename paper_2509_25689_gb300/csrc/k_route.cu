@@ -1,0 +1,315 @@
+// Router and permutation kernels.
+//
+// Router (arXiv 2509.25689 Sec. 3.2: sigmoid expert scores, topk_group
+// groups over the pruned experts, num_experts_per_tok experts per token)
+// in a canonical fp32 order so that expert ids are bit-exact with the CPU
+// reference:
+//   logit:   the row is cut in segments of 8 chunks x 128 elements; lane l
+//            of the segment's warp runs one fma chain over chunk i, elements
+//            128 i + 4 l + c (c = 0..3); an xor butterfly (16, 8, 4, 2, 1)
+//            adds partners; segment results are added left to right.
+//   sigmoid: Cody-Waite reduction a = n ln2 + r, degree-7 Taylor for e^r
+//            (coefficients 1/i! rounded to fp32, Horner), exact 2^n scaling,
+//            1/(1+e) with IEEE division; |a| clamped to 87.
+//   select:  u = s + bias; group score = sum of the two largest u of a
+//            group; keep topk_group groups, then top_k experts by u; ties go
+//            to the lower index; weights s_j / sum(s) in slot order.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mq_internal.h"
+
+namespace mq {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// ---------------------------------------------------------------------------
+// logits: grid (E, ceil(T / kTok)), one warp per 1024-element segment
+// ---------------------------------------------------------------------------
+constexpr int kTok = 8;
+
+__global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
+                                                             const float* __restrict__ W, int H, int T,
+                                                             int E, float* __restrict__ z) {
+    __shared__ float part[32][kTok];
+    const int e = blockIdx.x, t0 = blockIdx.y * kTok;
+    const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
+    const int c0 = seg * 8, nc = min(8, nchunk - c0);
+    const float* wrow = W + (size_t)e * H;
+    float4 wv[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(wrow + (c0 + c) * 128 + 4 * lane));
+    float acc[kTok];
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) acc[j] = 0.0f;
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) {
+        const int t = t0 + j;
+        if (t >= T) break;
+        const uint16_t* xr = x + (size_t)t * H;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            if (c < nc) {
+                const uint2 xv = __ldg(reinterpret_cast<const uint2*>(xr + (c0 + c) * 128 + 4 * lane));
+                acc[j] = __fmaf_rn(bf16_lo(xv.x), wv[c].x, acc[j]);
+                acc[j] = __fmaf_rn(bf16_hi(xv.x), wv[c].y, acc[j]);
+                acc[j] = __fmaf_rn(bf16_lo(xv.y), wv[c].z, acc[j]);
+                acc[j] = __fmaf_rn(bf16_hi(xv.y), wv[c].w, acc[j]);
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) {
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) acc[j] = __fadd_rn(acc[j], __shfl_xor_sync(kFull, acc[j], off));
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int j = 0; j < kTok; ++j) part[seg][j] = acc[j];
+    }
+    __syncthreads();
+    if (threadIdx.x < kTok) {
+        const int t = t0 + threadIdx.x;
+        if (t < T) {
+            float r = part[0][threadIdx.x];
+            for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
+            z[(size_t)t * E + e] = r;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// scores + group-limited top-k: one warp per token
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float canonical_sigmoid(float z) {
+    const float kLog2e = 0x1.715476p+0f, kLn2Hi = 0x1.62e4p-1f, kLn2Lo = 0x1.7f7d1cp-20f;
+    float a = __fsub_rn(0.0f, z);
+    if (a > 87.0f) a = 87.0f;
+    if (a < -87.0f) a = -87.0f;
+    const float n = rintf(__fmul_rn(a, kLog2e));
+    float r = __fmaf_rn(-n, kLn2Hi, a);
+    r = __fmaf_rn(-n, kLn2Lo, r);
+    // e^r = sum r^i / i!, i <= 7
+    float p = 0x1.a01a02p-13f;
+    p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);
+    p = __fmaf_rn(p, r, 0x1.111112p-7f);
+    p = __fmaf_rn(p, r, 0x1.555556p-5f);
+    p = __fmaf_rn(p, r, 0x1.555556p-3f);
+    p = __fmaf_rn(p, r, 0.5f);
+    p = __fmaf_rn(p, r, 1.0f);
+    p = __fmaf_rn(p, r, 1.0f);
+    const float two_n = __int_as_float(((int)n + 127) << 23);
+    const float ex = __fmul_rn(p, two_n);
+    return __fdiv_rn(1.0f, __fadd_rn(1.0f, ex));
+}
+
+// (value, index) argmax: larger value wins, equal values -> lower index
+__device__ __forceinline__ void better(float& v, int& i, float v2, int i2) {
+    if (i2 >= 0 && (i < 0 || v2 > v || (v2 == v && i2 < i))) { v = v2; i = i2; }
+}
+__device__ __forceinline__ int warp_argmax(float v, int i) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+        const float v2 = __shfl_xor_sync(kFull, v, off);
+        const int i2 = __shfl_xor_sync(kFull, i, off);
+        better(v, i, v2, i2);
+    }
+    return i;
+}
+
+constexpr int kTopkWarps = 4;
+
+__global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __restrict__ z,
+                                                               const float* __restrict__ bias, Dims d,
+                                                               int32_t* __restrict__ idx,
+                                                               float* __restrict__ wts) {
+    __shared__ float s_sh[kTopkWarps][kMaxExperts];
+    __shared__ float u_sh[kTopkWarps][kMaxExperts];
+    __shared__ float g_sh[kTopkWarps][kMaxGroups];
+    __shared__ uint8_t keep_g[kTopkWarps][kMaxGroups];
+    __shared__ uint8_t taken[kTopkWarps][kMaxExperts];
+    __shared__ int32_t sel[kTopkWarps][kMaxTopK];
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t = blockIdx.x * kTopkWarps + w;
+    if (t >= d.T) return;
+    const int E = d.E, G = d.G, gs = E / G;
+    for (int e = lane; e < E; e += 32) {
+        const float s = canonical_sigmoid(z[(size_t)t * E + e]);
+        s_sh[w][e] = s;
+        u_sh[w][e] = __fadd_rn(s, bias ? bias[e] : 0.0f);
+        taken[w][e] = 0;
+    }
+    __syncwarp();
+    for (int g = lane; g < G; g += 32) {
+        float top1 = -INFINITY, top2 = -INFINITY;
+        for (int i = 0; i < gs; ++i) {
+            const float v = u_sh[w][g * gs + i];
+            if (v > top1) { top2 = top1; top1 = v; }
+            else if (v > top2) top2 = v;
+        }
+        g_sh[w][g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
+        keep_g[w][g] = 0;
+    }
+    __syncwarp();
+    for (int r = 0; r < d.Gk; ++r) {
+        float bv = 0.0f; int bi = -1;
+        for (int g = lane; g < G; g += 32)
+            if (!keep_g[w][g]) better(bv, bi, g_sh[w][g], g);
+        bi = warp_argmax(bv, bi);
+        if (lane == 0) keep_g[w][bi] = 1;
+        __syncwarp();
+    }
+    for (int j = 0; j < d.K; ++j) {
+        float bv = 0.0f; int bi = -1;
+        for (int e = lane; e < E; e += 32)
+            if (keep_g[w][e / gs] && !taken[w][e]) better(bv, bi, u_sh[w][e], e);
+        bi = warp_argmax(bv, bi);
+        if (lane == 0) { taken[w][bi] = 1; sel[w][j] = bi; }
+        __syncwarp();
+    }
+    if (lane == 0) {
+        float sum = 0.0f;
+        for (int j = 0; j < d.K; ++j) sum = __fadd_rn(sum, s_sh[w][sel[w][j]]);
+        for (int j = 0; j < d.K; ++j) {
+            const int e = sel[w][j];
+            idx[(size_t)t * d.K + j] = e;
+            wts[(size_t)t * d.K + j] = __fmul_rn(__fdiv_rn(s_sh[w][e], sum), d.routed_scale);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// permutation: one CTA; stable counting sort of entries a = t*K + j by expert
+// ---------------------------------------------------------------------------
+constexpr int kPermThreads = 1024;
+constexpr int kPermWarps = kPermThreads / 32;
+
+__global__ void __launch_bounds__(kPermThreads) permute_kernel(const int32_t* __restrict__ idx, int n, int E,
+                                                               int32_t* __restrict__ offsets,
+                                                               int32_t* __restrict__ perm,
+                                                               int32_t* __restrict__ inv,
+                                                               int32_t* __restrict__ active) {
+    __shared__ int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
+    __shared__ int32_t total[kMaxExperts + 1];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int i = threadIdx.x; i < kPermWarps * kMaxExperts; i += kPermThreads) (&cnt[0][0])[i] = 0;
+    __syncthreads();
+    const int seg = (n + kPermWarps - 1) / kPermWarps;
+    const int a0 = warp * seg, a1 = min(n, a0 + seg);
+    for (int a = a0 + lane; a < a1; a += 32) atomicAdd(&cnt[warp][idx[a]], 1);
+    __syncthreads();
+    // per-expert totals and per-warp starting cursors (warp order = entry order)
+    if (threadIdx.x < E) {
+        const int e = threadIdx.x;
+        int run = 0;
+        for (int wv = 0; wv < kPermWarps; ++wv) { const int c = cnt[wv][e]; cnt[wv][e] = run; run += c; }
+        total[e] = run;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        // exclusive scan of totals over experts (E <= 256: 8 per lane)
+        int local[8], sum = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int e = lane * 8 + q;
+            local[q] = e < E ? total[e] : 0;
+            sum += local[q];
+        }
+        int incl = sum;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int v = __shfl_up_sync(kFull, incl, off);
+            if (lane >= off) incl += v;
+        }
+        int run = incl - sum;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int e = lane * 8 + q;
+            if (e < E) { offsets[e] = run; total[e] = run; }
+            run += local[q];
+        }
+        if (lane == 31) { offsets[E] = run; }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < kPermWarps * E; i += kPermThreads) {
+        const int wv = i / E, e = i % E;
+        cnt[wv][e] += total[e];
+    }
+    __syncthreads();
+    // stable scatter: each warp walks its segment in order, 32 entries a step
+    for (int base = a0; base < a1; base += 32) {
+        const int a = base + lane;
+        const bool ok = a < a1;
+        const int e = ok ? idx[a] : -1 - lane;
+        const unsigned peers = __match_any_sync(kFull, e);
+        const int rank = __popc(peers & ((1u << lane) - 1u));
+        if (ok) {
+            const int pos = cnt[warp][e] + rank;
+            perm[pos] = a;
+            inv[a] = pos;
+        }
+        __syncwarp();
+        if (ok && rank == 0) cnt[warp][e] += __popc(peers);
+        __syncwarp();
+    }
+    __syncthreads();
+    // active expert list (ascending ids), active[0] = count
+    if (warp == 0) {
+        int flags = 0, c = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int e = lane * 8 + q;
+            const int f = (e < E && offsets[e + 1] > offsets[e]) ? 1 : 0;
+            flags |= f << q;
+            c += f;
+        }
+        int incl = c;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int v = __shfl_up_sync(kFull, incl, off);
+            if (lane >= off) incl += v;
+        }
+        int pos = incl - c;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (flags & (1 << q)) active[1 + pos++] = lane * 8 + q;
+        if (lane == 31) active[0] = incl;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, cudaStream_t s) {
+    if (d.T == 0) return cudaSuccess;
+    const int nseg = (d.H / 128 + 7) / 8;
+    dim3 grid(d.E, (d.T + kTok - 1) / kTok);
+    prof_begin("router_logits", s);
+    router_logits_kernel<<<grid, nseg * 32, 0, s>>>(x, W, d.H, d.T, d.E, z);
+    prof_end(s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
+                        cudaStream_t s) {
+    if (d.T == 0) return cudaSuccess;
+    prof_begin("router_topk", s);
+    topk_kernel<<<(d.T + kTopkWarps - 1) / kTopkWarps, kTopkWarps * 32, 0, s>>>(z, bias, d, idx, wts);
+    prof_end(s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
+                           int32_t* active, cudaStream_t s) {
+    prof_begin("permute", s);
+    permute_kernel<<<1, kPermThreads, 0, s>>>(idx, d.T * d.K, d.E, offsets, perm, inv, active);
+    prof_end(s);
+    return cudaGetLastError();
+}
+
+}  // namespace mq

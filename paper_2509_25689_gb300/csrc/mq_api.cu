@@ -1,0 +1,269 @@
+// C ABI of libmoeq: argument checks, workspace carving, kernel dispatch,
+// optional kernel timing.  See include/moeq.h for the contract.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/moeq.h"
+#include "mq_internal.h"
+
+namespace mq {
+namespace {
+
+size_t up256(size_t v) { return (v + 255) & ~size_t(255); }
+
+int g_path_mode = -1;        // -1: not yet read from the environment
+int32_t g_prefill_threshold = 64;
+
+int path_mode() {
+    if (g_path_mode < 0) {
+        const char* env = std::getenv("MQ_FORCE_PATH");
+        g_path_mode = 0;
+        if (env && std::strcmp(env, "decode") == 0) g_path_mode = 1;
+        if (env && std::strcmp(env, "prefill") == 0) g_path_mode = 2;
+    }
+    return g_path_mode;
+}
+
+int check_cfg(const mq_layer_cfg* c) {
+    if (!c) return MQ_EINVAL;
+    if (c->hidden < 128 || c->hidden % 128 || c->hidden > 32768) return MQ_ESHAPE;
+    if (c->inter < 128 || c->inter % 128 || c->inter > 16384) return MQ_ESHAPE;
+    if (c->n_experts < 1 || c->n_experts > kMaxExperts) return MQ_ESHAPE;
+    if (c->n_groups < 1 || c->n_groups > kMaxGroups || c->n_experts % c->n_groups) return MQ_ESHAPE;
+    if (c->topk_group < 1 || c->topk_group > c->n_groups) return MQ_ESHAPE;
+    if (c->top_k < 1 || c->top_k > kMaxTopK) return MQ_ESHAPE;
+    if (c->top_k > c->topk_group * (c->n_experts / c->n_groups)) return MQ_ESHAPE;
+    if (c->has_shared != 0 && c->has_shared != 1) return MQ_EINVAL;
+    if (!std::isfinite(c->routed_scale)) return MQ_EINVAL;
+    return MQ_OK;
+}
+
+Dims dims_of(const mq_layer_cfg* c, int32_t T) {
+    Dims d;
+    d.H = c->hidden; d.I = c->inter; d.E = c->n_experts; d.G = c->n_groups; d.Gk = c->topk_group;
+    d.K = c->top_k; d.T = T; d.has_shared = c->has_shared; d.routed_scale = c->routed_scale;
+    return d;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ---- kernel timing -------------------------------------------------------
+struct ProfRec { const char* name; cudaEvent_t a, b; };
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+int32_t g_prof_cap = 0;
+std::vector<ProfRec> g_prof;
+
+}  // namespace
+
+size_t workspace_plan(const Dims& d, void* base, Work* w) {
+    const size_t TK = (size_t)d.T * d.K;
+    size_t at = 0;
+    auto take = [&](size_t bytes) { const size_t o = at; at += up256(bytes); return o; };
+    const size_t o_z = take((size_t)d.T * d.E * 4);
+    const size_t o_idx = take(TK * 4), o_w = take(TK * 4);
+    const size_t o_off = take((size_t)(d.E + 1) * 4);
+    const size_t o_perm = take(TK * 4), o_inv = take(TK * 4);
+    const size_t o_act = take((size_t)(d.E + 2) * 4);
+    const size_t o_h = take((TK + (size_t)d.T) * d.I * 4);
+    const size_t o_err = take(4);
+    if (w && base) {
+        char* b = static_cast<char*>(base);
+        w->z = reinterpret_cast<float*>(b + o_z);
+        w->idx = reinterpret_cast<int32_t*>(b + o_idx);
+        w->wts = reinterpret_cast<float*>(b + o_w);
+        w->offsets = reinterpret_cast<int32_t*>(b + o_off);
+        w->perm = reinterpret_cast<int32_t*>(b + o_perm);
+        w->inv = reinterpret_cast<int32_t*>(b + o_inv);
+        w->active = reinterpret_cast<int32_t*>(b + o_act);
+        w->h = reinterpret_cast<float*>(b + o_h);
+        w->xq = nullptr; w->xq_bytes = 0;
+        w->err = reinterpret_cast<uint32_t*>(b + o_err);
+    }
+    return at;
+}
+
+void prof_begin(const char* name, cudaStream_t s) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (!g_prof_on || (int32_t)g_prof.size() >= g_prof_cap) return;
+    ProfRec r{name, nullptr, nullptr};
+    cudaEventCreate(&r.a);
+    cudaEventCreate(&r.b);
+    cudaEventRecord(r.a, s);
+    g_prof.push_back(r);
+}
+
+void prof_end(cudaStream_t s) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (!g_prof_on || g_prof.empty()) return;
+    ProfRec& r = g_prof.back();
+    if (r.b) cudaEventRecord(r.b, s);
+}
+
+}  // namespace mq
+
+using namespace mq;
+
+extern "C" const char* mq_strerror(int status) {
+    switch (status) {
+    case MQ_OK: return "ok";
+    case MQ_EINVAL: return "invalid argument";
+    case MQ_EFORMAT: return "unknown packed format";
+    case MQ_EALIGN: return "pointer not 16-byte aligned";
+    case MQ_ESHAPE: return "inconsistent layer shape";
+    case MQ_EWORKSPACE: return "workspace missing or too small";
+    case MQ_ECUDA: return "CUDA error";
+    case MQ_EDEVICE: return "device-side check failed";
+    case MQ_ERANGE: return "size beyond supported maximum";
+    default: return "unknown status";
+    }
+}
+
+extern "C" int mq_set_path(int mode, int32_t prefill_threshold) {
+    if (mode < 0 || mode > 2) return MQ_EINVAL;
+    path_mode();
+    g_path_mode = mode;
+    if (prefill_threshold > 0) g_prefill_threshold = prefill_threshold;
+    return MQ_OK;
+}
+
+extern "C" size_t moe_quant_workspace_size(const mq_layer_cfg* cfg, int32_t n_tokens) {
+    if (check_cfg(cfg) != MQ_OK || n_tokens < 0 || n_tokens > 65536) return 0;
+    return workspace_plan(dims_of(cfg, n_tokens), nullptr, nullptr);
+}
+
+namespace {
+
+int check_common(const mq_layer_cfg* cfg, int32_t T, const void* x, const float* router_w, const float* bias,
+                 void* ws, size_t ws_bytes) {
+    const int rc = check_cfg(cfg);
+    if (rc != MQ_OK) return rc;
+    if (T < 0 || T > 65536) return MQ_ESHAPE;
+    if (T > 0 && (!x || !router_w)) return MQ_EINVAL;
+    if (T > 0 && (!aligned16(x) || !aligned16(router_w))) return MQ_EALIGN;
+    (void)bias;
+    const size_t need = workspace_plan(dims_of(cfg, T), nullptr, nullptr);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u)) return MQ_EWORKSPACE;
+    return MQ_OK;
+}
+
+int run_route(const Dims& d, const void* x, const float* router_w, const float* bias, Work& w,
+              cudaStream_t s) {
+    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, s) != cudaSuccess) return MQ_ECUDA;
+    if (launch_topk(d, w.z, bias, w.idx, w.wts, s) != cudaSuccess) return MQ_ECUDA;
+    if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, s) != cudaSuccess) return MQ_ECUDA;
+    return MQ_OK;
+}
+
+}  // namespace
+
+extern "C" int moe_quant_route(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x, const float* router_w,
+                               const float* bias, int32_t* topk_idx, float* topk_w, int32_t* offsets,
+                               int32_t* perm, int32_t* inv, void* workspace, size_t ws_bytes, void* stream) {
+    int rc = check_common(cfg, n_tokens, x, router_w, bias, workspace, ws_bytes);
+    if (rc != MQ_OK) return rc;
+    if (n_tokens > 0 && (!topk_idx || !topk_w)) return MQ_EINVAL;
+    const Dims d = dims_of(cfg, n_tokens);
+    Work w;
+    workspace_plan(d, workspace, &w);
+    w.idx = topk_idx;
+    w.wts = topk_w;
+    if (offsets) w.offsets = offsets;
+    if (perm) w.perm = perm;
+    if (inv) w.inv = inv;
+    return run_route(d, x, router_w, bias, w, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x, const float* router_w,
+                                 const float* bias, const mq_expert_table* table, const uint8_t* fmt,
+                                 float* out, int32_t* topk_idx, float* topk_w, void* workspace, size_t ws_bytes,
+                                 void* stream) {
+    int rc = check_common(cfg, n_tokens, x, router_w, bias, workspace, ws_bytes);
+    if (rc != MQ_OK) return rc;
+    if (!table || !table->experts || !fmt) return MQ_EINVAL;
+    if (cfg->has_shared && !table->shared) return MQ_EINVAL;
+    if (n_tokens > 0 && !out) return MQ_EINVAL;
+    const Dims d = dims_of(cfg, n_tokens);
+    static thread_local ExpertTab tab;
+    const int n = d.E + d.has_shared;
+    for (int e = 0; e < n; ++e) {
+        const mq_expert_weights& ew = e < d.E ? table->experts[e] : *table->shared;
+        const void* ps[3] = {ew.gate, ew.up, ew.down};
+        for (int j = 0; j < 3; ++j) {
+            if (!valid_format(fmt[3 * e + j])) return MQ_EFORMAT;
+            if (!ps[j]) return MQ_EINVAL;
+            if (!aligned16(ps[j])) return MQ_EALIGN;
+            tab.p[e][j] = static_cast<const uint8_t*>(ps[j]);
+            tab.fmt[e][j] = fmt[3 * e + j];
+        }
+    }
+    if (n_tokens == 0) return MQ_OK;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Work w;
+    workspace_plan(d, workspace, &w);
+    if (topk_idx) w.idx = topk_idx;
+    if (topk_w) w.wts = topk_w;
+    rc = run_route(d, x, router_w, bias, w, s);
+    if (rc != MQ_OK) return rc;
+    (void)path_mode();
+    if (launch_decode_ffn(d, tab, static_cast<const uint16_t*>(x), w, out, s) != cudaSuccess) return MQ_ECUDA;
+    return MQ_OK;
+}
+
+extern "C" int mq_unpack_device(int fmt, const void* src, int64_t rows, int64_t cols, float* dst, void* stream) {
+    if (!valid_format(fmt)) return MQ_EFORMAT;
+    if (rows < 0 || cols < 0) return MQ_EINVAL;
+    if (rows * cols == 0) return MQ_OK;
+    if (!src || !dst) return MQ_EINVAL;
+    if (!aligned16(src)) return MQ_EALIGN;
+    if (launch_unpack(fmt, static_cast<const uint8_t*>(src), rows, cols, dst, static_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
+        return MQ_ECUDA;
+    return MQ_OK;
+}
+
+extern "C" int mq_profile_enable(int32_t max_launches) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (max_launches < 0) return MQ_EINVAL;
+    for (auto& r : g_prof) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
+    g_prof.clear();
+    g_prof.reserve((size_t)max_launches);
+    g_prof_cap = max_launches;
+    g_prof_on = max_launches > 0;
+    return MQ_OK;
+}
+
+extern "C" int mq_profile_collect(mq_kernel_stat* out, int32_t max) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    std::vector<mq_kernel_stat> agg;
+    for (auto& r : g_prof) {
+        cudaEventSynchronize(r.b);
+        float ms = 0.0f;
+        cudaEventElapsedTime(&ms, r.a, r.b);
+        size_t i = 0;
+        for (; i < agg.size(); ++i)
+            if (std::strcmp(agg[i].name, r.name) == 0) break;
+        if (i == agg.size()) {
+            mq_kernel_stat st;
+            std::memset(&st, 0, sizeof(st));
+            std::strncpy(st.name, r.name, sizeof(st.name) - 1);
+            agg.push_back(st);
+        }
+        agg[i].launches += 1;
+        agg[i].total_ms += ms;
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+    }
+    g_prof.clear();
+    g_prof_on = false;
+    g_prof_cap = 0;
+    const int n = (int)agg.size() < max ? (int)agg.size() : max;
+    for (int i = 0; i < n && out; ++i) out[i] = agg[i];
+    return n;
+}

@@ -1,0 +1,55 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mq_layout.h"
+
+namespace mq {
+
+// Device pointers and formats of every expert of a layer, passed to kernels
+// by value (kernel parameter space) so a forward needs no host->device copy
+// and can be captured in a CUDA graph.  Index kMaxExperts... is not used:
+// the shared expert sits at index E (n_experts).
+struct ExpertTab {
+    const uint8_t* p[kMaxExperts + 1][3];
+    uint8_t fmt[kMaxExperts + 1][3];
+};
+
+struct Dims {
+    int H, I, E, G, Gk, K, T;
+    int has_shared;
+    float routed_scale;
+};
+
+// Carved out of the caller's workspace (see workspace_plan).
+struct Work {
+    float* z;          // [T, E] router logits
+    int32_t* idx;      // [T, K]
+    float* wts;        // [T, K]
+    int32_t* offsets;  // [E + 1]
+    int32_t* perm;     // [T*K]
+    int32_t* inv;      // [T*K]
+    int32_t* active;   // [E + 2]: active[0] = count, active[1..] = expert ids
+    float* h;          // [T*K + T, I] SwiGLU activations (fp32)
+    uint32_t* xq;      // per-token prepared activations (decode kernels)
+    size_t xq_bytes;
+    uint32_t* err;     // device error word
+};
+
+size_t workspace_plan(const Dims& d, void* base, Work* w);
+
+// launch helpers; each returns cudaGetLastError() of its launch
+cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, cudaStream_t s);
+cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
+cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
+                           int32_t* active, cudaStream_t s);
+cudaError_t launch_decode_ffn(const Dims& d, const ExpertTab& tab, const uint16_t* x, const Work& w,
+                              float* out, cudaStream_t s);
+cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);
+
+// kernel timing hooks (no-ops unless profiling is enabled)
+void prof_begin(const char* name, cudaStream_t s);
+void prof_end(cudaStream_t s);
+
+}  // namespace mq

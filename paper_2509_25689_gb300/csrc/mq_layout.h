@@ -1,0 +1,158 @@
+// Packed-format geometry shared by the library's host codec and kernels.
+// The block formats are the k-quant style types the compressed experts are
+// stored in (arXiv 2509.25689 Sec. 3.3, Sec. 4.1); the byte layout is this
+// library's own (documented in include/moeq.h).
+#pragma once
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __CUDACC__
+#define MQ_HD __host__ __device__ __forceinline__
+#else
+#define MQ_HD inline
+#endif
+
+namespace mq {
+
+enum Format : int { kQ2K = 1, kQ3K = 2, kQ4K = 3, kQ80 = 4 };
+
+constexpr int kPlaneAlign = 256;
+constexpr int kMaxExperts = 256;     // routed experts per layer
+constexpr int kMaxTopK = 32;
+constexpr int kMaxGroups = 64;
+
+MQ_HD bool valid_format(int f) { return f >= kQ2K && f <= kQ80; }
+
+// weights per block along the contraction axis
+MQ_HD int block_len(int f) { return f == kQ80 ? 32 : 256; }
+
+// bytes per block of each plane, planes in storage order
+struct PlaneBytes { int n; int b[4]; };
+MQ_HD PlaneBytes plane_bytes(int f) {
+    PlaneBytes p{0, {0, 0, 0, 0}};
+    if (f == kQ4K) { p.n = 4; p.b[0] = 2; p.b[1] = 2; p.b[2] = 12; p.b[3] = 128; }
+    else if (f == kQ2K) { p.n = 4; p.b[0] = 2; p.b[1] = 2; p.b[2] = 16; p.b[3] = 64; }
+    else if (f == kQ3K) { p.n = 4; p.b[0] = 2; p.b[1] = 12; p.b[2] = 64; p.b[3] = 32; }
+    else if (f == kQ80) { p.n = 2; p.b[0] = 2; p.b[1] = 32; }
+    return p;
+}
+
+MQ_HD int64_t pad_plane(int64_t v) { return (v + kPlaneAlign - 1) / kPlaneAlign * kPlaneAlign; }
+
+// Where each plane of a [rows x cols] tensor starts, and the total size.
+struct TensorLayout {
+    int64_t blocks_per_row;
+    int64_t plane[4];
+    int64_t total;
+};
+
+MQ_HD TensorLayout tensor_layout(int f, int64_t rows, int64_t cols) {
+    TensorLayout t{};
+    const int qk = block_len(f);
+    t.blocks_per_row = (cols + qk - 1) / qk;
+    const int64_t nblk = rows * t.blocks_per_row;
+    const PlaneBytes pb = plane_bytes(f);
+    int64_t at = 0;
+    for (int p = 0; p < pb.n; ++p) { t.plane[p] = at; at += pad_plane(nblk * pb.b[p]); }
+    for (int p = pb.n; p < 4; ++p) t.plane[p] = at;
+    t.total = at;
+    return t;
+}
+
+// ---- positions inside a block --------------------------------------------
+// k = 16 i + 8 h + 2 t + e; returns word index and bit offset of the code.
+struct CodePos { int word; int bit; };
+
+MQ_HD CodePos pos2(int k) {   // 2-bit codes
+    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
+    return CodePos{4 * t + (i >> 2), 16 * e + 2 * (2 * (i & 3) + h)};
+}
+MQ_HD CodePos pos1(int k) {   // Q3_K high-bit plane
+    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
+    return CodePos{2 * t + (i >> 3), 16 * e + 2 * (i & 7) + h};
+}
+MQ_HD CodePos pos4(int k) {   // 4-bit codes
+    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
+    return CodePos{8 * t + (i >> 1), 16 * e + 4 * (2 * (i & 1) + h)};
+}
+MQ_HD CodePos pos8(int k) {   // Q8_0 codes, k < 32
+    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
+    return CodePos{2 * t + i, 16 * e + 8 * h};
+}
+
+// slot of sub-block j (< 16) in the Q2_K / Q3_K scale fields
+MQ_HD int q16_slot(int j) { return 4 * ((j & 7) >> 1) + 2 * (j >> 3) + (j & 1); }
+
+MQ_HD uint32_t load_le32(const uint8_t* p) {
+    return (uint32_t)p[0] | ((uint32_t)p[1] << 8) | ((uint32_t)p[2] << 16) | ((uint32_t)p[3] << 24);
+}
+MQ_HD uint16_t load_le16(const uint8_t* p) { return (uint16_t)(p[0] | (p[1] << 8)); }
+
+// Q3_K stored 6-bit scale of sub-block j
+MQ_HD int q3_scale_field(const uint8_t* s, int j) {
+    const int u = q16_slot(j);
+    const int lo = (s[u >> 1] >> ((u & 1) * 4)) & 15;
+    const int hi = (s[8 + (u >> 2)] >> ((u & 3) * 2)) & 3;
+    return lo | (hi << 4);
+}
+
+// Q4_K 6-bit sub-scale and sub-min of sub-block j (< 8)
+MQ_HD void q4_fields(const uint8_t* s, int j, int& sc, int& m) {
+    const uint32_t high = load_le32(s + 8) >> (4 * j);
+    sc = (s[j] & 15) | (int)((high & 3u) << 4);
+    m = (s[j] >> 4) | (int)(((high >> 2) & 3u) << 4);
+}
+
+// exact fp16 -> fp32 (library's own conversion)
+MQ_HD float half_bits_to_float(uint16_t h) {
+    const uint32_t s = (uint32_t)(h >> 15) << 31;
+    const uint32_t ex = (h >> 10) & 31u, mt = h & 1023u;
+    uint32_t bits;
+    if (ex == 31u) bits = s | 0x7f800000u | (mt << 13);
+    else if (ex != 0u) bits = s | ((ex + 112u) << 23) | (mt << 13);
+    else {
+        // subnormal / zero: mt * 2^-24 (exact)
+        float v = (float)mt * 5.9604644775390625e-08f;
+        return s ? -v : v;
+    }
+    union { uint32_t u; float f; } c; c.u = bits; return c.f;
+}
+
+// Scalar dequantization of weight (row r, column c) of a packed tensor.
+// Slow reference-style access used by the device unpack kernel.
+MQ_HD float dequant_at(int f, const uint8_t* base, const TensorLayout& L, int64_t r, int64_t c) {
+    const int qk = block_len(f);
+    const int64_t blk = r * L.blocks_per_row + c / qk;
+    const int k = (int)(c % qk);
+    if (f == kQ80) {
+        const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
+        const CodePos p = pos8(k);
+        const int q = (int)(int8_t)(uint8_t)(load_le32(base + L.plane[1] + 32 * blk + 4 * p.word) >> p.bit);
+        return d * (float)q;
+    }
+    if (f == kQ3K) {
+        const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
+        const int s = q3_scale_field(base + L.plane[1] + 12 * blk, k >> 4);
+        const CodePos pl = pos2(k), ph = pos1(k);
+        const int lo = (int)((load_le32(base + L.plane[2] + 64 * blk + 4 * pl.word) >> pl.bit) & 3u);
+        const int hi = (int)((load_le32(base + L.plane[3] + 32 * blk + 4 * ph.word) >> ph.bit) & 1u);
+        return (d * (float)(s - 32)) * (float)((lo | (hi << 2)) - 4);
+    }
+    const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
+    const float dm = half_bits_to_float(load_le16(base + L.plane[1] + 2 * blk));
+    int sc, m, q;
+    if (f == kQ4K) {
+        q4_fields(base + L.plane[2] + 12 * blk, k >> 5, sc, m);
+        const CodePos p = pos4(k);
+        q = (int)((load_le32(base + L.plane[3] + 128 * blk + 4 * p.word) >> p.bit) & 15u);
+    } else {
+        const uint8_t b = base[L.plane[2] + 16 * blk + q16_slot(k >> 4)];
+        sc = b & 15; m = b >> 4;
+        const CodePos p = pos2(k);
+        q = (int)((load_le32(base + L.plane[3] + 64 * blk + 4 * p.word) >> p.bit) & 3u);
+    }
+    // (d*sc)*q is exact; the subtraction is the only rounding (FMA-invariant)
+    return (d * (float)sc) * (float)q - dm * (float)m;
+}
+
+}  // namespace mq

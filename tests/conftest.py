@@ -18,3 +18,9 @@ def orc():
     import oracle
     oracle.build()
     return oracle
+
+
+def pytest_sessionstart(session):
+    # compile the library and the oracle before any test module imports them
+    import __graft_entry__
+    __graft_entry__.build()

@@ -1,0 +1,109 @@
+"""CPU tests of the C ABI: the library loads and exports every symbol that
+include/moeq.h declares, the host codec is byte-identical to the oracle's
+quantizer/dequantizer, and argument checks reject bad calls before any GPU
+work (no GPU needed for any of these)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def mq():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2509_25689_gb300 as m
+    return m
+
+
+def _declared_functions():
+    with open(os.path.join(ROOT, "include", "moeq.h")) as f:
+        src = f.read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*([a-z_][a-z0-9_]*)\s*\(", src, flags=re.M)
+    return sorted(set(n for n in names if n.startswith(("mq_", "moe_"))))
+
+
+def test_library_exports_every_declared_symbol(mq):
+    names = _declared_functions()
+    assert len(names) >= 11
+    lib = ctypes.CDLL(mq.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+        assert n in mq.EXPORTED, n
+
+
+@pytest.mark.parametrize("fmt", ["Q2_K", "Q3_K", "Q4_K", "Q8_0"])
+@pytest.mark.parametrize("shape", [(1, 32), (3, 256), (5, 300), (16, 1024), (7, 2051)])
+def test_host_pack_unpack_match_oracle(mq, orc, fmt, shape):
+    rng = np.random.default_rng(hash((fmt, shape)) % 2**32)
+    w = rng.normal(0, 0.02, shape).astype(np.float32)
+    w[:, :3] *= 40.0   # a few outliers per row
+    a, b = mq.mq_pack(fmt, w), orc.pack(fmt, w)
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(mq.mq_unpack(fmt, a, *shape), orc.unpack(fmt, b, *shape))
+    assert mq.mq_packed_size(fmt, *shape) == orc.packed_size(fmt, *shape)
+
+
+@pytest.mark.parametrize("fmt", [1, 2, 3, 4])
+def test_host_unpack_random_planes_match_oracle(mq, orc, fmt):
+    from workloads.synth import random_packed, rng_for
+    p = random_packed(fmt, 9, 768, rng_for(fmt))
+    np.testing.assert_array_equal(mq.mq_unpack(fmt, p, 9, 768), orc.unpack(fmt, p, 9, 768))
+
+
+def test_bad_format_and_sizes(mq):
+    assert mq.mq_packed_size(7, 4, 256) == 0
+    assert mq.mq_packed_size(1, -1, 256) == 0
+    with pytest.raises(mq.MoeqError):
+        mq.mq_pack(9, np.zeros((1, 32), np.float32))
+    with pytest.raises(mq.MoeqError):
+        mq.mq_pack("Q8_0", np.full((1, 32), np.inf, np.float32))
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("hidden", 100, -4), ("inter", 0, -4), ("n_experts", 300, -4), ("n_groups", 5, -4),
+    ("topk_group", 9, -4), ("top_k", 33, -4), ("top_k", 0, -4),
+])
+def test_shape_checks_reject_before_launch(mq, field, value, code):
+    cfg = mq.make_cfg(7168, 2048, 192, 8, 4, 8, has_shared=True)
+    setattr(cfg, field, value)
+    assert mq.moe_quant_workspace_size(cfg, 1) == 0
+    table = mq.ExpertTable([(16, 16, 16)] * 192, shared=(16, 16, 16))
+    rc = mq._lib.moe_quant_forward(ctypes.byref(cfg), 1, 16, 16, None, ctypes.byref(table.table),
+                                   np.full(193 * 3, 1, np.uint8).ctypes.data, 16, None, None, 256, 1 << 30, None)
+    assert rc == code
+
+
+def test_topk_exceeding_kept_groups_is_rejected(mq):
+    cfg = mq.make_cfg(7168, 2048, 192, 8, 1, 25)   # 1 group of 24 cannot supply 25
+    assert mq.moe_quant_workspace_size(cfg, 1) == 0
+
+
+def test_pointer_and_workspace_checks(mq):
+    cfg = mq.make_cfg(256, 128, 8, 1, 1, 2)
+    ws = mq.moe_quant_workspace_size(cfg, 4)
+    assert ws > 0 and ws % 256 == 0
+    fmt = np.full(24, 3, np.uint8)
+    ok = mq.ExpertTable([(256, 256, 256)] * 8)
+    f = lambda x=256, rw=256, table=ok, fm=fmt, out=256, wsp=256, wsb=ws: mq._lib.moe_quant_forward(
+        ctypes.byref(cfg), 4, x, rw, None, ctypes.byref(table.table), fm.ctypes.data, out, None, None, wsp, wsb, None)
+    assert f(x=0) == -1                         # null activations
+    assert f(x=8) == -3                         # misaligned activations
+    assert f(wsb=ws - 1) == -5                  # workspace too small
+    assert f(wsp=128) == -5                     # workspace not 256-byte aligned
+    assert f(table=mq.ExpertTable([(256, 256, 8)] * 8)) == -3   # misaligned packed tensor
+    assert f(table=mq.ExpertTable([(256, 0, 256)] * 8)) == -1   # null packed tensor
+    bad = fmt.copy(); bad[5] = 9
+    assert f(fm=bad) == -2                      # unknown format
+    cfg.has_shared = 1
+    assert f(wsb=mq.moe_quant_workspace_size(cfg, 4)) == -1     # shared expert missing
+
+
+def test_strerror(mq):
+    assert mq.mq_strerror(0) == "ok"
+    assert "workspace" in mq.mq_strerror(-5)

@@ -1,0 +1,156 @@
+"""GPU parity: the CUDA path through the C ABI vs the oracle on the same
+seeded inputs.  Bit-exact for unpacked weights, expert ids, routing weights
+and the permutation; max |err| <= 2e-3 * max|y| for the layer output."""
+import numpy as np
+import pytest
+
+from tests.gpu_helpers import DeviceLayer, assert_close, mq_lib, tokens
+from workloads import get_config
+from workloads.configs import LayerSpec
+from workloads.synth import random_packed, rng_for
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch_cuda():
+    import torch
+    assert torch.cuda.is_available()
+    return torch
+
+
+# ---------------------------------------------------------------- unpack ---
+@pytest.mark.parametrize("fmt", [1, 2, 3, 4])
+@pytest.mark.parametrize("shape", [(16, 256), (33, 300), (128, 7168), (7168, 2048)])
+def test_unpack_device_bit_exact(torch_cuda, orc, fmt, shape):
+    mq = mq_lib()
+    rows, cols = shape
+    p = random_packed(fmt, rows, cols, rng_for(fmt * 31 + rows))
+    dev = torch_cuda.from_numpy(p).cuda()
+    out = torch_cuda.empty((rows, cols), dtype=torch_cuda.float32, device="cuda")
+    mq.mq_unpack_device(fmt, dev, rows, cols, out)
+    got = out.cpu().numpy()
+    ref = orc.unpack(fmt, p, rows, cols)
+    np.testing.assert_array_equal(got.view(np.uint32), ref.view(np.uint32))
+
+
+# --------------------------------------------------------------- routing ---
+def _route(torch, layer: DeviceLayer, x_bits):
+    mq = mq_lib()
+    T, K, E = x_bits.shape[0], layer.spec.top_k, layer.spec.n_experts
+    x = torch.from_numpy(np.ascontiguousarray(x_bits).view(np.int16)).cuda()
+    idx = torch.full((T, K), -1, dtype=torch.int32, device="cuda")
+    w = torch.zeros((T, K), dtype=torch.float32, device="cuda")
+    off = torch.zeros(E + 1, dtype=torch.int32, device="cuda")
+    perm = torch.zeros(max(T * K, 1), dtype=torch.int32, device="cuda")
+    inv = torch.zeros(max(T * K, 1), dtype=torch.int32, device="cuda")
+    wsb = mq.moe_quant_workspace_size(layer.cfg, T)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    mq.moe_quant_route(layer.cfg, T, x, layer.router_w, layer.bias, idx, w, off, perm, inv, ws, wsb)
+    torch.cuda.synchronize()
+    return idx.cpu().numpy(), w.cpu().numpy(), off.cpu().numpy(), perm.cpu().numpy()[:T * K], inv.cpu().numpy()[:T * K]
+
+
+class _RouterOnly:
+    """Router inputs of a config without allocating expert tensors."""
+
+    def __init__(self, spec, seed):
+        import torch
+        from workloads.synth import draw_router
+        mq = mq_lib()
+        self.spec = spec
+        rw, b = draw_router(spec, seed)
+        self.router_w_host, self.bias_host = rw, b
+        self.router_w, self.bias = torch.from_numpy(rw).cuda(), torch.from_numpy(b).cuda()
+        self.cfg = mq.make_cfg(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
+                               spec.top_k, spec.routed_scale, spec.has_shared)
+
+
+@pytest.mark.parametrize("name,T", [("tiny", 4), ("tiny", 1), ("v3_decode_t1", 1), ("v3_decode_t1", 7),
+                                    ("v3_decode_t32_mixed", 32), ("v3_prefill_t2048_zipf", 2048)])
+def test_routing_bit_exact(torch_cuda, orc, name, T):
+    spec = get_config(name)
+    lay = _RouterOnly(spec, 0)
+    x = tokens(spec, 0, T)
+    idx, w, off, perm, inv = _route(torch_cuda, lay, x)
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group, spec.top_k,
+                           spec.routed_scale, spec.has_shared)
+    ridx, rw, _, _ = orc.route(layer, x, lay.router_w_host, lay.bias_host)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    roff, rperm, rinv = orc.permute(ridx, spec.n_experts)
+    np.testing.assert_array_equal(off, roff)
+    np.testing.assert_array_equal(perm, rperm)
+    np.testing.assert_array_equal(inv, rinv)
+
+
+def test_routing_tie_break_on_device(torch_cuda, orc):
+    """All-zero activations tie every expert; lowest ids must win."""
+    spec = LayerSpec(name="ties", hidden=256, inter=128, n_experts=32, n_groups=4, topk_group=2, top_k=5,
+                     tokens=3, has_shared=False, router_std=0.1, bias_std=0.0)
+    lay = _RouterOnly(spec, 1)
+    x = np.zeros((3, 256), np.uint16)
+    idx, w, *_ = _route(torch_cuda, lay, x)
+    assert (idx == np.arange(5)).all()
+    assert (w == np.float32(0.2)).all()
+
+
+# --------------------------------------------------------------- forward ---
+def test_forward_tiny_layer(torch_cuda, orc):
+    spec = get_config("tiny")
+    layer = DeviceLayer(spec, 0, orc=orc)
+    x = tokens(spec, 0)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    assert_close(y, ry)
+
+
+@pytest.mark.parametrize("T", [1, 3, 5, 9])
+def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T):
+    spec = LayerSpec(name="small_mixed", hidden=512, inter=256, n_experts=12, n_groups=4, topk_group=2,
+                     top_k=3, tokens=T, has_shared=True, mixed=True, router_std=1 / 22.6, bias_std=0.01)
+    fm = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
+    layer = DeviceLayer(spec, T, fmts=fm)
+    x = tokens(spec, T)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
+
+
+def test_forward_v3_decode_t1(torch_cuda, orc):
+    spec = get_config("v3_decode_t1")
+    layer = DeviceLayer(spec, 0)
+    x = tokens(spec, 0)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x, idx_hint=idx)
+    np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
+
+
+def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc):
+    spec = get_config("v3_decode_t32_mixed")
+    layer = DeviceLayer(spec, 0)
+    x = tokens(spec, 0)
+    y, idx, w = layer.forward(x)
+    for t in (0, 13, 31):
+        ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
+        np.testing.assert_array_equal(idx[t:t + 1], ridx)
+        assert_close(y[t:t + 1], ry)
+
+
+def test_forward_zero_tokens_is_noop(torch_cuda):
+    import torch
+    mq = mq_lib()
+    spec = get_config("tiny")
+    layer = DeviceLayer(spec, 0)
+    out = torch.full((1, spec.hidden), 7.0, device="cuda")
+    wsb = mq.moe_quant_workspace_size(layer.cfg, 0)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device="cuda")
+    x = torch.zeros((1, spec.hidden), dtype=torch.int16, device="cuda")
+    mq.moe_quant_forward(layer.cfg, 0, x, layer.router_w, layer.bias, layer.table, layer.fmts, out,
+                         workspace=ws, ws_bytes=wsb)
+    torch.cuda.synchronize()
+    assert (out == 7.0).all()
