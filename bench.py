@@ -111,7 +111,7 @@ def step_bytes(spec, fmts, idx_steps):
         b_dn = sum(dn(e) for e in touched) + (dn(sh) if sh is not None else 0) + (T * K + T) * I * 4 + T * H * 4
         b_rt = E * H * 4 + T * H * 2 + T * E * 4
         quant = sum(gu(e) + dn(e) for e in touched) + ((gu(sh) + dn(sh)) if sh is not None else 0)
-        out.append({"gateup": b_gu, "down": b_dn, "router_logits": b_rt, "quantized": quant,
+        out.append({"gateup_mma": b_gu, "down_mma": b_dn, "router_logits": b_rt, "quantized": quant,
                     "total": b_gu + b_dn + b_rt})
     return out
 

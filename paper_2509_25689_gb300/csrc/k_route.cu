@@ -17,6 +17,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "mq_actprep.cuh"
 #include "mq_internal.h"
 
 namespace mq {
@@ -34,7 +35,8 @@ constexpr int kTok = 8;
 
 __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
                                                              const float* __restrict__ W, int H, int T,
-                                                             int E, float* __restrict__ z) {
+                                                             int E, float* __restrict__ z,
+                                                             __half* __restrict__ xq, float* __restrict__ xs) {
     __shared__ float part[32][kTok];
     const int e = blockIdx.x, t0 = blockIdx.y * kTok;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -80,6 +82,22 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
             float r = part[0][threadIdx.x];
             for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
             z[(size_t)t * E + e] = r;
+        }
+    }
+    // The CTAs of expert 0 also prepare the tokens' activations for the
+    // expert-FFN kernels: warp `seg` covers 32-element blocks 32*seg.., the
+    // blocks past the hidden size (up to the 256 padding) are zero.
+    if (e == 0 && xq != nullptr) {
+        const int nsb = (H + 255) / 256;
+        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)stat_off(nsb).total;
+        for (int j = 0; j < kTok; ++j) {
+            const int t = t0 + j;
+            if (t >= T) break;
+            for (int jb = 32 * seg; jb < 32 * seg + 32 && jb < 8 * nsb; ++jb) {
+                const int k = 32 * jb + lane;
+                const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
+                prep_block32(v, jb, 0xF, xq + (size_t)t * qstride, xs + (size_t)t * sstride, nsb);
+            }
         }
     }
 }
@@ -285,12 +303,13 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int32_t* __
 
 }  // namespace
 
-cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, cudaStream_t s) {
+cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
+                                 cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
     dim3 grid(d.E, (d.T + kTok - 1) / kTok);
     prof_begin("router_logits", s);
-    router_logits_kernel<<<grid, nseg * 32, 0, s>>>(x, W, d.H, d.T, d.E, z);
+    router_logits_kernel<<<grid, nseg * 32, 0, s>>>(x, W, d.H, d.T, d.E, z, xq, xs);
     prof_end(s);
     return cudaGetLastError();
 }

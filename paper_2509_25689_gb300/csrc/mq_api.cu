@@ -10,6 +10,7 @@
 #include <vector>
 
 #include "../../include/moeq.h"
+#include "mq_actprep.cuh"
 #include "mq_internal.h"
 
 namespace mq {
@@ -64,6 +65,8 @@ std::vector<ProfRec> g_prof;
 
 size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t TK = (size_t)d.T * d.K;
+    const size_t A = TK + (size_t)d.T;             // routed assignments + shared-expert rows
+    const size_t nsbx = (size_t)(d.H + 255) / 256, nsbi = (size_t)(d.I + 255) / 256;
     size_t at = 0;
     auto take = [&](size_t bytes) { const size_t o = at; at += up256(bytes); return o; };
     const size_t o_z = take((size_t)d.T * d.E * 4);
@@ -71,7 +74,14 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_off = take((size_t)(d.E + 1) * 4);
     const size_t o_perm = take(TK * 4), o_inv = take(TK * 4);
     const size_t o_act = take((size_t)(d.E + 2) * 4);
-    const size_t o_h = take((TK + (size_t)d.T) * d.I * 4);
+    const size_t o_xq = take((size_t)d.T * 4 * nsbx * 256 * 2);
+    const size_t o_xs = take((size_t)d.T * stat_off((int)nsbx).total * 4);
+    const size_t o_hq = take(A * 4 * nsbi * 256 * 2);
+    const size_t o_hs = take(A * stat_off((int)nsbi).total * 4);
+    const size_t o_pgu = take(A * 2 * 4 * d.I * 4);
+    const size_t o_pdn = take(A * d.H * 4);
+    const size_t cnt_bytes = decode_counter_bytes(d);
+    const size_t o_cnt = take(cnt_bytes);
     const size_t o_err = take(4);
     if (w && base) {
         char* b = static_cast<char*>(base);
@@ -82,8 +92,14 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->perm = reinterpret_cast<int32_t*>(b + o_perm);
         w->inv = reinterpret_cast<int32_t*>(b + o_inv);
         w->active = reinterpret_cast<int32_t*>(b + o_act);
-        w->h = reinterpret_cast<float*>(b + o_h);
-        w->xq = nullptr; w->xq_bytes = 0;
+        w->xq = reinterpret_cast<__half*>(b + o_xq);
+        w->xs = reinterpret_cast<float*>(b + o_xs);
+        w->hq = reinterpret_cast<__half*>(b + o_hq);
+        w->hs = reinterpret_cast<float*>(b + o_hs);
+        w->pgu = reinterpret_cast<float*>(b + o_pgu);
+        w->pdn = reinterpret_cast<float*>(b + o_pdn);
+        w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
+        w->counter_bytes = cnt_bytes;
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
     }
     return at;
@@ -154,8 +170,10 @@ int check_common(const mq_layer_cfg* cfg, int32_t T, const void* x, const float*
 }
 
 int run_route(const Dims& d, const void* x, const float* router_w, const float* bias, Work& w,
-              cudaStream_t s) {
-    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, s) != cudaSuccess) return MQ_ECUDA;
+              cudaStream_t s, bool prep_tokens) {
+    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, prep_tokens ? w.xq : nullptr, w.xs,
+                             s) != cudaSuccess)
+        return MQ_ECUDA;
     if (launch_topk(d, w.z, bias, w.idx, w.wts, s) != cudaSuccess) return MQ_ECUDA;
     if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, s) != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
@@ -177,7 +195,7 @@ extern "C" int moe_quant_route(const mq_layer_cfg* cfg, int32_t n_tokens, const 
     if (offsets) w.offsets = offsets;
     if (perm) w.perm = perm;
     if (inv) w.inv = inv;
-    return run_route(d, x, router_w, bias, w, static_cast<cudaStream_t>(stream));
+    return run_route(d, x, router_w, bias, w, static_cast<cudaStream_t>(stream), false);
 }
 
 extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x, const float* router_w,
@@ -209,10 +227,11 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     workspace_plan(d, workspace, &w);
     if (topk_idx) w.idx = topk_idx;
     if (topk_w) w.wts = topk_w;
-    rc = run_route(d, x, router_w, bias, w, s);
+    if (cudaMemsetAsync(w.counters, 0, w.counter_bytes, s) != cudaSuccess) return MQ_ECUDA;
+    rc = run_route(d, x, router_w, bias, w, s, true);
     if (rc != MQ_OK) return rc;
     (void)path_mode();
-    if (launch_decode_ffn(d, tab, static_cast<const uint16_t*>(x), w, out, s) != cudaSuccess) return MQ_ECUDA;
+    if (launch_decode_mma(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
 }
 

@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cuda_fp16.h>
+
 #include "mq_layout.h"
 
 namespace mq {
@@ -31,21 +33,28 @@ struct Work {
     int32_t* perm;     // [T*K]
     int32_t* inv;      // [T*K]
     int32_t* active;   // [E + 2]: active[0] = count, active[1..] = expert ids
-    float* h;          // [T*K + T, I] SwiGLU activations (fp32)
-    uint32_t* xq;      // per-token prepared activations (decode kernels)
-    size_t xq_bytes;
+    __half* xq;        // [T][4][nsb(H)*256] prepared token activations (fp16 fragments)
+    float* xs;         // [T][80*nsb(H)] their statistics
+    __half* hq;        // [A][4][nsb(I)*256] prepared SwiGLU outputs, A = T*K + T
+    float* hs;         // [A][80*nsb(I)]
+    float* pgu;        // [A][2][4][I] gate/up split-K partials
+    float* pdn;        // [A][H] down partials
+    uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
+    size_t counter_bytes;
     uint32_t* err;     // device error word
 };
 
 size_t workspace_plan(const Dims& d, void* base, Work* w);
 
 // launch helpers; each returns cudaGetLastError() of its launch
-cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, cudaStream_t s);
+cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
+                                 cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, cudaStream_t s);
-cudaError_t launch_decode_ffn(const Dims& d, const ExpertTab& tab, const uint16_t* x, const Work& w,
-                              float* out, cudaStream_t s);
+cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
+size_t decode_scratch_bytes(const Dims& d);
+size_t decode_counter_bytes(const Dims& d);
 cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);
 
 // kernel timing hooks (no-ops unless profiling is enabled)
