@@ -11,10 +11,13 @@
  *    block formats Q2_K/Q3_K/Q4_K and Q8; Sec. 4.1 implementation details).
  *    The paper gives no byte layout, so the layout below is this project's
  *    own "-style" definition: every format blocks along the contraction
- *    (column) axis, rows are padded to whole blocks with zero weights, and
- *    each field lives in its own plane (row-major over (row, block), each
- *    plane 256-byte aligned).  Code bits are placed in "fragment order"
- *    (see code_pos_*), sub-block scale fields in "slot order" (slot_of).
+ *    (column) axis, rows are padded to whole blocks with zero weights and
+ *    to whole tiles of 32 rows with zero rows, and each field lives in its
+ *    own 256-byte aligned plane.  A plane lists, for each 32-row tile and
+ *    each block, the field's record of the 32 rows (records longer than 64
+ *    bytes are cut in 64-byte units, unit-major; see unit_at).  Code bits
+ *    are placed in "fragment order" (see code_pos_*), sub-block scale
+ *    fields in "slot order" (slot_of).
  *      PINNED by hand-built blocks (tests/golden/hand_blocks.json), by
  *      single-bit placement tests, by grid blocks that must re-pack to
  *      themselves, and by nearest-grid-point brute force on random blocks.
@@ -95,31 +98,47 @@ static float bf16_to_float(uint16_t b) { return bits_to_f32((uint32_t)b << 16); 
 typedef struct {
     int qk;                 /* weights per block along the contraction axis */
     int nplanes;
-    int bytes[MAX_PLANES];  /* bytes per block in each plane */
+    int bytes[MAX_PLANES];  /* bytes per (row, block) record in each plane */
+    int unit[MAX_PLANES];   /* records are stored in units of this many bytes */
 } geom;
 
 static int get_geom(int fmt, geom* g) {
     memset(g, 0, sizeof(*g));
     switch (fmt) {
     case ORC_Q4_K: g->qk = 256; g->nplanes = 4;
-        g->bytes[0] = 2; g->bytes[1] = 2; g->bytes[2] = 12; g->bytes[3] = 128; return 0;
+        g->bytes[0] = 2; g->bytes[1] = 2; g->bytes[2] = 12; g->bytes[3] = 128;
+        g->unit[0] = 2; g->unit[1] = 2; g->unit[2] = 12; g->unit[3] = 64; return 0;
     case ORC_Q2_K: g->qk = 256; g->nplanes = 4;
-        g->bytes[0] = 2; g->bytes[1] = 2; g->bytes[2] = 16; g->bytes[3] = 64; return 0;
+        g->bytes[0] = 2; g->bytes[1] = 2; g->bytes[2] = 16; g->bytes[3] = 64;
+        g->unit[0] = 2; g->unit[1] = 2; g->unit[2] = 16; g->unit[3] = 64; return 0;
     case ORC_Q3_K: g->qk = 256; g->nplanes = 4;
-        g->bytes[0] = 2; g->bytes[1] = 12; g->bytes[2] = 64; g->bytes[3] = 32; return 0;
+        g->bytes[0] = 2; g->bytes[1] = 12; g->bytes[2] = 64; g->bytes[3] = 32;
+        g->unit[0] = 2; g->unit[1] = 12; g->unit[2] = 64; g->unit[3] = 32; return 0;
     case ORC_Q8_0: g->qk = 32; g->nplanes = 2;
-        g->bytes[0] = 2; g->bytes[1] = 32; return 0;
+        g->bytes[0] = 2; g->bytes[1] = 32;
+        g->unit[0] = 2; g->unit[1] = 32; return 0;
     default: return -1;
     }
 }
 
+#define ROW_TILE 32
+
 static int64_t round_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
 
-/* plane base offsets for a tensor with nblk blocks in total */
+/* plane base offsets for a tensor with nblk (row, block) records in total,
+   rows counted after padding to whole 32-row tiles */
 static void plane_offsets(const geom* g, int64_t nblk, int64_t off[MAX_PLANES + 1]) {
     off[0] = 0;
     for (int p = 0; p < g->nplanes; p++)
         off[p + 1] = off[p] + round_up(nblk * g->bytes[p], PLANE_ALIGN);
+}
+
+/* Byte offset, inside plane p, of unit u of the record (row r, block b):
+   records are grouped in tiles of 32 rows; a plane lists, for each tile,
+   each block, each unit of the record, the 32 rows of the tile. */
+static int64_t unit_at(const geom* g, int p, int64_t nb, int64_t r, int64_t b, int u) {
+    int64_t nu = g->bytes[p] / g->unit[p];
+    return ((((r / ROW_TILE) * nb + b) * nu + u) * ROW_TILE + r % ROW_TILE) * g->unit[p];
 }
 
 size_t oracle_packed_size(int fmt, int64_t rows, int64_t cols) {
@@ -127,7 +146,7 @@ size_t oracle_packed_size(int fmt, int64_t rows, int64_t cols) {
     if (get_geom(fmt, &g) || rows < 0 || cols < 0) return 0;
     int64_t nb = (cols + g.qk - 1) / g.qk;
     int64_t off[MAX_PLANES + 1];
-    plane_offsets(&g, rows * nb, off);
+    plane_offsets(&g, round_up(rows, ROW_TILE) * nb, off);
     return (size_t)off[g.nplanes];
 }
 
@@ -159,10 +178,11 @@ static void code_pos_1bit(int k, int* word, int* bit) {
     *bit = 16 * e + (2 * (i & 7) + h);
 }
 
-/* 4-bit codes (Q4_K): 32 words/block */
+/* 4-bit codes (Q4_K): 32 words/block, stored as two 64-byte units
+   (unit = i / 8) */
 static void code_pos_4bit(int k, int* word, int* bit) {
     int i, t, h, e; split_k(k, &i, &t, &h, &e);
-    *word = 8 * t + (i >> 1);
+    *word = 16 * (i >> 3) + 4 * t + ((i & 7) >> 1);
     *bit = 16 * e + 4 * (2 * (i & 1) + h);
 }
 
@@ -273,33 +293,33 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
     for (int64_t i = 0; i < rows * cols; i++)
         if (!isfinite(w[i])) return -2;
     memset(dst, 0, need);
-    int64_t nb = (cols + g.qk - 1) / g.qk, nblk = rows * nb;
+    int64_t nb = (cols + g.qk - 1) / g.qk, prow = round_up(rows, ROW_TILE);
     int64_t off[MAX_PLANES + 1];
-    plane_offsets(&g, nblk, off);
+    plane_offsets(&g, prow * nb, off);
     float wb[256];
     int q[256], sc[16], m[16];
-    for (int64_t r = 0; r < rows; r++) {
+    uint8_t rec[MAX_PLANES][128];
+    /* padding rows (up to a whole tile) are quantized zero rows */
+    for (int64_t r = 0; r < prow; r++) {
         for (int64_t b = 0; b < nb; b++) {
-            int64_t blk = r * nb + b;
             for (int k = 0; k < g.qk; k++) {
                 int64_t c = b * g.qk + k;
-                wb[k] = c < cols ? w[r * cols + c] : 0.0f;
+                wb[k] = (r < rows && c < cols) ? w[r * cols + c] : 0.0f;
             }
+            memset(rec, 0, sizeof(rec));
             if (fmt == ORC_Q4_K || fmt == ORC_Q2_K) {
                 int is4 = fmt == ORC_Q4_K;
                 uint16_t dh, mh;
                 quant_asym(wb, is4 ? 8 : 16, is4 ? 32 : 16, is4 ? 15 : 3, is4 ? 63 : 15,
                            &dh, &mh, sc, m, q);
-                wr16(dst + off[0] + 2 * blk, dh);
-                wr16(dst + off[1] + 2 * blk, mh);
-                uint8_t* s = dst + off[2] + (int64_t)g.bytes[2] * blk;
-                uint8_t* cp = dst + off[3] + (int64_t)g.bytes[3] * blk;
+                wr16(rec[0], dh);
+                wr16(rec[1], mh);
                 if (is4) {
-                    for (int j = 0; j < 8; j++) q4_put(s, j, sc[j], m[j]);
-                    for (int k = 0; k < 256; k++) { int wd, bt; code_pos_4bit(k, &wd, &bt); put_field(cp, wd, bt, 4, (uint32_t)q[k]); }
+                    for (int j = 0; j < 8; j++) q4_put(rec[2], j, sc[j], m[j]);
+                    for (int k = 0; k < 256; k++) { int wd, bt; code_pos_4bit(k, &wd, &bt); put_field(rec[3], wd, bt, 4, (uint32_t)q[k]); }
                 } else {
-                    for (int j = 0; j < 16; j++) s[slot_of(j)] = (uint8_t)(sc[j] | (m[j] << 4));
-                    for (int k = 0; k < 256; k++) { int wd, bt; code_pos_2bit(k, &wd, &bt); put_field(cp, wd, bt, 2, (uint32_t)q[k]); }
+                    for (int j = 0; j < 16; j++) rec[2][slot_of(j)] = (uint8_t)(sc[j] | (m[j] << 4));
+                    for (int k = 0; k < 256; k++) { int wd, bt; code_pos_2bit(k, &wd, &bt); put_field(rec[3], wd, bt, 2, (uint32_t)q[k]); }
                 }
             } else if (fmt == ORC_Q3_K) {
                 float scale[16], maxabs = 0.0f;
@@ -312,21 +332,18 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
                 }
                 uint16_t dh = float_to_half(maxabs / 31.0f);
                 float df = half_to_float(dh);
-                wr16(dst + off[0] + 2 * blk, dh);
-                uint8_t* s = dst + off[1] + 12 * blk;
-                uint8_t* lo = dst + off[2] + 64 * blk;
-                uint8_t* hi = dst + off[3] + 32 * blk;
+                wr16(rec[0], dh);
                 for (int j = 0; j < 16; j++) {
                     int scj = df > 0.0f ? clampi(rn(scale[j] / df), -32, 31) : 0;
-                    q3_put_scale(s, j, scj + 32);
+                    q3_put_scale(rec[1], j, scj + 32);
                     float den = df * (float)scj;
                     for (int i = 0; i < 16; i++) {
                         int k = 16 * j + i;
                         int qi = den != 0.0f ? clampi(rn(wb[k] / den), -4, 3) : 0;
                         int code = qi + 4;
                         int wd, bt;
-                        code_pos_2bit(k, &wd, &bt); put_field(lo, wd, bt, 2, (uint32_t)(code & 3));
-                        code_pos_1bit(k, &wd, &bt); put_field(hi, wd, bt, 1, (uint32_t)(code >> 2));
+                        code_pos_2bit(k, &wd, &bt); put_field(rec[2], wd, bt, 2, (uint32_t)(code & 3));
+                        code_pos_1bit(k, &wd, &bt); put_field(rec[3], wd, bt, 1, (uint32_t)(code >> 2));
                     }
                 }
             } else { /* Q8_0 */
@@ -334,14 +351,16 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
                 for (int k = 0; k < 32; k++) if (fabsf(wb[k]) > amax) amax = fabsf(wb[k]);
                 uint16_t dh = float_to_half(amax / 127.0f);
                 float df = half_to_float(dh);
-                wr16(dst + off[0] + 2 * blk, dh);
-                uint8_t* cp = dst + off[1] + 32 * blk;
+                wr16(rec[0], dh);
                 for (int k = 0; k < 32; k++) {
                     int qi = df > 0.0f ? clampi(rn(wb[k] / df), -127, 127) : 0;
                     int wd, bt; code_pos_8bit(k, &wd, &bt);
-                    put_field(cp, wd, bt, 8, (uint32_t)(qi & 0xff));
+                    put_field(rec[1], wd, bt, 8, (uint32_t)(qi & 0xff));
                 }
             }
+            for (int p = 0; p < g.nplanes; p++)
+                for (int u = 0; u < g.bytes[p] / g.unit[p]; u++)
+                    memcpy(dst + off[p] + unit_at(&g, p, nb, r, b, u), rec[p] + u * g.unit[p], (size_t)g.unit[p]);
         }
     }
     return 0;
@@ -354,45 +373,49 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
 int oracle_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst) {
     geom g;
     if (get_geom(fmt, &g) || !src || !dst || rows < 0 || cols < 0) return -1;
-    int64_t nb = (cols + g.qk - 1) / g.qk, nblk = rows * nb;
+    int64_t nb = (cols + g.qk - 1) / g.qk, prow = round_up(rows, ROW_TILE);
     int64_t off[MAX_PLANES + 1];
-    plane_offsets(&g, nblk, off);
+    plane_offsets(&g, prow * nb, off);
+    uint8_t rec[MAX_PLANES][128];
     for (int64_t r = 0; r < rows; r++) {
         for (int64_t b = 0; b < nb; b++) {
-            int64_t blk = r * nb + b;
+            /* gather the record of (row r, block b) from its units */
+            for (int p = 0; p < g.nplanes; p++)
+                for (int u = 0; u < g.bytes[p] / g.unit[p]; u++)
+                    memcpy(rec[p] + u * g.unit[p], src + off[p] + unit_at(&g, p, nb, r, b, u), (size_t)g.unit[p]);
             for (int k = 0; k < g.qk; k++) {
                 int64_t c = b * g.qk + k;
                 if (c >= cols) break;
                 float v;
                 int wd, bt;
                 if (fmt == ORC_Q4_K) {
-                    float df = half_to_float(rd16(src + off[0] + 2 * blk));
-                    float mf = half_to_float(rd16(src + off[1] + 2 * blk));
-                    int sc, m; q4_get(src + off[2] + 12 * blk, k / 32, &sc, &m);
+                    float df = half_to_float(rd16(rec[0]));
+                    float mf = half_to_float(rd16(rec[1]));
+                    int sc, m; q4_get(rec[2], k / 32, &sc, &m);
                     code_pos_4bit(k, &wd, &bt);
-                    int q = (int)get_field(src + off[3] + 128 * blk, wd, bt, 4);
+                    int q = (int)get_field(rec[3], wd, bt, 4);
                     v = (df * (float)sc) * (float)q - mf * (float)m;
                 } else if (fmt == ORC_Q2_K) {
-                    float df = half_to_float(rd16(src + off[0] + 2 * blk));
-                    float mf = half_to_float(rd16(src + off[1] + 2 * blk));
-                    uint8_t s = src[off[2] + 16 * blk + slot_of(k / 16)];
+                    float df = half_to_float(rd16(rec[0]));
+                    float mf = half_to_float(rd16(rec[1]));
+                    uint8_t s = rec[2][slot_of(k / 16)];
                     int sc = s & 15, m = s >> 4;
                     code_pos_2bit(k, &wd, &bt);
-                    int q = (int)get_field(src + off[3] + 64 * blk, wd, bt, 2);
+                    int q = (int)get_field(rec[3], wd, bt, 2);
                     v = (df * (float)sc) * (float)q - mf * (float)m;
                 } else if (fmt == ORC_Q3_K) {
-                    float df = half_to_float(rd16(src + off[0] + 2 * blk));
-                    int s = q3_get_scale(src + off[1] + 12 * blk, k / 16);
+                    float df = half_to_float(rd16(rec[0]));
+                    int s = q3_get_scale(rec[1], k / 16);
                     code_pos_2bit(k, &wd, &bt);
-                    int lo = (int)get_field(src + off[2] + 64 * blk, wd, bt, 2);
+                    int lo = (int)get_field(rec[2], wd, bt, 2);
                     code_pos_1bit(k, &wd, &bt);
-                    int hi = (int)get_field(src + off[3] + 32 * blk, wd, bt, 1);
+                    int hi = (int)get_field(rec[3], wd, bt, 1);
                     int q = lo | (hi << 2);
                     v = (df * (float)(s - 32)) * (float)(q - 4);
                 } else {
-                    float df = half_to_float(rd16(src + off[0] + 2 * blk));
+                    float df = half_to_float(rd16(rec[0]));
                     code_pos_8bit(k, &wd, &bt);
-                    int q = (int)(int8_t)(uint8_t)get_field(src + off[1] + 32 * blk, wd, bt, 8);
+                    int q = (int)(int8_t)(uint8_t)get_field(rec[1], wd, bt, 8);
                     v = df * (float)q;
                 }
                 dst[r * cols + c] = v;
