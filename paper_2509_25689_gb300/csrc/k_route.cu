@@ -84,16 +84,17 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
             z[(size_t)t * E + e] = r;
         }
     }
-    // The CTAs of expert 0 also prepare the tokens' activations for the
-    // expert-FFN kernels: warp `seg` covers 32-element blocks 32*seg.., the
-    // blocks past the hidden size (up to the 256 padding) are zero.
-    if (e == 0 && xq != nullptr) {
+    // The CTAs also prepare the tokens' activations for the expert-FFN
+    // kernels, spread over all of them: warp `seg` of the CTA of expert e
+    // takes the 32-element blocks 32*seg + e, 32*seg + e + E, ... of its
+    // segment (blocks past the hidden size, up to the 256 padding, are zero).
+    if (xq != nullptr) {
         const int nsb = (H + 255) / 256;
         const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)stat_off(nsb).total;
         for (int j = 0; j < kTok; ++j) {
             const int t = t0 + j;
             if (t >= T) break;
-            for (int jb = 32 * seg; jb < 32 * seg + 32 && jb < 8 * nsb; ++jb) {
+            for (int jb = 32 * seg + e; jb < 32 * seg + 32 && jb < 8 * nsb; jb += E) {
                 const int k = 32 * jb + lane;
                 const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
                 prep_block32(v, jb, 0xF, xq + (size_t)t * qstride, xs + (size_t)t * sstride, nsb);
@@ -141,65 +142,92 @@ __device__ __forceinline__ int warp_argmax(float v, int i) {
     return i;
 }
 
+// One warp routes one token.  Lane l holds experts l, l+32, ... (E <= 256).
+// uw: per-warp scratch of E floats; g_sh: per-warp scratch of G floats.
+__device__ __forceinline__ void route_token(const float* __restrict__ z, const float* __restrict__ bias, const Dims& d,
+                                            int t, float* uw, float* g_sh, int32_t* __restrict__ idx,
+                                            float* __restrict__ wts) {
+    const int lane = threadIdx.x & 31;
+    const int E = d.E, G = d.G, gs = E / G;
+    float s[8], u[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        const int e = lane + 32 * m;
+        s[m] = 0.0f; u[m] = -INFINITY;
+        if (e < E) {
+            s[m] = canonical_sigmoid(z[(size_t)t * E + e]);
+            u[m] = __fadd_rn(s[m], bias ? bias[e] : 0.0f);
+        }
+    }
+    // group score = sum of the two largest u of the group (scan in index order)
+#pragma unroll
+    for (int m = 0; m < 8; ++m) if (lane + 32 * m < E) uw[lane + 32 * m] = u[m];
+    __syncwarp();
+    for (int g = lane; g < G; g += 32) {
+        float top1 = -INFINITY, top2 = -INFINITY;
+        for (int i = 0; i < gs; ++i) {
+            const float v = uw[g * gs + i];
+            if (v > top1) { top2 = top1; top1 = v; }
+            else if (v > top2) top2 = v;
+        }
+        g_sh[g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
+    }
+    __syncwarp();
+    // keep topk_group groups: repeated argmax, ties to the lower index
+    uint64_t kept = 0;
+    float gv0 = lane < G ? g_sh[lane] : 0.0f, gv1 = lane + 32 < G ? g_sh[lane + 32] : 0.0f;
+    for (int r = 0; r < d.Gk; ++r) {
+        float bv = 0.0f; int bi = -1;
+        if (lane < G && !((kept >> lane) & 1)) better(bv, bi, gv0, lane);
+        if (lane + 32 < G && !((kept >> (lane + 32)) & 1)) better(bv, bi, gv1, lane + 32);
+        bi = warp_argmax(bv, bi);
+        kept |= 1ull << bi;
+    }
+    // top_k experts by u among the kept groups, descending, ties to the lower id
+    uint32_t avail = 0;
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        const int e = lane + 32 * m;
+        if (e < E && ((kept >> (e / gs)) & 1)) avail |= 1u << m;
+    }
+    int sel = 0;
+    float ssum = 0.0f, mys = 0.0f;
+    for (int j = 0; j < d.K; ++j) {
+        float bv = 0.0f; int bi = -1;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) if ((avail >> m) & 1) better(bv, bi, u[m], lane + 32 * m);
+        bi = warp_argmax(bv, bi);
+        float win = 0.0f;
+        if ((bi & 31) == lane) {
+            const int m = bi >> 5;
+            avail &= ~(1u << m);
+            win = s[0];
+#pragma unroll
+            for (int mm = 1; mm < 8; ++mm) if (mm == m) win = s[mm];
+        }
+        const float sv = __shfl_sync(kFull, win, bi & 31);
+        ssum = __fadd_rn(ssum, sv);   // slot order, identical on every lane
+        if (lane == j) { sel = bi; mys = sv; }   // lane j keeps slot j
+    }
+    // weights: s_j / sum(s), summed in slot order, times routed_scale
+    if (lane < d.K) {
+        idx[(size_t)t * d.K + lane] = sel;
+        wts[(size_t)t * d.K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), d.routed_scale);
+    }
+}
+
 constexpr int kTopkWarps = 4;
 
 __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __restrict__ z,
                                                                const float* __restrict__ bias, Dims d,
                                                                int32_t* __restrict__ idx,
                                                                float* __restrict__ wts) {
-    __shared__ float s_sh[kTopkWarps][kMaxExperts];
     __shared__ float u_sh[kTopkWarps][kMaxExperts];
     __shared__ float g_sh[kTopkWarps][kMaxGroups];
-    __shared__ uint8_t keep_g[kTopkWarps][kMaxGroups];
-    __shared__ uint8_t taken[kTopkWarps][kMaxExperts];
-    __shared__ int32_t sel[kTopkWarps][kMaxTopK];
-    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int w = threadIdx.x >> 5;
     const int t = blockIdx.x * kTopkWarps + w;
     if (t >= d.T) return;
-    const int E = d.E, G = d.G, gs = E / G;
-    for (int e = lane; e < E; e += 32) {
-        const float s = canonical_sigmoid(z[(size_t)t * E + e]);
-        s_sh[w][e] = s;
-        u_sh[w][e] = __fadd_rn(s, bias ? bias[e] : 0.0f);
-        taken[w][e] = 0;
-    }
-    __syncwarp();
-    for (int g = lane; g < G; g += 32) {
-        float top1 = -INFINITY, top2 = -INFINITY;
-        for (int i = 0; i < gs; ++i) {
-            const float v = u_sh[w][g * gs + i];
-            if (v > top1) { top2 = top1; top1 = v; }
-            else if (v > top2) top2 = v;
-        }
-        g_sh[w][g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
-        keep_g[w][g] = 0;
-    }
-    __syncwarp();
-    for (int r = 0; r < d.Gk; ++r) {
-        float bv = 0.0f; int bi = -1;
-        for (int g = lane; g < G; g += 32)
-            if (!keep_g[w][g]) better(bv, bi, g_sh[w][g], g);
-        bi = warp_argmax(bv, bi);
-        if (lane == 0) keep_g[w][bi] = 1;
-        __syncwarp();
-    }
-    for (int j = 0; j < d.K; ++j) {
-        float bv = 0.0f; int bi = -1;
-        for (int e = lane; e < E; e += 32)
-            if (keep_g[w][e / gs] && !taken[w][e]) better(bv, bi, u_sh[w][e], e);
-        bi = warp_argmax(bv, bi);
-        if (lane == 0) { taken[w][bi] = 1; sel[w][j] = bi; }
-        __syncwarp();
-    }
-    if (lane == 0) {
-        float sum = 0.0f;
-        for (int j = 0; j < d.K; ++j) sum = __fadd_rn(sum, s_sh[w][sel[w][j]]);
-        for (int j = 0; j < d.K; ++j) {
-            const int e = sel[w][j];
-            idx[(size_t)t * d.K + j] = e;
-            wts[(size_t)t * d.K + j] = __fmul_rn(__fdiv_rn(s_sh[w][e], sum), d.routed_scale);
-        }
-    }
+    route_token(z, bias, d, t, u_sh[w], g_sh[w], idx, wts);
 }
 
 // ---------------------------------------------------------------------------
@@ -208,14 +236,27 @@ __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __re
 constexpr int kPermThreads = 1024;
 constexpr int kPermWarps = kPermThreads / 32;
 
-__global__ void __launch_bounds__(kPermThreads) permute_kernel(const int32_t* __restrict__ idx, int n, int E,
+// With `z` given, the same CTA first routes every token (one warp per token,
+// decode-sized batches) and then permutes.
+__global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restrict__ idx, Dims d,
                                                                int32_t* __restrict__ offsets,
                                                                int32_t* __restrict__ perm,
                                                                int32_t* __restrict__ inv,
-                                                               int32_t* __restrict__ active) {
+                                                               int32_t* __restrict__ active,
+                                                               Plan* __restrict__ plan,
+                                                               const float* __restrict__ z,
+                                                               const float* __restrict__ bias,
+                                                               float* __restrict__ wts) {
+    const int n = d.T * d.K, E = d.E;
     __shared__ int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
     __shared__ int32_t total[kMaxExperts + 1];
+    __shared__ float g_sh[kPermWarps][kMaxGroups];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (z != nullptr) {
+        for (int t = warp; t < d.T; t += kPermWarps)
+            route_token(z, bias, d, t, reinterpret_cast<float*>(cnt[warp]), g_sh[warp], idx, wts);
+        __syncthreads();
+    }
     for (int i = threadIdx.x; i < kPermWarps * kMaxExperts; i += kPermThreads) (&cnt[0][0])[i] = 0;
     __syncthreads();
     const int seg = (n + kPermWarps - 1) / kPermWarps;
@@ -299,6 +340,49 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int32_t* __
             if (flags & (1 << q)) active[1 + pos++] = lane * 8 + q;
         if (lane == 31) active[0] = incl;
     }
+    if (plan == nullptr) return;
+    __syncthreads();
+    // decode work plan: items per expert slot (shared expert first)
+    if (warp == 0) {
+        const int n_slots = active[0] + d.has_shared;
+        int cg[9], cd[9], sg = 0, sd = 0, tgs = 0, tgmax = 0;
+#pragma unroll
+        for (int q = 0; q < 9; ++q) {
+            const int p = lane * 9 + q;
+            int ntok = 0;
+            if (p < n_slots) {
+                if (p < d.has_shared) ntok = d.T;
+                else { const int e = active[1 + p - d.has_shared]; ntok = offsets[e + 1] - offsets[e]; }
+            }
+            const int ntg = (ntok + kDecodeTok - 1) / kDecodeTok;
+            cg[q] = (d.I / 32) * ntg;     // gate/up items: 32 rows x both tensors x full K
+            cd[q] = (d.H / 32) * ntg;     // down items: 32 rows x full K
+            sg += cg[q]; sd += cd[q]; tgs += ntg; tgmax = max(tgmax, ntg);
+        }
+        int ig = sg, id = sd;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int vg = __shfl_up_sync(kFull, ig, off), vd = __shfl_up_sync(kFull, id, off);
+            if (lane >= off) { ig += vg; id += vd; }
+        }
+        int rg = ig - sg, rd = id - sd;
+#pragma unroll
+        for (int q = 0; q < 9; ++q) {
+            const int p = lane * 9 + q;
+            if (p <= kMaxExperts + 1) { plan->pre_gu[p] = rg; plan->pre_dn[p] = rd; }
+            rg += cg[q]; rd += cd[q];
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) {
+            tgs += __shfl_xor_sync(kFull, tgs, off);
+            tgmax = max(tgmax, __shfl_xor_sync(kFull, tgmax, off));
+        }
+        if (lane == 0) {
+            plan->n_slots = n_slots;
+            plan->dn_target = tgs;
+            plan->ntg_max = tgmax;
+        }
+    }
 }
 
 }  // namespace
@@ -324,9 +408,19 @@ cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_
 }
 
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
-                           int32_t* active, cudaStream_t s) {
+                           int32_t* active, Plan* plan, cudaStream_t s) {
     prof_begin("permute", s);
-    permute_kernel<<<1, kPermThreads, 0, s>>>(idx, d.T * d.K, d.E, offsets, perm, inv, active);
+    permute_kernel<<<1, kPermThreads, 0, s>>>(const_cast<int32_t*>(idx), d, offsets, perm, inv, active, plan,
+                                               nullptr, nullptr, nullptr);
+    prof_end(s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
+                                 int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
+                                 cudaStream_t s) {
+    prof_begin("route_permute", s);
+    permute_kernel<<<1, kPermThreads, 0, s>>>(idx, d, offsets, perm, inv, active, plan, z, bias, wts);
     prof_end(s);
     return cudaGetLastError();
 }

@@ -18,6 +18,8 @@ namespace {
 
 size_t up256(size_t v) { return (v + 255) & ~size_t(255); }
 
+constexpr int32_t kFusedRouteTokens = 256;   // up to this many tokens: one routing CTA
+
 int g_path_mode = -1;        // -1: not yet read from the environment
 int32_t g_prefill_threshold = 64;
 
@@ -78,8 +80,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_xs = take((size_t)d.T * stat_off((int)nsbx).total * 4);
     const size_t o_hq = take(A * 4 * nsbi * 256 * 2);
     const size_t o_hs = take(A * stat_off((int)nsbi).total * 4);
-    const size_t o_pgu = take(A * 2 * 4 * d.I * 4);
     const size_t o_pdn = take(A * d.H * 4);
+    const size_t o_plan = take(sizeof(Plan));
     const size_t cnt_bytes = decode_counter_bytes(d);
     const size_t o_cnt = take(cnt_bytes);
     const size_t o_err = take(4);
@@ -96,8 +98,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->xs = reinterpret_cast<float*>(b + o_xs);
         w->hq = reinterpret_cast<__half*>(b + o_hq);
         w->hs = reinterpret_cast<float*>(b + o_hs);
-        w->pgu = reinterpret_cast<float*>(b + o_pgu);
         w->pdn = reinterpret_cast<float*>(b + o_pdn);
+        w->plan = reinterpret_cast<Plan*>(b + o_plan);
         w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
         w->counter_bytes = cnt_bytes;
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
@@ -174,8 +176,16 @@ int run_route(const Dims& d, const void* x, const float* router_w, const float* 
     if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, prep_tokens ? w.xq : nullptr, w.xs,
                              s) != cudaSuccess)
         return MQ_ECUDA;
+    if (d.T <= kFusedRouteTokens) {
+        // decode-sized batch: top-k, permutation and work plan in one CTA
+        if (launch_route_permute(d, w.z, bias, w.idx, w.wts, w.offsets, w.perm, w.inv, w.active,
+                                 prep_tokens ? w.plan : nullptr, s) != cudaSuccess)
+            return MQ_ECUDA;
+        return MQ_OK;
+    }
     if (launch_topk(d, w.z, bias, w.idx, w.wts, s) != cudaSuccess) return MQ_ECUDA;
-    if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, s) != cudaSuccess) return MQ_ECUDA;
+    if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, prep_tokens ? w.plan : nullptr, s) != cudaSuccess)
+        return MQ_ECUDA;
     return MQ_OK;
 }
 
@@ -228,6 +238,7 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     if (topk_idx) w.idx = topk_idx;
     if (topk_w) w.wts = topk_w;
     if (cudaMemsetAsync(w.counters, 0, w.counter_bytes, s) != cudaSuccess) return MQ_ECUDA;
+    if (cudaMemsetAsync(w.err, 0, 4, s) != cudaSuccess) return MQ_ECUDA;
     rc = run_route(d, x, router_w, bias, w, s, true);
     if (rc != MQ_OK) return rc;
     (void)path_mode();

@@ -161,16 +161,23 @@ extern "C" int mq_pack(int fmt, const float* w, int64_t rows, int64_t cols, void
     const int qk = block_len(fmt);
     const PlaneBytes pb = plane_bytes(fmt);
     std::vector<float> blk(qk);
-    for (int64_t r = 0; r < rows; ++r) {
+    uint8_t rec[4][128];
+    // rows past `rows` (up to the 32-row tile) are encoded as zero rows
+    for (int64_t r = 0; r < pad_rows(rows); ++r) {
         for (int64_t b = 0; b < L.blocks_per_row; ++b) {
             for (int k = 0; k < qk; ++k) {
                 const int64_t c = b * qk + k;
-                blk[k] = c < cols ? w[r * cols + c] : 0.0f;
+                blk[k] = (r < rows && c < cols) ? w[r * cols + c] : 0.0f;
             }
-            const int64_t id = r * L.blocks_per_row + b;
-            uint8_t* planes[4] = {nullptr, nullptr, nullptr, nullptr};
-            for (int p = 0; p < pb.n; ++p) planes[p] = out + L.plane[p] + id * pb.b[p];
+            std::memset(rec, 0, sizeof(rec));
+            uint8_t* planes[4] = {rec[0], rec[1], rec[2], rec[3]};
             encode_block(fmt, blk.data(), planes);
+            for (int p = 0; p < pb.n; ++p) {
+                const int ub = unit_bytes(pb.b[p]);
+                for (int u = 0; u < pb.b[p] / ub; ++u)
+                    std::memcpy(out + L.plane[p] + unit_offset(L.blocks_per_row, pb.b[p], r, b, u), rec[p] + u * ub,
+                                (size_t)ub);
+            }
         }
     }
     return MQ_OK;

@@ -24,6 +24,21 @@ struct Dims {
     float routed_scale;
 };
 
+// Decode work plan: the expert-FFN kernels cut work into items of 32 rows x
+// full K x up to kDecodeTok tokens (gate/up items cover both tensors).  The
+// permutation kernel counts items per expert slot (shared expert first, then
+// the active routed experts in id order) so the kernels can map an item id to
+// its slot.
+constexpr int kDecodeTok = 4;
+struct Plan {
+    int32_t n_slots;
+    int32_t dn_target;            // token groups summed over slots
+    int32_t ntg_max;              // token groups of the largest slot
+    int32_t pad;
+    int32_t pre_gu[kMaxExperts + 2];
+    int32_t pre_dn[kMaxExperts + 2];
+};
+
 // Carved out of the caller's workspace (see workspace_plan).
 struct Work {
     float* z;          // [T, E] router logits
@@ -33,15 +48,15 @@ struct Work {
     int32_t* perm;     // [T*K]
     int32_t* inv;      // [T*K]
     int32_t* active;   // [E + 2]: active[0] = count, active[1..] = expert ids
+    Plan* plan;        // decode work plan
     __half* xq;        // [T][4][nsb(H)*256] prepared token activations (fp16 fragments)
     float* xs;         // [T][80*nsb(H)] their statistics
     __half* hq;        // [A][4][nsb(I)*256] prepared SwiGLU outputs, A = T*K + T
     float* hs;         // [A][80*nsb(I)]
-    float* pgu;        // [A][2][4][I] gate/up split-K partials
-    float* pdn;        // [A][H] down partials
+    float* pdn;        // [A][H] down outputs per assignment (combined by a last pass)
     uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
     size_t counter_bytes;
-    uint32_t* err;     // device error word
+    uint32_t* err;     // device error word (bounded waits that ran out)
 };
 
 size_t workspace_plan(const Dims& d, void* base, Work* w);
@@ -51,9 +66,11 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
                                  cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
-                           int32_t* active, cudaStream_t s);
+                           int32_t* active, Plan* plan, cudaStream_t s);
+cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
+                                 int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
+                                 cudaStream_t s);
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
-size_t decode_scratch_bytes(const Dims& d);
 size_t decode_counter_bytes(const Dims& d);
 cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);
 

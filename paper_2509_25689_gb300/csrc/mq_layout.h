@@ -17,6 +17,7 @@ namespace mq {
 enum Format : int { kQ2K = 1, kQ3K = 2, kQ4K = 3, kQ80 = 4 };
 
 constexpr int kPlaneAlign = 256;
+constexpr int kRowTile = 32;         // records are grouped in tiles of 32 rows
 constexpr int kMaxExperts = 256;     // routed experts per layer
 constexpr int kMaxTopK = 32;
 constexpr int kMaxGroups = 64;
@@ -26,7 +27,8 @@ MQ_HD bool valid_format(int f) { return f >= kQ2K && f <= kQ80; }
 // weights per block along the contraction axis
 MQ_HD int block_len(int f) { return f == kQ80 ? 32 : 256; }
 
-// bytes per block of each plane, planes in storage order
+// bytes per (row, block) record of each plane, planes in storage order; a
+// record is stored in units of at most 64 bytes (only Q4_K codes have 2)
 struct PlaneBytes { int n; int b[4]; };
 MQ_HD PlaneBytes plane_bytes(int f) {
     PlaneBytes p{0, {0, 0, 0, 0}};
@@ -36,21 +38,33 @@ MQ_HD PlaneBytes plane_bytes(int f) {
     else if (f == kQ80) { p.n = 2; p.b[0] = 2; p.b[1] = 32; }
     return p;
 }
+MQ_HD int unit_bytes(int record_bytes) { return record_bytes > 64 ? 64 : record_bytes; }
 
 MQ_HD int64_t pad_plane(int64_t v) { return (v + kPlaneAlign - 1) / kPlaneAlign * kPlaneAlign; }
 
 // Where each plane of a [rows x cols] tensor starts, and the total size.
+// Inside a plane, unit u of the record of (row r, block b) is at
+//   ((((r / 32) * blocks_per_row + b) * units + u) * 32 + r % 32) * unit_bytes
+// so any block range of a 32-row tile is one contiguous byte range.
 struct TensorLayout {
     int64_t blocks_per_row;
     int64_t plane[4];
     int64_t total;
 };
 
+MQ_HD int64_t pad_rows(int64_t rows) { return (rows + kRowTile - 1) / kRowTile * kRowTile; }
+
+// byte offset, from the plane start, of unit u of record (r, b)
+MQ_HD int64_t unit_offset(int64_t bpr, int record_bytes, int64_t r, int64_t b, int u) {
+    const int ub = unit_bytes(record_bytes), nu = record_bytes / ub;
+    return ((((r / kRowTile) * bpr + b) * nu + u) * kRowTile + r % kRowTile) * ub;
+}
+
 MQ_HD TensorLayout tensor_layout(int f, int64_t rows, int64_t cols) {
     TensorLayout t{};
     const int qk = block_len(f);
     t.blocks_per_row = (cols + qk - 1) / qk;
-    const int64_t nblk = rows * t.blocks_per_row;
+    const int64_t nblk = pad_rows(rows) * t.blocks_per_row;
     const PlaneBytes pb = plane_bytes(f);
     int64_t at = 0;
     for (int p = 0; p < pb.n; ++p) { t.plane[p] = at; at += pad_plane(nblk * pb.b[p]); }
@@ -71,9 +85,9 @@ MQ_HD CodePos pos1(int k) {   // Q3_K high-bit plane
     const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
     return CodePos{2 * t + (i >> 3), 16 * e + 2 * (i & 7) + h};
 }
-MQ_HD CodePos pos4(int k) {   // 4-bit codes
+MQ_HD CodePos pos4(int k) {   // 4-bit codes: two 64-byte units, unit = i / 8
     const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
-    return CodePos{8 * t + (i >> 1), 16 * e + 4 * (2 * (i & 1) + h)};
+    return CodePos{16 * (i >> 3) + 4 * t + ((i & 7) >> 1), 16 * e + 4 * (2 * (i & 1) + h)};
 }
 MQ_HD CodePos pos8(int k) {   // Q8_0 codes, k < 32
     const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
@@ -119,37 +133,46 @@ MQ_HD float half_bits_to_float(uint16_t h) {
 }
 
 // Scalar dequantization of weight (row r, column c) of a packed tensor.
-// Slow reference-style access used by the device unpack kernel.
+// Slow reference-style access used by the device unpack kernel and the host
+// codec.
+MQ_HD uint32_t rec_word(const uint8_t* plane, const TensorLayout& L, int rb, int64_t r, int64_t b, int word) {
+    const int ub = unit_bytes(rb);
+    const int u = (4 * word) / ub;
+    return load_le32(plane + unit_offset(L.blocks_per_row, rb, r, b, u) + (4 * word) % ub);
+}
+MQ_HD const uint8_t* rec_ptr(const uint8_t* plane, const TensorLayout& L, int rb, int64_t r, int64_t b) {
+    return plane + unit_offset(L.blocks_per_row, rb, r, b, 0);
+}
+
 MQ_HD float dequant_at(int f, const uint8_t* base, const TensorLayout& L, int64_t r, int64_t c) {
     const int qk = block_len(f);
-    const int64_t blk = r * L.blocks_per_row + c / qk;
+    const int64_t b = c / qk;
     const int k = (int)(c % qk);
+    const PlaneBytes pb = plane_bytes(f);
+    const float d = half_bits_to_float(load_le16(rec_ptr(base + L.plane[0], L, 2, r, b)));
     if (f == kQ80) {
-        const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
         const CodePos p = pos8(k);
-        const int q = (int)(int8_t)(uint8_t)(load_le32(base + L.plane[1] + 32 * blk + 4 * p.word) >> p.bit);
+        const int q = (int)(int8_t)(uint8_t)(rec_word(base + L.plane[1], L, 32, r, b, p.word) >> p.bit);
         return d * (float)q;
     }
     if (f == kQ3K) {
-        const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
-        const int s = q3_scale_field(base + L.plane[1] + 12 * blk, k >> 4);
+        const int s = q3_scale_field(rec_ptr(base + L.plane[1], L, 12, r, b), k >> 4);
         const CodePos pl = pos2(k), ph = pos1(k);
-        const int lo = (int)((load_le32(base + L.plane[2] + 64 * blk + 4 * pl.word) >> pl.bit) & 3u);
-        const int hi = (int)((load_le32(base + L.plane[3] + 32 * blk + 4 * ph.word) >> ph.bit) & 1u);
+        const int lo = (int)((rec_word(base + L.plane[2], L, 64, r, b, pl.word) >> pl.bit) & 3u);
+        const int hi = (int)((rec_word(base + L.plane[3], L, 32, r, b, ph.word) >> ph.bit) & 1u);
         return (d * (float)(s - 32)) * (float)((lo | (hi << 2)) - 4);
     }
-    const float d = half_bits_to_float(load_le16(base + L.plane[0] + 2 * blk));
-    const float dm = half_bits_to_float(load_le16(base + L.plane[1] + 2 * blk));
+    const float dm = half_bits_to_float(load_le16(rec_ptr(base + L.plane[1], L, 2, r, b)));
     int sc, m, q;
     if (f == kQ4K) {
-        q4_fields(base + L.plane[2] + 12 * blk, k >> 5, sc, m);
+        q4_fields(rec_ptr(base + L.plane[2], L, 12, r, b), k >> 5, sc, m);
         const CodePos p = pos4(k);
-        q = (int)((load_le32(base + L.plane[3] + 128 * blk + 4 * p.word) >> p.bit) & 15u);
+        q = (int)((rec_word(base + L.plane[3], L, pb.b[3], r, b, p.word) >> p.bit) & 15u);
     } else {
-        const uint8_t b = base[L.plane[2] + 16 * blk + q16_slot(k >> 4)];
-        sc = b & 15; m = b >> 4;
+        const uint8_t bt = rec_ptr(base + L.plane[2], L, 16, r, b)[q16_slot(k >> 4)];
+        sc = bt & 15; m = bt >> 4;
         const CodePos p = pos2(k);
-        q = (int)((load_le32(base + L.plane[3] + 64 * blk + 4 * p.word) >> p.bit) & 3u);
+        q = (int)((rec_word(base + L.plane[3], L, 64, r, b, p.word) >> p.bit) & 3u);
     }
     // (d*sc)*q is exact; the subtraction is the only rounding (FMA-invariant)
     return (d * (float)sc) * (float)q - dm * (float)m;

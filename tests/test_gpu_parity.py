@@ -67,7 +67,8 @@ class _RouterOnly:
 
 
 @pytest.mark.parametrize("name,T", [("tiny", 4), ("tiny", 1), ("v3_decode_t1", 1), ("v3_decode_t1", 7),
-                                    ("v3_decode_t32_mixed", 32), ("v3_prefill_t2048_zipf", 2048)])
+                                    ("v3_decode_t32_mixed", 32), ("v3_decode_t32_mixed", 256),
+                                    ("v3_decode_t32_mixed", 257), ("v3_prefill_t2048_zipf", 2048)])
 def test_routing_bit_exact(torch_cuda, orc, name, T):
     spec = get_config(name)
     lay = _RouterOnly(spec, 0)

@@ -23,9 +23,12 @@ PLANES = {
 PLANE_ALIGN = 256
 
 
+ROW_TILE = 32
+
+
 def packed_bytes(fmt: int, rows: int, cols: int) -> int:
     qk, planes = PLANES[fmt]
-    nblk = rows * ((cols + qk - 1) // qk)
+    nblk = (-(-rows // ROW_TILE) * ROW_TILE) * ((cols + qk - 1) // qk)
     return sum(-(-nblk * b // PLANE_ALIGN) * PLANE_ALIGN for _, b in planes)
 
 

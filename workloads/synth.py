@@ -17,7 +17,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from .configs import PLANES, PLANE_ALIGN, Q2_K, Q3_K, Q4_K, Q8_0, LayerSpec, packed_bytes
+from .configs import PLANES, PLANE_ALIGN, Q2_K, Q3_K, Q4_K, Q8_0, ROW_TILE, LayerSpec, packed_bytes
 
 # fp16 scale bases: decoded weights then have mean ~0 and std ~0.02
 FP16_BASE = {
@@ -94,7 +94,7 @@ def draw_fp32_weights(spec: LayerSpec, seed: int):
 
 def _plane_layout(fmt: int, rows: int, cols: int):
     qk, planes = PLANES[fmt]
-    nblk = rows * ((cols + qk - 1) // qk)
+    nblk = (-(-rows // ROW_TILE) * ROW_TILE) * ((cols + qk - 1) // qk)
     off = 0
     out = []
     for kind, b in planes:
