@@ -146,6 +146,31 @@ int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
                       float* out, int32_t* topk_idx, float* topk_w,
                       void* workspace, size_t ws_bytes, void* cuda_stream);
 
+/* moe_quant_forward without a workspace argument, for callers that cannot
+ * allocate device memory: plugins whose host owns every allocation, code
+ * running while a stream is being captured (cudaMalloc is not allowed
+ * there), or latency-bound loops that must not call cudaMalloc/cudaFree,
+ * which can synchronize the device.  The paper has no counterpart; it is a
+ * deployment convenience of this library.
+ *   Arguments, layouts and results are those of moe_quant_forward.
+ *   Scratch: a fixed 16 MiB device array inside this library, held on every
+ *   device that loads it until the process exits.  A call whose
+ *   moe_quant_workspace_size(cfg, n_tokens) exceeds 16 MiB returns MQ_ERANGE
+ *   and enqueues nothing (a V3-shaped layer, hidden 7168 / inter 2048 /
+ *   top-8 + shared expert, fits up to about 32 tokens).
+ *   The first call on a device looks the array's device address up
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.  It allocates nothing itself.
+ *   All calls share the one array and each call overwrites it: calls that
+ *   overlap on the GPU (different streams, or several host threads) race
+ *   and give wrong results.  Order them on one stream.
+ *   Returns the codes of moe_quant_forward, plus MQ_ERANGE as above and
+ *   MQ_ECUDA if the address lookup fails. */
+int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
+                              const float* router_w, const float* bias,
+                              const mq_expert_table* expert_table, const uint8_t* fmt_per_tensor,
+                              float* out, int32_t* topk_idx, float* topk_w, void* cuda_stream);
+
 /* Routing and permutation only (steps 1-2 of the layer):
  *   topk_idx/topk_w device [n_tokens, top_k] (required),
  *   offsets  device int32 [n_experts + 1]: exclusive prefix of per-expert counts,

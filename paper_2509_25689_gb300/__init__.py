@@ -17,6 +17,7 @@ LIB_PATH = os.path.join(_HERE, "libmoeq.so")
 MQ_Q2_K, MQ_Q3_K, MQ_Q4_K, MQ_Q8_0 = 1, 2, 3, 4
 FORMATS = {"Q2_K": MQ_Q2_K, "Q3_K": MQ_Q3_K, "Q4_K": MQ_Q4_K, "Q8_0": MQ_Q8_0}
 MQ_OK = 0
+MQ_EINVAL, MQ_EFORMAT, MQ_EALIGN, MQ_ESHAPE, MQ_EWORKSPACE, MQ_ECUDA, MQ_EDEVICE, MQ_ERANGE = range(-1, -9, -1)
 
 
 class MoeqError(RuntimeError):
@@ -60,6 +61,8 @@ def _load():
         "moe_quant_workspace_size": (sz, [cfgp, i32]),
         "moe_quant_forward": (ctypes.c_int, [cfgp, i32, vp, vp, vp, ctypes.POINTER(mq_expert_table), vp,
                                              vp, vp, vp, vp, sz, vp]),
+        "moe_quant_forward_noalloc": (ctypes.c_int, [cfgp, i32, vp, vp, vp, ctypes.POINTER(mq_expert_table), vp,
+                                                     vp, vp, vp, vp]),
         "moe_quant_route": (ctypes.c_int, [cfgp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
         "mq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "mq_set_path": (ctypes.c_int, [ctypes.c_int, i32]),
@@ -74,7 +77,7 @@ def _load():
 
 _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
-            "moe_quant_forward", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
+            "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
             "mq_profile_collect")
 
 
@@ -182,6 +185,18 @@ def moe_quant_forward(cfg, n_tokens, x, router_w, bias, expert_table: ExpertTabl
                                 ctypes.byref(expert_table.table), fmt.ctypes.data, _ptr(out), _ptr(topk_idx),
                                 _ptr(topk_w), _ptr(workspace), ws_bytes, _stream(stream))
     return _check("moe_quant_forward", rc)
+
+
+def moe_quant_forward_noalloc(cfg, n_tokens, x, router_w, bias, expert_table: ExpertTable, fmt_per_tensor, out,
+                              topk_idx=None, topk_w=None, stream=None):
+    """moe_quant_forward with the library's fixed 16 MiB device scratch instead
+    of a caller workspace (nothing is allocated)."""
+    import numpy as np
+    fmt = np.ascontiguousarray(fmt_per_tensor, dtype=np.uint8).reshape(-1)
+    rc = _lib.moe_quant_forward_noalloc(ctypes.byref(cfg), n_tokens, _ptr(x), _ptr(router_w), _ptr(bias),
+                                        ctypes.byref(expert_table.table), fmt.ctypes.data, _ptr(out),
+                                        _ptr(topk_idx), _ptr(topk_w), _stream(stream))
+    return _check("moe_quant_forward_noalloc", rc)
 
 
 def moe_quant_route(cfg, n_tokens, x, router_w, bias, topk_idx, topk_w, offsets=None, perm=None, inv=None,

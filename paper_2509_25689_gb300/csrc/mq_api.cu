@@ -246,6 +246,59 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     return MQ_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Forward pass that allocates nothing: its scratch is a fixed device array
+// owned by this library.  For callers that cannot call cudaMalloc (see
+// include/moeq.h).
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB
+constexpr int kNoAllocMaxDevices = 64;
+
+// Every device that loads this library holds this array until the process
+// exits.  Host code must not pass `g_noalloc_scratch` itself to a kernel: on
+// the host the name is only a stand-in for the device symbol, so its device
+// address is looked up once per device below.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch array on the current device (looked up on
+// the first call made with that device current).
+int noalloc_scratch(void** out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MQ_ECUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return MQ_ERANGE;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return MQ_ECUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return MQ_OK;
+}
+
+}  // namespace
+
+extern "C" int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
+                                         const float* router_w, const float* bias, const mq_expert_table* table,
+                                         const uint8_t* fmt, float* out, int32_t* topk_idx, float* topk_w,
+                                         void* stream) {
+    const int rc = check_cfg(cfg);
+    if (rc != MQ_OK) return rc;
+    if (n_tokens < 0 || n_tokens > 65536) return MQ_ESHAPE;
+    if (workspace_plan(dims_of(cfg, n_tokens), nullptr, nullptr) > kNoAllocScratchBytes) return MQ_ERANGE;
+    void* scratch = nullptr;
+    const int sr = noalloc_scratch(&scratch);
+    if (sr != MQ_OK) return sr;
+    // the forward pass clears the parts of its scratch that must start at zero
+    return moe_quant_forward(cfg, n_tokens, x, router_w, bias, table, fmt, out, topk_idx, topk_w, scratch,
+                             kNoAllocScratchBytes, stream);
+}
+
 extern "C" int mq_unpack_device(int fmt, const void* src, int64_t rows, int64_t cols, float* dst, void* stream) {
     if (!valid_format(fmt)) return MQ_EFORMAT;
     if (rows < 0 || cols < 0) return MQ_EINVAL;
