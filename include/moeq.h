@@ -28,22 +28,29 @@
  * Packed tensor format (all formats): a tensor has `rows` output rows and
  * `cols` contraction columns.  Each row is cut into blocks of QK weights
  * along the columns (QK = 256 for Q2_K/Q3_K/Q4_K, 32 for Q8_0), the last
- * block padded with zero weights.  Every field of a block lives in its own
- * plane; a plane is row-major over (row, block) and starts at an offset that
- * is a multiple of 256 bytes from the tensor base.  Planes in order:
+ * block padded with zero weights, and rows are padded with zero rows to a
+ * multiple of 32 (a tile).  Every field of a block lives in its own plane,
+ * starting at a multiple of 256 bytes from the tensor base.  A field's
+ * record (the field of one row and one block) is stored in units of at most
+ * 64 bytes (only the Q4_K codes have two units), and unit u of the record of
+ * (row r, block b) sits at byte
+ *   ((((r / 32) * nb + b) * nu + u) * 32 + r % 32) * unit_bytes
+ * of its plane (nb blocks per row, nu units per record), so any block range
+ * of a 32-row tile is one contiguous byte range of every plane.  Planes:
  *   Q4_K: d fp16 | dmin fp16 | 12 B sub-scale/min (8 x (6+6) bits) | 128 B 4-bit codes
  *         w = (d*sc)*q - dmin*m,        sub-blocks of 32
  *   Q2_K: d fp16 | dmin fp16 | 16 B (sc | m<<4) per sub-block | 64 B 2-bit codes
  *         w = (d*sc)*q - dmin*m,        sub-blocks of 16
  *   Q3_K: d fp16 | 12 B 6-bit sub-scales (stored sc+32) | 64 B low 2 bits | 32 B high bit
  *         w = (d*(s-32))*(q-4),         sub-blocks of 16
- *   Q8_0: d fp16 | 32 B int8 codes,     w = d*q
- * Inside a block, weight k = 16 i + 8 h + 2 t + e (i < QK/16, h,e < 2, t < 4).
- * Codes are little-endian 32-bit words:
- *   2-bit: word 4t + i/4,  bit 16e + 2(2(i%4) + h)
- *   1-bit: word 2t + i/8,  bit 16e + 2(i%8) + h
- *   4-bit: word 8t + i/2,  bit 16e + 4(2(i%2) + h)
- *   8-bit: word 2t + i,    bit 16e + 8h
+ *   Q8_0: d fp16 | 32 B codes stored as q+128,  w = d*q
+ * Inside a block, weight k is in sub-block j = k/n (n = 16 for 2-bit and
+ * 1-bit codes, 32 for 4-bit and 8-bit codes) at pair m = (k%n)/2, e = k%2.
+ * Codes are little-endian 32-bit words ("pair order"):
+ *   2-bit: word 4(j%4) + j/4,          bit 16e + 2m
+ *   1-bit: word 2(j%4) + j/8,          bit 16e + 8((j/4)%2) + m
+ *   4-bit: word 16(j/4) + 4(j%4) + m/4, bit 16e + 4(m%4)
+ *   8-bit: word m/2,                   bit 16e + 8(m%2)
  * Sub-block j of Q2_K/Q3_K sits in slot u = 4((j%8)/2) + 2(j/8) + j%2:
  *   Q2_K: byte u = sc | m << 4.
  *   Q3_K: bits 4u..4u+3 of bytes 0-7 (LE) = low nibble of s,

@@ -16,8 +16,9 @@
  *    own 256-byte aligned plane.  A plane lists, for each 32-row tile and
  *    each block, the field's record of the 32 rows (records longer than 64
  *    bytes are cut in 64-byte units, unit-major; see unit_at).  Code bits
- *    are placed in "fragment order" (see code_pos_*), sub-block scale
- *    fields in "slot order" (slot_of).
+ *    are placed in "pair order" (see code_pos_*: the two codes of a pair
+ *    sit 16 bits apart in one word), sub-block scale fields in "slot
+ *    order" (slot_of); Q8_0 codes are stored offset by 128.
  *      PINNED by hand-built blocks (tests/golden/hand_blocks.json), by
  *      single-bit placement tests, by grid blocks that must re-pack to
  *      themselves, and by nearest-grid-point brute force on random blocks.
@@ -153,44 +154,46 @@ size_t oracle_packed_size(int fmt, int64_t rows, int64_t cols) {
 /* ------------------------------------------------------------------ */
 /* Positions of fields inside a block                                   */
 /* ------------------------------------------------------------------ */
-/* A weight index k inside a block is split as
- *   i = k / 16  (16-wide step), r = k % 16,
- *   t = (r % 8) / 2,  h = r / 8,  e = r % 2,
- * i.e. k = 16 i + 8 h + 2 t + e.  Codes are stored in little-endian
- * 32-bit words; these functions give (word index, bit position). */
+/* Codes are stored in little-endian 32-bit words; these functions give
+ * (word index, bit position) of the code of weight k of a block.  A block
+ * is cut in sub-blocks of n weights (n = 16 for the 2-bit / 1-bit codes of
+ * Q2_K and Q3_K, 32 for Q4_K and for a Q8_0 block):
+ *   j = k / n  (sub-block),  p = k % n,  m = p / 2,  e = p % 2,
+ * so each sub-block is a sequence of code pairs m = 0, 1, ... and the two
+ * codes of a pair (e = 0, 1) always sit 16 bits apart in one word. */
 
-static void split_k(int k, int* i, int* t, int* h, int* e) {
-    int r = k & 15;
-    *i = k >> 4; *t = (r & 7) >> 1; *h = r >> 3; *e = r & 1;
-}
-
-/* 2-bit codes (Q2_K codes, low two bits of Q3_K codes): 16 words/block */
+/* 2-bit codes (Q2_K codes, low two bits of Q3_K codes): 16 words/block.
+   Word 4 (j % 4) + j / 4 holds sub-block j; pair m at bit 2 m (+16 e). */
 static void code_pos_2bit(int k, int* word, int* bit) {
-    int i, t, h, e; split_k(k, &i, &t, &h, &e);
-    *word = 4 * t + (i >> 2);
-    *bit = 16 * e + 2 * (2 * (i & 3) + h);
+    int j = k >> 4, p = k & 15, m = p >> 1, e = p & 1;
+    *word = 4 * (j & 3) + (j >> 2);
+    *bit = 16 * e + 2 * m;
 }
 
-/* 1-bit plane (high bit of Q3_K codes): 8 words/block */
+/* 1-bit plane (high bit of Q3_K codes): 8 words/block.  Word
+   2 (j % 4) + j / 8 holds sub-blocks j with equal j % 4 and j / 8; the one
+   with (j / 4) % 2 = 1 takes the upper byte of each 16-bit half. */
 static void code_pos_1bit(int k, int* word, int* bit) {
-    int i, t, h, e; split_k(k, &i, &t, &h, &e);
-    *word = 2 * t + (i >> 3);
-    *bit = 16 * e + (2 * (i & 7) + h);
+    int j = k >> 4, p = k & 15, m = p >> 1, e = p & 1;
+    *word = 2 * (j & 3) + (j >> 3);
+    *bit = 16 * e + 8 * ((j >> 2) & 1) + m;
 }
 
-/* 4-bit codes (Q4_K): 32 words/block, stored as two 64-byte units
-   (unit = i / 8) */
+/* 4-bit codes (Q4_K, 8 sub-blocks of 32): 32 words/block, stored as two
+   64-byte units (unit = j / 4).  Sub-block j takes words
+   16 (j / 4) + 4 (j % 4) + 0..3; pair m at word m / 4, bit 4 (m % 4). */
 static void code_pos_4bit(int k, int* word, int* bit) {
-    int i, t, h, e; split_k(k, &i, &t, &h, &e);
-    *word = 16 * (i >> 3) + 4 * t + ((i & 7) >> 1);
-    *bit = 16 * e + 4 * (2 * (i & 1) + h);
+    int j = k >> 5, p = k & 31, m = p >> 1, e = p & 1;
+    *word = 16 * (j >> 2) + 4 * (j & 3) + (m >> 2);
+    *bit = 16 * e + 4 * (m & 3);
 }
 
-/* 8-bit codes (Q8_0, 32-weight block): 8 words/block */
+/* 8-bit codes (Q8_0, 32-weight block): 8 words/block; pair m at word m / 2,
+   bit 8 (m % 2).  The stored byte is q + 128 (offset binary). */
 static void code_pos_8bit(int k, int* word, int* bit) {
-    int i, t, h, e; split_k(k, &i, &t, &h, &e);
-    *word = 2 * t + i;
-    *bit = 16 * e + 8 * h;
+    int m = k >> 1, e = k & 1;
+    *word = m >> 1;
+    *bit = 16 * e + 8 * (m & 1);
 }
 
 static uint32_t get_word(const uint8_t* p, int w) {
@@ -355,7 +358,7 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
                 for (int k = 0; k < 32; k++) {
                     int qi = df > 0.0f ? clampi(rn(wb[k] / df), -127, 127) : 0;
                     int wd, bt; code_pos_8bit(k, &wd, &bt);
-                    put_field(rec[1], wd, bt, 8, (uint32_t)(qi & 0xff));
+                    put_field(rec[1], wd, bt, 8, (uint32_t)(qi + 128));
                 }
             }
             for (int p = 0; p < g.nplanes; p++)
@@ -415,7 +418,7 @@ int oracle_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float
                 } else {
                     float df = half_to_float(rd16(rec[0]));
                     code_pos_8bit(k, &wd, &bt);
-                    int q = (int)(int8_t)(uint8_t)get_field(rec[1], wd, bt, 8);
+                    int q = (int)get_field(rec[1], wd, bt, 8) - 128;
                     v = df * (float)q;
                 }
                 dst[r * cols + c] = v;

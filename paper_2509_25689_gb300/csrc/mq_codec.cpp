@@ -10,7 +10,7 @@
 //   Q3_K: a = sub-block weight of largest |w| (first), scale = a / -4,
 //     d = fp16(max |scale| / 31), sc = clamp(rne(scale/d), -32, 31),
 //     q = clamp(rne(w / (d*sc)), -4, 3); stored sc+32 and q+4
-//   Q8_0: d = fp16(max|w| / 127), q = clamp(rne(w/d), -127, 127)
+//   Q8_0: d = fp16(max|w| / 127), q = clamp(rne(w/d), -127, 127), stored q+128
 // All arithmetic is IEEE fp32 (this file is built with -ffp-contract=off),
 // rne = round half to even; a zero denominator gives code 0.
 #include <cmath>
@@ -91,7 +91,7 @@ void encode_block(int f, const float* w, uint8_t* const planes[4]) {
         store16(planes[0], dh);
         for (int k = 0; k < 32; ++k) {
             const int q = d > 0.0f ? clip(rne(w[k] / d), -127, 127) : 0;
-            set_bits(planes[1], pos8(k), (uint32_t)(q & 0xff), 0xffu);
+            set_bits(planes[1], pos8(k), (uint32_t)(q + 128), 0xffu);
         }
         return;
     }

@@ -74,24 +74,27 @@ MQ_HD TensorLayout tensor_layout(int f, int64_t rows, int64_t cols) {
 }
 
 // ---- positions inside a block --------------------------------------------
-// k = 16 i + 8 h + 2 t + e; returns word index and bit offset of the code.
+// Weight k of a block lies in sub-block j = k / n (n = 16 for 2-bit and
+// 1-bit codes, 32 for 4-bit and 8-bit codes), at pair m = (k % n) / 2,
+// e = k % 2: the two codes of a pair sit 16 bits apart in one word, so one
+// masked word is an fp16x2 MMA operand register ("pair order").
 struct CodePos { int word; int bit; };
 
-MQ_HD CodePos pos2(int k) {   // 2-bit codes
-    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
-    return CodePos{4 * t + (i >> 2), 16 * e + 2 * (2 * (i & 3) + h)};
+MQ_HD CodePos pos2(int k) {   // 2-bit codes: sub-block j in word 4 (j % 4) + j / 4
+    const int j = k >> 4, m = (k & 15) >> 1, e = k & 1;
+    return CodePos{4 * (j & 3) + (j >> 2), 16 * e + 2 * m};
 }
 MQ_HD CodePos pos1(int k) {   // Q3_K high-bit plane
-    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
-    return CodePos{2 * t + (i >> 3), 16 * e + 2 * (i & 7) + h};
+    const int j = k >> 4, m = (k & 15) >> 1, e = k & 1;
+    return CodePos{2 * (j & 3) + (j >> 3), 16 * e + 8 * ((j >> 2) & 1) + m};
 }
-MQ_HD CodePos pos4(int k) {   // 4-bit codes: two 64-byte units, unit = i / 8
-    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
-    return CodePos{16 * (i >> 3) + 4 * t + ((i & 7) >> 1), 16 * e + 4 * (2 * (i & 1) + h)};
+MQ_HD CodePos pos4(int k) {   // 4-bit codes: two 64-byte units, unit = j / 4
+    const int j = k >> 5, m = (k & 31) >> 1, e = k & 1;
+    return CodePos{16 * (j >> 2) + 4 * (j & 3) + (m >> 2), 16 * e + 4 * (m & 3)};
 }
-MQ_HD CodePos pos8(int k) {   // Q8_0 codes, k < 32
-    const int i = k >> 4, h = (k >> 3) & 1, t = (k >> 1) & 3, e = k & 1;
-    return CodePos{2 * t + i, 16 * e + 8 * h};
+MQ_HD CodePos pos8(int k) {   // Q8_0 codes (stored q + 128), k < 32
+    const int m = k >> 1, e = k & 1;
+    return CodePos{m >> 1, 16 * e + 8 * (m & 1)};
 }
 
 // slot of sub-block j (< 16) in the Q2_K / Q3_K scale fields
@@ -152,7 +155,7 @@ MQ_HD float dequant_at(int f, const uint8_t* base, const TensorLayout& L, int64_
     const float d = half_bits_to_float(load_le16(rec_ptr(base + L.plane[0], L, 2, r, b)));
     if (f == kQ80) {
         const CodePos p = pos8(k);
-        const int q = (int)(int8_t)(uint8_t)(rec_word(base + L.plane[1], L, 32, r, b, p.word) >> p.bit);
+        const int q = (int)((rec_word(base + L.plane[1], L, 32, r, b, p.word) >> p.bit) & 0xffu) - 128;
         return d * (float)q;
     }
     if (f == kQ3K) {

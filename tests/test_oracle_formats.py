@@ -53,9 +53,10 @@ def test_all_zero_weights_pack_to_zero(orc):
     w = np.zeros((3, 300), np.float32)
     for f in FMTS:
         p = orc.pack(f, w)
-        # Q3_K stores sub-scales and codes with an offset (sc+32, q+4), so
-        # its zero block is not all-zero bytes; every format decodes to 0.
-        if f != "Q3_K":
+        # Q3_K stores sub-scales and codes with an offset (sc+32, q+4) and
+        # Q8_0 its codes as q+128, so their zero blocks are not all-zero
+        # bytes; every format decodes to 0.
+        if f not in ("Q3_K", "Q8_0"):
             assert not p.any()
         u = orc.unpack(f, p, 3, 300)
         assert not u.any()
