@@ -117,7 +117,6 @@ __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
                  ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
-__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(512) : "memory"); }
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
@@ -145,14 +144,16 @@ __device__ __forceinline__ uint32_t lds8(uint32_t a) {
 }
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
-constexpr int kConsumers = 16;                      // consumer warps (the last also produces)
-constexpr int kThreads = kConsumers * 32;
-constexpr int kProducerWarp = kConsumers - 1;
-constexpr int kNST = 4;                             // ring stages
-constexpr int kStageBytes = 48 * 1024;
-constexpr int kStageSb = 8;                         // superblocks per stage (Q8_0: 4), fewer if over budget
+constexpr int kConsumers = 8;                       // consumer warps
+constexpr int kThreads = (kConsumers + 1) * 32;     // + one producer warp
+constexpr int kProducerWarp = kConsumers;
+constexpr int kNST = 3;                             // ring stages
+constexpr int kStageBytes = 64 * 1024;
+constexpr int kStageSb = 16;                        // superblocks per stage (Q8_0: 8), fewer if over budget
 constexpr int kMaxCachedAssign = 2048;              // routed assignments cached in smem
 constexpr uint32_t kErrFull = 1u, kErrEmpty = 2u;
+// named barrier 1: the consumer warps only
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers * 32) : "memory"); }
 
 struct DecodeArgs {
     Dims d;
@@ -167,26 +168,24 @@ struct DecodeArgs {
     float* out;
 };
 
-// stage header written by the producer (one per ring slot)
-struct Hdr {
-    int32_t item, j, nst, s0, ks, kl;     // kl: superblocks the stage layout is sized for
-    int32_t fmt, e, tensor, rb, tg, ntok, shared;
-    int32_t vec[kDecodeTok], asg[kDecodeTok];
-    int32_t woff[4];         // weight plane regions in the stage
-    int32_t tok0, tstride;   // token regions
+// stage header written by the producer (one per ring slot); the stage's
+// byte layout is geo[fmt - 1][ntok - 1]
+struct __align__(16) Hdr {
+    int32_t item, j, nst, s0;
+    int32_t ks, fmt, tensor, ntok;
+    int32_t rb, e, shared, pad;
+    int32_t asg[kDecodeTok];
 };
 
-struct TokLay { int x, x1, sig, o, s, stride; };
+// token pieces in a stage: the family fragments, the Q3_K high-bit fragments
+// and the per-superblock statistics, each for the stage's ks superblocks
+struct TokLay { int x, x1, s, stride; };
 __device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
     TokLay t;
-    const bool wide = fmt == kQ4K || fmt == kQ80;
     int at = 0;
     t.x = at; at += ks * 512;
     t.x1 = at; if (fmt == kQ3K) at += ks * 512;
-    t.sig = at; at += ks * 32;
-    const int no = wide ? 8 : 16;
-    t.o = at; at += ks * no * 4;
-    t.s = at; if (fmt == kQ2K || fmt == kQ4K) at += ks * no * 4;
+    t.s = at; at += ks * kStatFloats * 4;
     t.stride = (at + 127) & ~127;
     return t;
 }
@@ -209,6 +208,19 @@ __device__ __forceinline__ int stage_sb(int fmt, int ntok) {
 struct SlotCache {
     int32_t e[kMaxExperts + 1], first[kMaxExperts + 1], ntot[kMaxExperts + 1];
     int32_t pre[kMaxExperts + 2];
+    const uint8_t* ptr[kMaxExperts + 1];   // the streamed tensor(s) of the slot's expert (gate or down)
+    const uint8_t* ptr_up[kMaxExperts + 1];
+    uint8_t fmt[kMaxExperts + 1][2];
+};
+
+// Stage geometry of one (format, tokens per item) pair, computed once per CTA
+// so the producer does no layout arithmetic per stage.
+struct Geo {
+    int64_t pl[4];       // plane starts in the tensor
+    int64_t rbstr[4];    // bytes per 32-row block in each plane
+    int per, nst, npl;   // superblocks per stage, stages per tensor, planes
+    int woff[4], cstr[4];// plane regions in the stage, bytes per superblock
+    int tok0, tstride, tx, tx1, ts;
 };
 
 struct ItemDesc {            // decoded item (producer side)
@@ -217,18 +229,21 @@ struct ItemDesc {            // decoded item (producer side)
 };
 
 template <bool kDown>
-__device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache& sc, const int32_t* s_perm, int n_slots,
-                                            int id, int& cursor, const ExpertTab& tab, ItemDesc& it) {
+__device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache& sc, const int32_t* s_perm,
+                                            const Geo (*geo)[kDecodeTok], int n_slots, int id, int& cursor,
+                                            ItemDesc& it, int& slot) {
     while (cursor + 1 < n_slots && sc.pre[cursor + 1] <= id) ++cursor;
     const int p = cursor;
-    int local = id - sc.pre[p];
+    slot = p;
+    const int local = id - sc.pre[p];
     const Dims& d = A.d;
     const int nrb = (kDown ? d.H : d.I) / 32;
-    it.rb = local % nrb;
     it.tg = local / nrb;
+    it.rb = local - it.tg * nrb;
     it.e = sc.e[p];
     it.shared = p < d.has_shared;
     it.ntok = min(kDecodeTok, sc.ntot[p] - it.tg * kDecodeTok);
+#pragma unroll
     for (int j = 0; j < kDecodeTok; ++j) {
         int t = 0, a = 0;
         if (j < it.ntok) {
@@ -243,197 +258,205 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
         it.asg[j] = a;
         it.vec[j] = kDown ? a : t;
     }
-    auto stages = [&](int fmt, int nsb) { const int per = stage_sb(fmt, it.ntok); return (nsb + per - 1) / per; };
-    if (!kDown) {
-        it.nst0 = stages(tab.fmt[it.e][0], A.nsbx);
-        it.nst = it.nst0 + stages(tab.fmt[it.e][1], A.nsbx);
-    } else {
-        it.nst0 = stages(tab.fmt[it.e][2], A.nsbi);
-        it.nst = it.nst0;
-    }
+    it.nst0 = geo[sc.fmt[p][0] - 1][it.ntok - 1].nst;
+    it.nst = kDown ? it.nst0 : it.nst0 + geo[sc.fmt[p][1] - 1][it.ntok - 1].nst;
 }
 
-// ---- consumer math: one warp = one 16-row tile x one superblock (Q8_0: half) ----
-// x one token.  k-steps alternate between two accumulators (the two slot
-// tiles of 16-wide sub-blocks, or even/odd steps of 32-wide ones) so
-// consecutive MMAs are independent.  acc[h]: row g + 8h of the tile.
+// ---- consumer math: one warp = the 32 rows of the stage (two 16-row MMA
+// tiles) x one superblock (Q8_0: half of its code pairs) x one token.
+//
+// MMA m16n8k16, rows g / g+8 of a tile for lane (g, t).  One MMA covers pair
+// m of eight sub-blocks: lane t feeds sub-block t of the group through a0/a1
+// and sub-block t+4 through a2/a3, so column n of B (and D) is sub-block n
+// of the group.  Operand B is static per lane: lane (g, t) supplies
+// activations only where g == t (b0) or g == t + 4 (b1) and zeros otherwise,
+// so no masking happens in the loop; the zero lanes read a zero block of
+// shared memory.  Both row tiles share the B registers.  D lane (g, t) then
+// holds sub-blocks 2t, 2t+1 of the group, whose scale fields are one word of
+// the slot-ordered record.  acc[2 * tile + h] accumulates row 16 tile + g + 8 h.
+__device__ __forceinline__ uint32_t sub4(uint4 v, int i) { return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w; }
+__device__ __forceinline__ float u8f(uint32_t w, int b) { return (float)((w >> (8 * b)) & 0xffu); }
+__device__ __forceinline__ void ld_frag8(uint32_t a, uint32_t (&X)[8]) {
+    const uint4 u = lds128(a), v = lds128(a + 16);
+    X[0] = u.x; X[1] = u.y; X[2] = u.z; X[3] = u.w; X[4] = v.x; X[5] = v.y; X[6] = v.z; X[7] = v.w;
+}
+
 template <int FMT>
-__device__ __forceinline__ void tile_token(const Hdr& h, uint32_t st, int jj, int half, int rt, int tk,
-                                           float (&acc)[2]) {
-    const int lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
-    constexpr bool kWide = FMT == kQ4K || FMT == kQ80;
-    // ---- weights of rows (tile rt, g + 8 hl) for superblock jj of the stage
-    uint32_t cw[2][8];
-    uint32_t hw[2][2];
-    uint32_t fld[2];
-    float dd[2], dm[2];
+__device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, int half, int tk, uint32_t zaddr,
+                                           float (&acc)[4]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const bool own0 = g == t, own1 = g == t + 4;
     const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
-#pragma unroll
-    for (int hl = 0; hl < 2; ++hl) {
-        const int r = 16 * rt + 8 * hl + g;
-        fld[hl] = 0u; dm[hl] = 0.0f;
-        if (FMT == kQ2K) {
-            const uint4 c = lds128(st + w3 + (jj * 32 + r) * 64 + 16 * t4);
-            cw[hl][0] = c.x; cw[hl][1] = c.y; cw[hl][2] = c.z; cw[hl][3] = c.w;
-            fld[hl] = lds32(st + w2 + (jj * 32 + r) * 16 + 4 * t4);
-            dd[hl] = h2f(lds16(st + w0 + (jj * 32 + r) * 2));
-            dm[hl] = h2f(lds16(st + w1 + (jj * 32 + r) * 2));
-        } else if (FMT == kQ3K) {
-            const uint4 c = lds128(st + w2 + (jj * 32 + r) * 64 + 16 * t4);
-            cw[hl][0] = c.x; cw[hl][1] = c.y; cw[hl][2] = c.z; cw[hl][3] = c.w;
-            const uint2 hv = lds64(st + w3 + (jj * 32 + r) * 32 + 8 * t4);
-            hw[hl][0] = hv.x; hw[hl][1] = hv.y;
-            const uint32_t sp = st + w1 + (jj * 32 + r) * 12;
-            fld[hl] = lds16(sp + 2 * t4) | (lds8(sp + 8 + t4) << 16);
-            dd[hl] = h2f(lds16(st + w0 + (jj * 32 + r) * 2));
-        } else if (FMT == kQ4K) {
-            const uint4 c0 = lds128(st + w3 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t4);
-            const uint4 c1 = lds128(st + w3 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t4);
-            cw[hl][0] = c0.x; cw[hl][1] = c0.y; cw[hl][2] = c0.z; cw[hl][3] = c0.w;
-            cw[hl][4] = c1.x; cw[hl][5] = c1.y; cw[hl][6] = c1.z; cw[hl][7] = c1.w;
-            const uint32_t sp = st + w2 + (jj * 32 + r) * 12;
-            fld[hl] = lds16(sp + 2 * t4) | (lds8(sp + 8 + t4) << 16);
-            dd[hl] = h2f(lds16(st + w0 + (jj * 32 + r) * 2));
-            dm[hl] = h2f(lds16(st + w1 + (jj * 32 + r) * 2));
-        } else {  // Q8_0: blocks 8*jj + 4*half + (0..3)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint2 v = lds64(st + w1 + ((8 * jj + 4 * half + q) * 32 + r) * 32 + 8 * t4);
-                cw[hl][2 * q] = v.x; cw[hl][2 * q + 1] = v.y;
-            }
-            dd[hl] = h2f(lds16(st + w0 + ((8 * jj + 2 * t4) * 32 + r) * 2));
-            dm[hl] = h2f(lds16(st + w0 + ((8 * jj + 2 * t4 + 1) * 32 + r) * 2));
-        }
-    }
-    const TokLay tl = tok_lay(FMT, h.kl);
     const uint32_t tb = st + h.tok0 + tk * h.tstride;
-    const uint4 X = lds128(tb + tl.x + jj * 512 + (g * 4 + t4) * 16);
-    uint4 X1 = make_uint4(0, 0, 0, 0);
-    if (FMT == kQ3K) X1 = lds128(tb + tl.x1 + jj * 512 + (g * 4 + t4) * 16);
-    float D[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-#pragma unroll
-    for (int ii = 0; ii < (FMT == kQ80 ? 8 : 16); ++ii) {
-        // 16-wide formats: i = 0, 8, 1, 9, ...; wide formats: in order (parity alternates)
-        const int i = FMT == kQ80 ? 8 * half + ii : (kWide ? ii : ((ii >> 1) + 8 * (ii & 1)));
-        const int owner = kWide ? (i >> 1) : (i & 7);
-        const int sel = kWide ? (i & 1) : (i >> 3);
-        const int acc_id = kWide ? (i & 1) : (i >> 3);
-        // slot mask: only lanes of group `owner` supply the activations
-        const uint32_t mk = g == owner ? 0x3C003C00u : 0u;
-        uint32_t a[4];
-        if (FMT == kQ2K || FMT == kQ3K) {
-#pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
-                const uint32_t w = cw[hl][i >> 2], w10 = w >> 10;
-                switch (i & 3) {
-                case 0: a[hl] = ext2<0>(w, w10); a[2 + hl] = ext2<1>(w, w10); break;
-                case 1: a[hl] = ext2<2>(w, w10); a[2 + hl] = ext2<3>(w, w10); break;
-                case 2: a[hl] = ext2<4>(w, w10); a[2 + hl] = ext2<5>(w, w10); break;
-                default: a[hl] = ext2<6>(w, w10); a[2 + hl] = ext2<7>(w, w10); break;
-                }
-            }
-        } else if (FMT == kQ4K) {
-#pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
-                const uint32_t w = cw[hl][4 * (i >> 3) + ((i & 7) >> 1)];
-                const uint32_t ws = (i & 1) ? (w >> 8) : w;
-                a[hl] = lop3_and_or(ws, 0x000F000Fu, 0x64006400u);
-                a[2 + hl] = lop3_and_or(ws, 0x00F000F0u, 0x64006400u);
-            }
-        } else {
-#pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
-                const uint32_t w = cw[hl][2 * ((i >> 1) - 4 * half) + (i & 1)];
-                a[hl] = lop3_q8(w);
-                a[2 + hl] = lop3_q8(w >> 8);
-            }
-        }
-        const uint32_t b0 = hmul2u(sel ? X.z : X.x, mk);
-        const uint32_t b1 = hmul2u(sel ? X.w : X.y, mk);
-        mma16816(D[acc_id], a[0], a[1], a[2], a[3], b0, b1);
-        if (FMT == kQ3K) {
-            uint32_t ah[4];
-#pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
-                const uint32_t w = hw[hl][i >> 3], w10 = w >> 10;
-                switch (i & 7) {
-                case 0: ah[hl] = ext1<0>(w, w10); ah[2 + hl] = ext1<1>(w, w10); break;
-                case 1: ah[hl] = ext1<2>(w, w10); ah[2 + hl] = ext1<3>(w, w10); break;
-                case 2: ah[hl] = ext1<4>(w, w10); ah[2 + hl] = ext1<5>(w, w10); break;
-                case 3: ah[hl] = ext1<6>(w, w10); ah[2 + hl] = ext1<7>(w, w10); break;
-                case 4: ah[hl] = ext1<8>(w, w10); ah[2 + hl] = ext1<9>(w, w10); break;
-                case 5: ah[hl] = ext1<10>(w, w10); ah[2 + hl] = ext1<11>(w, w10); break;
-                case 6: ah[hl] = ext1<12>(w, w10); ah[2 + hl] = ext1<13>(w, w10); break;
-                default: ah[hl] = ext1<14>(w, w10); ah[2 + hl] = ext1<15>(w, w10); break;
-                }
-            }
-            const uint32_t c0 = hmul2u(sel ? X1.z : X1.x, mk);
-            const uint32_t c1 = hmul2u(sel ? X1.w : X1.y, mk);
-            mma16816(D[acc_id], ah[0], ah[1], ah[2], ah[3], c0, c1);
-        }
-    }
-    // ---- epilogue: sub-block scales / mins in fp32
+    const uint32_t xb = tb + h.tx + jj * 512, sb = tb + h.ts + jj * (kStatFloats * 4);
+    const int rbase = jj * 32 + g;   // record index of row g of tile 0
+
     if (FMT == kQ2K || FMT == kQ3K) {
-        const uint4 Ou = lds128(tb + tl.o + jj * 64 + t4 * 16);
-        const float Ov[4] = {__uint_as_float(Ou.x), __uint_as_float(Ou.y), __uint_as_float(Ou.z), __uint_as_float(Ou.w)};
-        float Sv[4] = {0.f, 0.f, 0.f, 0.f};
-        if (FMT == kQ2K) {
-            const uint4 Su = lds128(tb + tl.s + jj * 64 + t4 * 16);
-            Sv[0] = __uint_as_float(Su.x); Sv[1] = __uint_as_float(Su.y);
-            Sv[2] = __uint_as_float(Su.z); Sv[3] = __uint_as_float(Su.w);
+        const uint32_t cp = FMT == kQ2K ? w3 : w2;   // 2-bit code plane
+        uint4 c[4];                                   // rows g, g+8, 16+g, 24+g
+        uint2 hv[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            c[i] = lds128(st + cp + (rbase + 8 * i) * 64 + 16 * t);
+            if (FMT == kQ3K) hv[i] = lds64(st + w3 + (rbase + 8 * i) * 32 + 8 * t);
         }
-        const float sg0 = ldsf(tb + tl.sig + (8 * jj + t4) * 4), sg1 = ldsf(tb + tl.sig + (8 * jj + 4 + t4) * 4);
+        float DD[2][2][2][4];   // [tile][group][pair parity]
 #pragma unroll
-        for (int hl = 0; hl < 2; ++hl) {
-            float a_sc = 0.0f, a_m = 0.0f;
+        for (int i = 0; i < 32; ++i) (&DD[0][0][0][0])[i] = 0.0f;
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {   // v = 2*tile + e
-                const float P = fmaf(D[v >> 1][2 * hl + (v & 1)], (v >> 1) ? sg1 : sg0, -Ov[v]);
-                if (FMT == kQ2K) {
-                    const uint32_t byte = (fld[hl] >> (8 * v)) & 0xffu;
-                    a_sc = fmaf((float)(byte & 15u), P, a_sc);
-                    a_m = fmaf((float)(byte >> 4), Sv[v], a_m);
-                } else {
-                    const uint32_t f = fld[hl];
-                    const int sfield = (int)((f >> (4 * v)) & 15u) | (int)(((f >> (16 + 2 * v)) & 3u) << 4);
-                    a_sc = fmaf((float)(sfield - 32), P, a_sc);
+        for (int gm = 0; gm < 2; ++gm) {
+            uint32_t XA[8], XB[8];
+            ld_frag8(own0 ? xb + 32 * (8 * gm + t) : zaddr, XA);
+            ld_frag8(own1 ? xb + 32 * (8 * gm + 4 + t) : zaddr, XB);
+            uint32_t qa[4], qb[4], sa[4], sbb[4];   // per row: sub-blocks t (a0/a1) and t+4 (a2/a3)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                qa[i] = sub4(c[i], 2 * gm); qb[i] = sub4(c[i], 2 * gm + 1);
+                sa[i] = qa[i] >> 10; sbb[i] = qb[i] >> 10;
+            }
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
+                const bool sh = m > 4;
+#pragma unroll
+                for (int tl = 0; tl < 2; ++tl)
+                    mma16816(DD[tl][gm][m & 1], (sh ? sa[2 * tl] : qa[2 * tl]) & mk,
+                             (sh ? sa[2 * tl + 1] : qa[2 * tl + 1]) & mk, (sh ? sbb[2 * tl] : qb[2 * tl]) & mk,
+                             (sh ? sbb[2 * tl + 1] : qb[2 * tl + 1]) & mk, XA[m], XB[m]);
+            }
+            if (FMT == kQ3K) {
+                ld_frag8(own0 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + t) : zaddr, XA);
+                ld_frag8(own1 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + 4 + t) : zaddr, XB);
+                uint32_t ha[4], hb[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) { ha[i] = gm ? hv[i].y : hv[i].x; hb[i] = ha[i] >> 8; }
+#pragma unroll
+                for (int m = 0; m < 8; ++m) {
+                    const uint32_t mk = 0x00010001u << m;
+#pragma unroll
+                    for (int tl = 0; tl < 2; ++tl)
+                        mma16816(DD[tl][gm][m & 1], ha[2 * tl] & mk, ha[2 * tl + 1] & mk, hb[2 * tl] & mk,
+                                 hb[2 * tl + 1] & mk, XA[m], XB[m]);
                 }
             }
-            float r = dd[hl] * a_sc;
-            if (FMT == kQ2K) r = fmaf(-dm[hl], a_m, r);
-            acc[hl] += r;
         }
-    } else {
-        const uint2 Ou = lds64(tb + tl.o + (8 * jj + 2 * t4) * 4);
-        const uint2 Gu = lds64(tb + tl.sig + (8 * jj + 2 * t4) * 4);
-        const float O0 = __uint_as_float(Ou.x), O1 = __uint_as_float(Ou.y);
-        const float sg0 = __uint_as_float(Gu.x), sg1 = __uint_as_float(Gu.y);
-        float S0 = 0.f, S1 = 0.f;
-        if (FMT == kQ4K) {
-            const uint2 Su = lds64(tb + tl.s + (8 * jj + 2 * t4) * 4);
-            S0 = __uint_as_float(Su.x); S1 = __uint_as_float(Su.y);
-        }
-        // Q8_0: this half holds blocks 4*half..4*half+3; lane t4 owns blocks 2*t4, 2*t4+1
-        if (FMT == kQ4K || (t4 >> 1) == half) {
+        // ---- epilogue: slot-ordered scale word of each row: bytes b = 2*group + col
+        const float cf0 = ldsf(sb + 4 * (kStatC + t)), cf1 = ldsf(sb + 4 * (kStatC + 4 + t));
+        const uint4 Su = lds128(sb + 4 * (kStatS16 + 4 * t));
+        const float S[4] = {__uint_as_float(Su.x), __uint_as_float(Su.y), __uint_as_float(Su.z),
+                            __uint_as_float(Su.w)};
 #pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
-                const float D0 = D[0][2 * hl] + D[1][2 * hl];
-                const float D1 = D[0][2 * hl + 1] + D[1][2 * hl + 1];
-                const float P0 = fmaf(D0, sg0, -O0), P1 = fmaf(D1, sg1, -O1);
-                if (FMT == kQ4K) {
-                    const uint32_t f = fld[hl];
-                    const int hi = (int)(f >> 16);
-                    const float sc0 = (float)((f & 15u) | ((hi & 3) << 4));
-                    const float m0 = (float)(((f >> 4) & 15u) | (((hi >> 2) & 3) << 4));
-                    const float sc1 = (float)(((f >> 8) & 15u) | (((hi >> 4) & 3) << 4));
-                    const float m1 = (float)(((f >> 12) & 15u) | (((hi >> 6) & 3) << 4));
-                    const float a_sc = fmaf(sc1, P1, sc0 * P0);
-                    const float a_m = fmaf(m1, S1, m0 * S0);
-                    acc[hl] += fmaf(dd[hl], a_sc, -dm[hl] * a_m);
-                } else {
-                    acc[hl] += fmaf(dd[hl], P0, dm[hl] * P1);
+        for (int i = 0; i < 4; ++i) {   // row g + 8 i = tile i / 2, half i % 2
+            const int tl = i >> 1, hl = i & 1;
+            float D[2][2];
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm)
+#pragma unroll
+                for (int cc = 0; cc < 2; ++cc) D[gm][cc] = DD[tl][gm][0][2 * hl + cc] + DD[tl][gm][1][2 * hl + cc];
+            const int rec = rbase + 8 * i;
+            const float d = h2f(lds16(st + w0 + rec * 2));
+            if (FMT == kQ2K) {
+                const float dm = h2f(lds16(st + w1 + rec * 2));
+                const uint32_t f = lds32(st + w2 + rec * 16 + 4 * t);
+                const uint32_t sc4 = f & 0x0F0F0F0Fu, m4 = (f >> 4) & 0x0F0F0F0Fu;
+                const float a0 = fmaf(u8f(sc4, 1), D[0][1], u8f(sc4, 0) * D[0][0]);
+                const float a1 = fmaf(u8f(sc4, 3), D[1][1], u8f(sc4, 2) * D[1][0]);
+                const float am = fmaf(u8f(m4, 3), S[3], fmaf(u8f(m4, 2), S[2], fmaf(u8f(m4, 1), S[1], u8f(m4, 0) * S[0])));
+                acc[i] += fmaf(d, fmaf(cf1, a1, cf0 * a0), -dm * am);
+            } else {
+                const uint32_t sp = st + w1 + rec * 12;
+                const uint32_t f = lds16(sp + 2 * t) | (lds8(sp + 8 + t) << 16);
+                float a = 0.0f;
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    const float sv = (float)((int)(((f >> (4 * b)) & 15u) | (((f >> (16 + 2 * b)) & 3u) << 4)) - 32);
+                    const float P = fmaf(D[b >> 1][b & 1], (b >> 1) ? cf1 : cf0, -4.0f * S[b]);
+                    a = fmaf(sv, P, a);
                 }
+                acc[i] = fmaf(d, a, acc[i]);
             }
+        }
+    } else if (FMT == kQ4K) {
+        uint4 cA[4], cB[4];   // rows g + 8 i: sub-blocks t (unit 0) and t+4 (unit 1)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int rec = rbase + 8 * i;
+            cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + (rec - jj * 32)) * 64 + 16 * t);
+            cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + (rec - jj * 32)) * 64 + 16 * t);
+        }
+        float DD[2][2][4];   // [tile][pair parity]
+#pragma unroll
+        for (int i = 0; i < 16; ++i) (&DD[0][0][0])[i] = 0.0f;
+#pragma unroll
+        for (int hm = 0; hm < 2; ++hm) {   // pairs 8 hm .. 8 hm + 7
+            uint32_t XA[8], XB[8];
+            ld_frag8(own0 ? xb + 64 * t + 32 * hm : zaddr, XA);
+            ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * hm : zaddr, XB);
+#pragma unroll
+            for (int mm = 0; mm < 8; ++mm) {
+                const int m = 8 * hm + mm, wi = m >> 2, j = m & 3;
+                const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
+                const int sh = j < 2 ? 0 : 8;
+#pragma unroll
+                for (int tl = 0; tl < 2; ++tl)
+                    mma16816(DD[tl][m & 1], (sub4(cA[2 * tl], wi) >> sh) & mk, (sub4(cA[2 * tl + 1], wi) >> sh) & mk,
+                             (sub4(cB[2 * tl], wi) >> sh) & mk, (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[mm], XB[mm]);
+            }
+        }
+        const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
+        const float cf0 = __uint_as_float(Cu.x), cf1 = __uint_as_float(Cu.y);
+        const float S0 = __uint_as_float(Su.x), S1 = __uint_as_float(Su.y);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int tl = i >> 1, hl = i & 1, rec = rbase + 8 * i;
+            const float d = h2f(lds16(st + w0 + rec * 2));
+            const float dm = h2f(lds16(st + w1 + rec * 2));
+            const uint32_t sp = st + w2 + rec * 12;
+            const uint32_t f = lds16(sp + 2 * t), hi = lds8(sp + 8 + t);
+            const float sc0 = (float)((f & 15u) | ((hi & 3u) << 4));
+            const float m0 = (float)(((f >> 4) & 15u) | (((hi >> 2) & 3u) << 4));
+            const float sc1 = (float)(((f >> 8) & 15u) | (((hi >> 4) & 3u) << 4));
+            const float m1 = (float)(((f >> 12) & 15u) | (((hi >> 6) & 3u) << 4));
+            const float D0 = DD[tl][0][2 * hl] + DD[tl][1][2 * hl], D1 = DD[tl][0][2 * hl + 1] + DD[tl][1][2 * hl + 1];
+            const float a_sc = fmaf(sc1 * cf1, D1, sc0 * cf0 * D0);
+            const float a_m = fmaf(m1, S1, m0 * S0);
+            acc[i] += fmaf(d, a_sc, -dm * a_m);
+        }
+    } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7
+        uint4 cA[4], cB[4];   // rows g + 8 i: blocks t and t+4
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int r = g + 8 * i;
+            cA[i] = lds128(st + w1 + ((8 * jj + t) * 32 + r) * 32 + 16 * half);
+            cB[i] = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r) * 32 + 16 * half);
+        }
+        uint32_t XA[8], XB[8];
+        ld_frag8(own0 ? xb + 64 * t + 32 * half : zaddr, XA);
+        ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * half : zaddr, XB);
+        float DD[2][2][4];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) (&DD[0][0][0])[i] = 0.0f;
+#pragma unroll
+        for (int mm = 0; mm < 8; ++mm) {
+            const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0;
+#pragma unroll
+            for (int tl = 0; tl < 2; ++tl)
+                mma16816(DD[tl][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
+                         (sub4(cA[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, (sub4(cB[2 * tl], wi) >> sh) & 0x00FF00FFu,
+                         (sub4(cB[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, XA[mm], XB[mm]);
+        }
+        const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
+        const float cf0 = __uint_as_float(Cu.x), cf1 = __uint_as_float(Cu.y);
+        // codes are stored q + 128: one half removes 128 * sum(x) per block
+        const float o0 = half ? 0.0f : 128.0f * __uint_as_float(Su.x);
+        const float o1 = half ? 0.0f : 128.0f * __uint_as_float(Su.y);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int tl = i >> 1, hl = i & 1, r = g + 8 * i;
+            const float d0 = h2f(lds16(st + w0 + ((8 * jj + 2 * t) * 32 + r) * 2));
+            const float d1 = h2f(lds16(st + w0 + ((8 * jj + 2 * t + 1) * 32 + r) * 2));
+            const float D0 = DD[tl][0][2 * hl] + DD[tl][1][2 * hl], D1 = DD[tl][0][2 * hl + 1] + DD[tl][1][2 * hl + 1];
+            acc[i] += fmaf(d1, fmaf(D1, cf1, -o1), d0 * fmaf(D0, cf0, -o0));
         }
     }
 }
@@ -446,24 +469,57 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     __shared__ int32_t s_perm[kMaxCachedAssign];
     __shared__ __align__(8) uint64_t bars[2 * kNST];
     __shared__ Hdr hdr[kNST];
-    __shared__ float red[2][kConsumers][2][kDecodeTok][16];   // double-buffered by item parity
+    __shared__ float red[2][kConsumers][2][kDecodeTok][32];   // double-buffered by item parity
     __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
+    __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
+    __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
     const Dims& d = A.d;
     const int n_slots = A.plan->n_slots;
+    __shared__ Geo geo[4][kDecodeTok];
     for (int i = threadIdx.x; i <= n_slots; i += blockDim.x) {
         sc.pre[i] = kDown ? A.plan->pre_dn[i] : A.plan->pre_gu[i];
         if (i < n_slots) {
-            if (i < d.has_shared) { sc.e[i] = d.E; sc.first[i] = 0; sc.ntot[i] = d.T; }
+            int e;
+            if (i < d.has_shared) { e = d.E; sc.first[i] = 0; sc.ntot[i] = d.T; }
             else {
-                const int e = A.active[1 + i - d.has_shared];
-                sc.e[i] = e; sc.first[i] = A.offsets[e]; sc.ntot[i] = A.offsets[e + 1] - A.offsets[e];
+                e = A.active[1 + i - d.has_shared];
+                sc.first[i] = A.offsets[e]; sc.ntot[i] = A.offsets[e + 1] - A.offsets[e];
             }
+            sc.e[i] = e;
+            sc.ptr[i] = tab.p[e][kDown ? 2 : 0];
+            sc.ptr_up[i] = tab.p[e][1];
+            sc.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
+            sc.fmt[i][1] = tab.fmt[e][1];
         }
+    }
+    if (threadIdx.x < 4 * kDecodeTok) {
+        const int fmt = 1 + threadIdx.x / kDecodeTok, ntok = 1 + threadIdx.x % kDecodeTok;
+        Geo& G = geo[fmt - 1][ntok - 1];
+        const int nsb = kDown ? (d.I + 255) / 256 : (d.H + 255) / 256;
+        const TensorLayout L = tensor_layout(fmt, kDown ? d.H : d.I, kDown ? d.I : d.H);
+        const PlaneBytes pb = plane_bytes(fmt);
+        const int bmul = fmt == kQ80 ? 8 : 1;
+        G.per = stage_sb(fmt, ntok);
+        G.nst = (nsb + G.per - 1) / G.per;
+        G.npl = pb.n;
+        int at = 0;
+        for (int pl = 0; pl < 4; ++pl) {
+            G.woff[pl] = at;
+            G.cstr[pl] = pl < pb.n ? 32 * bmul * pb.b[pl] : 0;
+            G.pl[pl] = L.plane[pl];
+            G.rbstr[pl] = pl < pb.n ? L.blocks_per_row * 32 * pb.b[pl] : 0;
+            if (pl < pb.n) at += (32 * bmul * G.per * pb.b[pl] + 127) & ~127;
+        }
+        const TokLay tl = tok_lay(fmt, G.per);
+        G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.tx1 = tl.x1; G.ts = tl.s;
     }
     const int n_routed = min(d.T * d.K, kMaxCachedAssign);
     for (int i = threadIdx.x; i < n_routed; i += blockDim.x) s_perm[i] = A.perm[i];
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
     if (threadIdx.x < kNST) s_posted[threadIdx.x] = -1;
+    if (threadIdx.x < 8) zero_blk[threadIdx.x] = 0u;
+    if (threadIdx.x == 0) s_fail = 0;
+    const uint32_t zaddr = (uint32_t)__cvta_generic_to_shared(zero_blk);
     if (threadIdx.x == 0) {
         for (int s = 0; s < kNST; ++s) {
             mbar_init(bar0 + 8 * s, 1);                       // full[s]: producer arrival + tx bytes
@@ -475,240 +531,214 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     const int n_items = sc.pre[n_slots];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
-    const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)stat_off(A.nsbi).total, A.nsbi}
-                            : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)stat_off(A.nsbx).total, A.nsbx};
 
-    // ====================== producer (run by warp 7) ========================
-    // Per phase (one tensor of one item) every lane of warp 7 owns at most one
-    // copy: lanes 0..3 a weight plane, lanes 4.. one piece of one token
-    // (fragments, high-bit fragments, sigma, offsets, sums).  A stage then only
-    // advances the source by the stage's first superblock.
-    int p_cursor = 0, p_item = -1, p_j = 0, p_q = 0, p_nst = 0, p_nst0 = 0;
-    int p_phase_j = 0, p_per = 1, p_nsb = vs.nsb, p_fmt = 0, p_tensor = 0;
-    bool p_failed = false, p_done = false;
-    const uint8_t* c_src = nullptr;       // this lane's copy: source at superblock 0
-    uint32_t c_stride = 0, c_dst = 0;     // bytes per superblock, offset in the stage
-    int h_woff0 = 0, h_woff1 = 0, h_woff2 = 0, h_woff3 = 0, h_tok0 = 0, h_tstride = 0;
-    ItemDesc P;
-    P.nst = 0; P.ntok = 0;
-    const StatOff so = stat_off(vs.nsb);
-    int next_id = 0;
-    if (warp == kProducerWarp && lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);
-
-#define MQ_PRODUCE_ONE()                                                                                   \
-    do {                                                                                                   \
-        if (p_done) break;                                                                                 \
-        if (p_j == p_nst) {                                                                                \
-            const int id = __shfl_sync(kFull, next_id, 0);                                                 \
-            p_item = id < n_items ? id : -1;                                                               \
-            if (p_item >= 0) {                                                                             \
-                decode_item<kDown>(A, sc, s_perm, n_slots, p_item, p_cursor, tab, P);                     \
-                if (lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);                       \
-                p_nst = P.nst; p_nst0 = P.nst0;                                                            \
-            }                                                                                              \
-            p_j = 0;                                                                                       \
-        }                                                                                                  \
-        const int slot = p_q % kNST;                                                                       \
-        const uint32_t full = bar0 + 8 * slot, empty = bar0 + 8 * (kNST + slot);                            \
-        if (p_q >= kNST && !mbar_wait(empty, ((p_q / kNST) & 1) ^ 1, A.err, kErrEmpty)) {                \
-            p_failed = true; p_done = true; break;                                                         \
-        }                                                                                                  \
-        if (p_item < 0) {                                                                                  \
-            if (lane == 0) { hdr[slot].item = -1; s_posted[slot] = p_q; mbar_arrive(full); }              \
-            p_done = true;                                                                                 \
-            break;                                                                                         \
-        }                                                                                                  \
-        if (p_j == 0 || (!kDown && p_j == p_nst0)) {                                                       \
-            /* new phase: tensor, format, stage geometry, this lane's copy */                             \
-            p_tensor = kDown ? 2 : (p_j == 0 ? 0 : 1);                                                     \
-            p_phase_j = p_j;                                                                               \
-            p_fmt = tab.fmt[P.e][p_tensor];                                                                \
-            p_per = stage_sb(p_fmt, P.ntok);                                                               \
-            const TensorLayout L = tensor_layout(p_fmt, kDown ? d.H : d.I, kDown ? d.I : d.H);            \
-            const PlaneBytes pb = plane_bytes(p_fmt);                                                      \
-            const int bmul = p_fmt == kQ80 ? 8 : 1;                                                        \
-            int at = 0, wo[4] = {0, 0, 0, 0};                                                              \
-            _Pragma("unroll") for (int pl = 0; pl < 4; ++pl) {                                             \
-                wo[pl] = at;                                                                               \
-                if (pl < pb.n) at += (32 * bmul * p_per * pb.b[pl] + 127) & ~127;                          \
-            }                                                                                              \
-            h_woff0 = wo[0]; h_woff1 = wo[1]; h_woff2 = wo[2]; h_woff3 = wo[3];                            \
-            const TokLay tl = tok_lay(p_fmt, p_per);                                                       \
-            h_tok0 = at; h_tstride = tl.stride;                                                            \
-            c_src = nullptr; c_stride = 0; c_dst = 0;                                                      \
-            const uint8_t* tbase = tab.p[P.e][p_tensor];                                                   \
-            _Pragma("unroll") for (int pl = 0; pl < 4; ++pl)                                               \
-                if (lane == pl && pl < pb.n) {                                                             \
-                    c_src = tbase + L.plane[pl] + (int64_t)P.rb * L.blocks_per_row * 32 * pb.b[pl];        \
-                    c_stride = 32 * bmul * pb.b[pl];                                                       \
-                    c_dst = wo[pl];                                                                        \
-                }                                                                                          \
-            if (lane >= 4 && lane < 4 + 5 * P.ntok) {                                                      \
-                const int tk = (lane - 4) / 5, piece = (lane - 4) % 5;                                     \
-                int v = P.vec[0];                                                                          \
-                _Pragma("unroll") for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) v = P.vec[t2];     \
-                const uint8_t* qv = reinterpret_cast<const uint8_t*>(vs.q + (size_t)v * vs.q_stride);      \
-                const uint8_t* sv = reinterpret_cast<const uint8_t*>(vs.st + (size_t)v * vs.st_stride);    \
-                const int fam = p_fmt == kQ2K || p_fmt == kQ3K ? kF2 : p_fmt == kQ4K ? kF4 : kF8;          \
-                const bool wide = p_fmt == kQ4K || p_fmt == kQ80;                                          \
-                const uint32_t tb = h_tok0 + tk * tl.stride;                                               \
-                if (piece == 0) { c_src = qv + (size_t)fam * vs.nsb * 512; c_stride = 512; c_dst = tb + tl.x; } \
-                if (piece == 1 && p_fmt == kQ3K) {                                                         \
-                    c_src = qv + (size_t)kF1 * vs.nsb * 512; c_stride = 512; c_dst = tb + tl.x1;           \
-                }                                                                                          \
-                if (piece == 2) { c_src = sv + 4 * so.sig; c_stride = 32; c_dst = tb + tl.sig; }            \
-                if (piece == 3) {                                                                          \
-                    const int o = p_fmt == kQ2K ? so.os2 : p_fmt == kQ3K ? so.oq3 : p_fmt == kQ4K ? so.os4 : so.os8; \
-                    c_src = sv + 4 * o; c_stride = wide ? 32 : 64; c_dst = tb + tl.o;                       \
-                }                                                                                          \
-                if (piece == 4 && (p_fmt == kQ2K || p_fmt == kQ4K)) {                                      \
-                    c_src = sv + 4 * (p_fmt == kQ2K ? so.sxs16 : so.sxs32); c_stride = wide ? 32 : 64;     \
-                    c_dst = tb + tl.s;                                                                     \
-                }                                                                                          \
-            }                                                                                              \
-        }                                                                                                  \
-        const int s0 = (p_j - p_phase_j) * p_per, ks = min(p_per, p_nsb - s0);                             \
-        const uint32_t stage = ring + slot * kStageBytes;                                                  \
-        const uint32_t bytes = c_src ? (uint32_t)ks * c_stride : 0u;                                       \
-        uint32_t total = bytes;                                                                            \
-        _Pragma("unroll") for (int off = 16; off >= 1; off >>= 1) total += __shfl_xor_sync(kFull, total, off); \
-        if (lane == 0) {                                                                                   \
-            Hdr& H = hdr[slot];                                                                            \
-            H.item = p_item; H.j = p_j; H.nst = p_nst; H.s0 = s0; H.ks = ks; H.kl = p_per;                  \
-            H.fmt = p_fmt; H.e = P.e; H.tensor = p_tensor; H.rb = P.rb; H.tg = P.tg; H.ntok = P.ntok;      \
-            H.shared = P.shared;                                                                           \
-            _Pragma("unroll") for (int t2 = 0; t2 < kDecodeTok; ++t2) { H.vec[t2] = P.vec[t2]; H.asg[t2] = P.asg[t2]; } \
-            H.woff[0] = h_woff0; H.woff[1] = h_woff1; H.woff[2] = h_woff2; H.woff[3] = h_woff3;            \
-            H.tok0 = h_tok0; H.tstride = h_tstride;                                                        \
-            s_posted[slot] = p_q;                                                                          \
-            mbar_arrive_tx(full, total);                                                                   \
-        }                                                                                                  \
-        __syncwarp();                                                                                      \
-        if (bytes) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);                   \
-        ++p_j;                                                                                             \
-        ++p_q;                                                                                             \
-    } while (0)
-
-    if (warp == kProducerWarp)
-        for (int i = 0; i < kNST - 1; ++i) MQ_PRODUCE_ONE();
-
-    // ============================ consumer warps =============================
-    // warp w: row tile w & 1; superblock w >> 1 of the stage (Q8_0: superblock
-    // w >> 2, half (w >> 1) & 1)
-    const int rt = warp & 1;
-    float acc[2][kDecodeTok][2];   // [0] gate (or down), [1] up; rows g, g+8 of the tile
-    float cur[kDecodeTok][2];      // the tensor being streamed
-#pragma unroll
-    for (int tk = 0; tk < kDecodeTok; ++tk) {
-        acc[0][tk][0] = acc[0][tk][1] = acc[1][tk][0] = acc[1][tk][1] = 0.0f;
-        cur[tk][0] = cur[tk][1] = 0.0f;
-    }
-    int n_done = 0;   // items finished by this CTA (selects the reduction buffer and the owner warps)
-    for (int q = 0;; ++q) {
-        if (warp == kProducerWarp) MQ_PRODUCE_ONE();   // posts stage q + kNST - 1
-        const int slot = q % kNST;
-        if (!mbar_wait(bar0 + 8 * slot, (q / kNST) & 1, A.err, kErrFull)) { p_failed = true; break; }
-        const Hdr& H = hdr[slot];
-        if (H.item < 0) break;
-        const uint32_t stage = ring + slot * kStageBytes;
-        const bool q8 = H.fmt == kQ80;
-        const int sbj = q8 ? (warp >> 2) : (warp >> 1), half = q8 ? ((warp >> 1) & 1) : 0;
-        if (!kDown && H.tensor == 1 && H.s0 == 0) {
-            // first stage of the up tensor: the gate sums are complete
-#pragma unroll
-            for (int tk = 0; tk < kDecodeTok; ++tk) {
-                acc[0][tk][0] += cur[tk][0]; acc[0][tk][1] += cur[tk][1];
-                cur[tk][0] = cur[tk][1] = 0.0f;
+    if (warp == kProducerWarp) {
+        // ===================== producer (dedicated warp) =====================
+        // Per phase (one tensor of one item) every lane owns at most one copy:
+        // lanes 0..3 a weight plane, lanes 4.. one piece of one token (family
+        // fragments, Q3_K high-bit fragments, statistics).  A stage then only
+        // advances the source by the stage's first superblock.
+        const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi}
+                                : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
+        int p_cursor = 0, p_q = 0;
+        const int p_nsb = vs.nsb;
+        int next_id = 0;
+        if (lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);
+        ItemDesc P;
+        int pslot = 0;
+        for (;;) {
+            const int id = __shfl_sync(kFull, next_id, 0);
+            const int item = id < n_items ? id : -1;
+            if (item >= 0) {
+                decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
+                if (lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);
             }
+            const int nst = item >= 0 ? P.nst : 1;
+            bool failed = false;
+            // this lane's copy for the current phase (one tensor of the item)
+            const uint8_t* c_src = nullptr;
+            uint32_t c_stride = 0, c_dst = 0;
+            const Geo* G = nullptr;
+            int fmt = 0, tensor = 0, phase_j = 0;
+            for (int pj = 0; pj < nst; ++pj) {
+                const int slot = p_q % kNST;
+                const uint32_t full = bar0 + 8 * slot, empty = bar0 + 8 * (kNST + slot);
+                if (p_q >= kNST && !mbar_wait(empty, ((p_q / kNST) & 1) ^ 1, A.err, kErrEmpty)) {
+                    failed = true;
+                    break;
+                }
+                if (item < 0) {   // sentinel: consumers stop here
+                    if (lane == 0) { hdr[slot].item = -1; s_posted[slot] = p_q; mbar_arrive(full); }
+                    ++p_q;
+                    break;
+                }
+                if (pj == 0 || (!kDown && pj == P.nst0)) {
+                    tensor = kDown ? 2 : (pj == 0 ? 0 : 1);
+                    phase_j = pj;
+                    fmt = sc.fmt[pslot][tensor == 1 ? 1 : 0];
+                    G = &geo[fmt - 1][P.ntok - 1];
+                    const uint8_t* tbase = tensor == 1 ? sc.ptr_up[pslot] : sc.ptr[pslot];
+                    c_src = nullptr; c_stride = 0; c_dst = 0;
+                    if (lane < G->npl) {
+                        c_src = tbase + G->pl[lane] + (int64_t)P.rb * G->rbstr[lane];
+                        c_stride = G->cstr[lane];
+                        c_dst = G->woff[lane];
+                    }
+                    if (lane >= 4 && lane < 4 + 3 * P.ntok) {
+                        const int tk = (lane - 4) / 3, piece = (lane - 4) - 3 * tk;
+                        int v = P.vec[0];
+#pragma unroll
+                        for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) v = P.vec[t2];
+                        const uint8_t* qv = reinterpret_cast<const uint8_t*>(vs.q + (size_t)v * vs.q_stride);
+                        const uint8_t* sv = reinterpret_cast<const uint8_t*>(vs.st + (size_t)v * vs.st_stride);
+                        const int fam = fmt == kQ2K || fmt == kQ3K ? kF2 : fmt == kQ4K ? kF4 : kF8;
+                        const uint32_t tb = G->tok0 + tk * G->tstride;
+                        if (piece == 0) { c_src = qv + (size_t)fam * vs.nsb * 512; c_stride = 512; c_dst = tb + G->tx; }
+                        if (piece == 1 && fmt == kQ3K) {
+                            c_src = qv + (size_t)kF1 * vs.nsb * 512; c_stride = 512; c_dst = tb + G->tx1;
+                        }
+                        if (piece == 2) { c_src = sv; c_stride = kStatFloats * 4; c_dst = tb + G->ts; }
+                    }
+                }
+                const int per = G->per;
+                const int s0 = (pj - phase_j) * per, ks = min(per, p_nsb - s0);
+                const uint32_t stage = ring + slot * kStageBytes;
+                const uint32_t bytes = c_src ? (uint32_t)ks * c_stride : 0u;
+                uint32_t total = bytes;
+#pragma unroll
+                for (int off = 16; off >= 1; off >>= 1) total += __shfl_xor_sync(kFull, total, off);
+                if (lane == 0) {
+                    int4* H = reinterpret_cast<int4*>(&hdr[slot]);
+                    H[0] = make_int4(item, pj, P.nst, s0);
+                    H[1] = make_int4(ks, fmt, tensor, P.ntok);
+                    H[2] = make_int4(P.rb, P.e, P.shared, 0);
+                    H[3] = make_int4(P.asg[0], P.asg[1], P.asg[2], P.asg[3]);
+                    s_posted[slot] = p_q;
+                    mbar_arrive_tx(full, total);
+                }
+                __syncwarp();
+                if (bytes) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
+                ++p_q;
+            }
+            if (failed) { if (lane == 0) { atomicOr(A.err, kErrEmpty); s_fail = 1; } break; }
+            if (item < 0) break;
         }
-        if (sbj < H.ks) {
-            const int ntok = H.ntok;
+    } else {
+        // ============================ consumer warps =============================
+        // warp w: all 32 rows of the stage, superblocks w, w + 8, ... (Q8_0:
+        // both halves of the code pairs of each)
+        float acc[2][kDecodeTok][4];   // [0] gate (or down), [1] up; rows g + 8 i
+        float cur[kDecodeTok][4];      // the tensor being streamed
+#pragma unroll
+        for (int tk = 0; tk < kDecodeTok; ++tk)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[0][tk][i] = acc[1][tk][i] = cur[tk][i] = 0.0f;
+        int n_done = 0;   // items finished by this CTA (selects the reduction buffer and the owner warps)
+        for (int q = 0;; ++q) {
+            const int slot = q % kNST;
+            if (!mbar_wait(bar0 + 8 * slot, (q / kNST) & 1, A.err, kErrFull)) {
+                if (lane == 0) s_fail = 1;
+                break;
+            }
+            const Hdr& H = hdr[slot];
+            if (H.item < 0) break;
+            const uint32_t stage = ring + slot * kStageBytes;
+            const int fmt = H.fmt, ks = H.ks, ntok = H.ntok;
+            const Geo& GS = geo[fmt - 1][ntok - 1];
+            if (!kDown && H.tensor == 1 && H.s0 == 0) {
+                // first stage of the up tensor: the gate sums are complete
+#pragma unroll
+                for (int tk = 0; tk < kDecodeTok; ++tk)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) { acc[0][tk][i] += cur[tk][i]; cur[tk][i] = 0.0f; }
+            }
 #pragma unroll
             for (int tk = 0; tk < kDecodeTok; ++tk) {
                 if (tk >= ntok) break;
-                switch (H.fmt) {
-                case kQ2K: tile_token<kQ2K>(H, stage, sbj, half, rt, tk, cur[tk]); break;
-                case kQ3K: tile_token<kQ3K>(H, stage, sbj, half, rt, tk, cur[tk]); break;
-                case kQ4K: tile_token<kQ4K>(H, stage, sbj, half, rt, tk, cur[tk]); break;
-                default: tile_token<kQ80>(H, stage, sbj, half, rt, tk, cur[tk]); break;
+                if (fmt == kQ80) {
+                    for (int jj = warp; jj < ks; jj += kConsumers) {
+                        tile_block<kQ80>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                        tile_block<kQ80>(GS, stage, jj, 1, tk, zaddr, cur[tk]);
+                    }
+                } else if (fmt == kQ2K) {
+                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ2K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                } else if (fmt == kQ3K) {
+                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ3K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                } else {
+                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ4K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
                 }
             }
-        }
-        // fields needed after the slot is released to the producer
-        const bool item_end = H.j == H.nst - 1;
-        int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0;
-        int e_asg[kDecodeTok];
-        if (item_end) {
-            e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e;
+            // fields needed after the slot is released to the producer
+            const bool item_end = H.j == H.nst - 1;
+            int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0;
+            int e_asg[kDecodeTok];
+            if (item_end) {
+                e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e;
 #pragma unroll
-            for (int tk = 0; tk < kDecodeTok; ++tk) e_asg[tk] = H.asg[tk];
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar0 + 8 * (kNST + slot));
-        if (!item_end) continue;
+                for (int tk = 0; tk < kDecodeTok; ++tk) e_asg[tk] = H.asg[tk];
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar0 + 8 * (kNST + slot));
+            if (!item_end) continue;
 
-        // ---- item done: the streamed tensor's sums go to acc[1] (up) or acc[0]
-        const int g = lane >> 2, t4 = lane & 3;
-        const int buf = n_done & 1;
+            // ---- item done: the streamed tensor's sums go to acc[1] (up) or acc[0]
+            const int g = lane >> 2, t4 = lane & 3;
+            const int buf = n_done & 1;
 #pragma unroll
-        for (int u = 0; u < (kDown ? 1 : 2); ++u)
+            for (int u = 0; u < (kDown ? 1 : 2); ++u)
+#pragma unroll
+                for (int tk = 0; tk < kDecodeTok; ++tk)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        float v = (u == (kDown ? 0 : 1)) ? acc[u][tk][i] + cur[tk][i] : acc[u][tk][i];
+                        v += __shfl_xor_sync(kFull, v, 1);
+                        v += __shfl_xor_sync(kFull, v, 2);
+                        if (t4 == 0) red[buf][warp][u][tk][8 * i + g] = v;
+                    }
 #pragma unroll
             for (int tk = 0; tk < kDecodeTok; ++tk)
 #pragma unroll
-                for (int hl = 0; hl < 2; ++hl) {
-                    float v = (u == (kDown ? 0 : 1)) ? acc[u][tk][hl] + cur[tk][hl] : acc[u][tk][hl];
-                    v += __shfl_xor_sync(kFull, v, 1);
-                    v += __shfl_xor_sync(kFull, v, 2);
-                    if (t4 == 0) red[buf][warp][u][tk][8 * hl + g] = v;
+                for (int i = 0; i < 4; ++i) acc[0][tk][i] = acc[1][tk][i] = cur[tk][i] = 0.0f;
+            consumer_sync();
+            // the finishing work of token tk goes to warp (n_done + tk) % kConsumers
+            const int tk = (warp - n_done % kConsumers + kConsumers) % kConsumers;
+            if (tk < e_ntok) {
+                int a = e_asg[0];
+#pragma unroll
+                for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) a = e_asg[t2];
+                // lane = row of the 32-row block
+                float v0 = 0.0f, v1 = 0.0f;
+#pragma unroll
+                for (int c2 = 0; c2 < kConsumers; ++c2) {
+                    v0 += red[buf][c2][0][tk][lane];
+                    if (!kDown) v1 += red[buf][c2][1][tk][lane];
                 }
-#pragma unroll
-        for (int tk = 0; tk < kDecodeTok; ++tk) {
-            acc[0][tk][0] = acc[0][tk][1] = acc[1][tk][0] = acc[1][tk][1] = 0.0f;
-            cur[tk][0] = cur[tk][1] = 0.0f;
-        }
-        consumer_sync();
-        // the finishing work of token tk goes to warp (n_done + tk) % kConsumers
-        const int tk = (warp - n_done % kConsumers + kConsumers) % kConsumers;
-        if (tk < e_ntok) {
-            int a = e_asg[0];
-#pragma unroll
-            for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) a = e_asg[t2];
-            // lane = row of the 32-row block: row tile lane/16, row lane%16
-            const int ort = lane >> 4, rr = lane & 15;
-            float v0 = 0.0f, v1 = 0.0f;
-#pragma unroll
-            for (int sb = 0; sb < kConsumers / 2; ++sb) {
-                v0 += red[buf][2 * sb + ort][0][tk][rr];
-                if (!kDown) v1 += red[buf][2 * sb + ort][1][tk][rr];
+                if (kDown) {
+                    A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
+                } else {
+                    // SwiGLU (routing weight folded in), then prepare h for the down projection
+                    const float w = e_shared ? 1.0f : A.wts[a];
+                    const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
+                    const int fam = families_of(tab.fmt[e_e][2]);
+                    __half* hq = A.hq + (size_t)a * 4 * A.nsbi * 256;
+                    float* hs = A.hs + (size_t)a * A.nsbi * kStatFloats;
+                    prep_block32(hv, e_rb, fam, hq, hs, A.nsbi);
+                    const int n_rb = d.I / 32;
+                    if (e_rb == n_rb - 1)
+                        for (int jb = n_rb; jb < 8 * A.nsbi; ++jb) prep_block32(0.0f, jb, fam, hq, hs, A.nsbi);
+                }
             }
-            if (kDown) {
-                A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
-            } else {
-                // SwiGLU (routing weight folded in), then prepare h for the down projection
-                const float w = e_shared ? 1.0f : A.wts[a];
-                const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
-                const int fam = families_of(tab.fmt[e_e][2]);
-                __half* hq = A.hq + (size_t)a * 4 * A.nsbi * 256;
-                float* hs = A.hs + (size_t)a * stat_off(A.nsbi).total;
-                prep_block32(hv, e_rb, fam, hq, hs, A.nsbi);
-                const int n_rb = d.I / 32;
-                if (e_rb == n_rb - 1)
-                    for (int jb = n_rb; jb < 8 * A.nsbi; ++jb) prep_block32(0.0f, jb, fam, hq, hs, A.nsbi);
-            }
+            // no barrier here: the next item end writes the other reduction buffer,
+            // and its barrier orders these reads before the buffer is reused
+            ++n_done;
         }
-        // no barrier here: the next item end writes the other reduction buffer,
-        // and its barrier orders these reads before the buffer is reused
-        ++n_done;
     }
-#undef MQ_PRODUCE_ONE
     // After a wait ran out, wait (bounded) for the copies still in flight into
-    // each slot before the CTA exits.  Normally every posted stage has been
-    // consumed, so nothing is in flight.
-    if (warp == kProducerWarp) {
-        __syncwarp();
-        if (p_failed && lane < kNST && s_posted[lane] >= 0)
-            mbar_wait(bar0 + 8 * lane, (s_posted[lane] / kNST) & 1, A.err, kErrFull);
-    }
+    // each slot before the CTA exits.  Without a failure every posted stage
+    // has been consumed, so nothing is in flight.
+    __syncthreads();
+    if (warp == kProducerWarp && s_fail && lane < kNST && s_posted[lane] >= 0)
+        mbar_wait(bar0 + 8 * lane, (s_posted[lane] / kNST) & 1, A.err, kErrFull);
 }
 
 // out[t] = sum of the token's routed expert outputs in slot order, then the

@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     // segment (blocks past the hidden size, up to the 256 padding, are zero).
     if (xq != nullptr) {
         const int nsb = (H + 255) / 256;
-        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)stat_off(nsb).total;
+        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)nsb * kStatFloats;
         for (int j = 0; j < kTok; ++j) {
             const int t = t0 + j;
             if (t >= T) break;

@@ -77,9 +77,9 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_perm = take(TK * 4), o_inv = take(TK * 4);
     const size_t o_act = take((size_t)(d.E + 2) * 4);
     const size_t o_xq = take((size_t)d.T * 4 * nsbx * 256 * 2);
-    const size_t o_xs = take((size_t)d.T * stat_off((int)nsbx).total * 4);
+    const size_t o_xs = take((size_t)d.T * nsbx * kStatFloats * 4);
     const size_t o_hq = take(A * 4 * nsbi * 256 * 2);
-    const size_t o_hs = take(A * stat_off((int)nsbi).total * 4);
+    const size_t o_hs = take(A * nsbi * kStatFloats * 4);
     const size_t o_pdn = take(A * d.H * 4);
     const size_t o_plan = take(sizeof(Plan));
     const size_t cnt_bytes = decode_counter_bytes(d);
