@@ -227,7 +227,6 @@ def run_native(args):
     clocks = ClockSampler(local)
     clocks.start()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    layer.mq.mq_profile_enable(K * 8)
     barrier()
     t_wall0 = time.perf_counter()
     for i in range(K):
@@ -237,8 +236,16 @@ def run_native(args):
         evs[i][1].record()
     barrier()
     t_wall = time.perf_counter() - t_wall0
-    kstats = layer.mq.mq_profile_collect()
     clk = clocks.stop()
+    # Per-kernel durations: the same K steps once more with a CUDA event pair
+    # around every kernel on the launching stream (kept out of the timed
+    # region above, where the events would add gaps between the kernels).
+    layer.mq.mq_profile_enable(K * 8)
+    for i in range(K):
+        flush.fill_(i)
+        layer.forward(x_dev[W + i], idx_all[W + i])
+    barrier()
+    kstats = layer.mq.mq_profile_collect()
     dev_ms = sum(a.elapsed_time(b) for a, b in evs)
     t = torch.tensor([dev_ms], dtype=torch.float64, device="cuda")
     if world > 1:

@@ -4,23 +4,26 @@
 //
 // Dequant-fused GEMV on the legacy tensor-core path (mma.sync m16n8k16,
 // fp16 x fp16 -> fp32):
-//   A (16 rows x 16 k) = weight codes as fp16 "1024 + s*q" built with one
-//     LOP3 per code pair straight from the packed words (s = a positional
-//     power of two, so most pairs need no shift);
+//   A (16 rows x 16 k) = weight codes read straight from the packed words:
+//     one AND per code pair leaves the code in the mantissa of an fp16
+//     subnormal (value code * 2^(s-24), s a positional power of two that the
+//     activation carries inverted);
 //   B (16 k x 8 cols) = the prepared activation (mq_actprep.cuh), column n
-//     carrying sub-block n of the 256-weight superblock and zero elsewhere;
+//     carrying sub-block n of an 8-sub-block group and zero elsewhere, fixed
+//     per lane so nothing is masked in the loop;
 //   D (16 rows x 8 cols) = per-(row, sub-block) partial dot products, so the
-//     sub-block scales and mins are applied once per 16x256 tile in fp32.
-// Work is cut into items (32 rows x 16 superblocks of one tensor of one
-// expert x up to 4 tokens) taken from a global counter by one persistent CTA
-// per SM.  The packed layout keeps any superblock range of a 32-row tile
-// contiguous in every plane, so a producer warp streams each item through a
-// 5-stage shared-memory ring with 1D bulk (TMA) copies that complete on
-// mbarriers; 8 consumer warps (2 row tiles x 4 superblocks per stage) run
-// the tensor-core math.  Item partial sums go to scratch; the last CTA to
-// finish a row block combines them in a fixed order (SwiGLU for gate/up,
-// routed + shared sum for down), so the results are deterministic.  Every
-// wait on an mbarrier is bounded (about 1 s) and reports to an error word.
+//     sub-block scales and mins are applied once per tile in fp32.
+// Work is cut into items (32 rows x all superblocks of one tensor (gate and
+// up together) of one expert x up to 4 tokens); CTA c of the persistent grid
+// (one CTA per SM) takes items c, c + grid, ...  The packed layout keeps any
+// superblock range of a 32-row tile contiguous in every plane, so a
+// dedicated producer warp streams each item through a 3-slot shared-memory
+// ring with 1D bulk (TMA) copies that complete on mbarriers; 8 consumer warps
+// (all 32 rows x every 8th superblock of a stage each) run the tensor-core
+// math.  At the end of an item the CTA reduces its warps' sums in a fixed
+// order (SwiGLU and the prepared h for gate/up, one partial output row block
+// per assignment for down), so results are deterministic.  Every wait on an
+// mbarrier is bounded (about 1 s) and reports to an error word.
 #include <cuda_fp16.h>
 
 #include "mq_actprep.cuh"
@@ -464,6 +467,8 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
 template <bool kDown>
 __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant__ ExpertTab tab,
                                                           const __grid_constant__ DecodeArgs A) {
+    pdl_wait();
+    pdl_launch();
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
@@ -534,7 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 
     if (warp == kProducerWarp) {
         // ===================== producer (dedicated warp) =====================
-        // Per phase (one tensor of one item) every lane owns at most one copy:
+        // The CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...  Per
+        // phase (one tensor of one item) every lane owns at most one copy:
         // lanes 0..3 a weight plane, lanes 4.. one piece of one token (family
         // fragments, Q3_K high-bit fragments, statistics).  A stage then only
         // advances the source by the stage's first superblock.
@@ -542,17 +548,12 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                                 : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
         int p_cursor = 0, p_q = 0;
         const int p_nsb = vs.nsb;
-        int next_id = 0;
-        if (lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);
         ItemDesc P;
         int pslot = 0;
-        for (;;) {
-            const int id = __shfl_sync(kFull, next_id, 0);
+        for (int k = 0;; ++k) {
+            const int id = blockIdx.x + k * gridDim.x;
             const int item = id < n_items ? id : -1;
-            if (item >= 0) {
-                decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
-                if (lane == 0) next_id = (int)atomicAdd(&A.next[kDown ? 1 : 0], 1u);
-            }
+            if (item >= 0) decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
             const int nst = item >= 0 ? P.nst : 1;
             bool failed = false;
             // this lane's copy for the current phase (one tensor of the item)
@@ -744,6 +745,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 // out[t] = sum of the token's routed expert outputs in slot order, then the
 // shared expert (deterministic order; routing weights are folded into h)
 __global__ void combine_kernel(Dims d, const float* __restrict__ pdn, float* __restrict__ out) {
+    pdl_wait();
+    pdl_launch();
     const int r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= d.H) return;
     for (int t = blockIdx.y; t < d.T; t += gridDim.y) {
@@ -786,19 +789,18 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.err = w.err;
     A.out = out;
     prof_begin("gateup_mma", s);
-    ffn_kernel<false><<<g_num_sms, kThreads, smem, s>>>(tab, A);
+    cudaError_t err = launch_pdl(ffn_kernel<false>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
-    cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     prof_begin("down_mma", s);
-    ffn_kernel<true><<<g_num_sms, kThreads, smem, s>>>(tab, A);
+    err = launch_pdl(ffn_kernel<true>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
-    err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     prof_begin("combine", s);
-    combine_kernel<<<dim3((d.H + 255) / 256, d.T < 8 ? d.T : 8), 256, 0, s>>>(d, w.pdn, out);
+    err = launch_pdl(combine_kernel, dim3((d.H + 255) / 256, d.T < 8 ? d.T : 8), dim3(256), 0, s, d,
+                     (const float*)w.pdn, out);
     prof_end(s);
-    return cudaGetLastError();
+    return err;
 }
 
 }  // namespace mq

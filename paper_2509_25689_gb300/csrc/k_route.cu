@@ -36,7 +36,13 @@ constexpr int kTok = 8;
 __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
                                                              const float* __restrict__ W, int H, int T,
                                                              int E, float* __restrict__ z,
-                                                             __half* __restrict__ xq, float* __restrict__ xs) {
+                                                             __half* __restrict__ xq, float* __restrict__ xs,
+                                                             uint32_t* __restrict__ zero_words, int n_zero) {
+    pdl_wait();
+    pdl_launch();
+    // per-call words that must start at zero (work counters, error word)
+    if (blockIdx.x == 0 && blockIdx.y == 0)
+        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
     __shared__ float part[32][kTok];
     const int e = blockIdx.x, t0 = blockIdx.y * kTok;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -128,45 +134,46 @@ __device__ __forceinline__ float canonical_sigmoid(float z) {
     return __fdiv_rn(1.0f, __fadd_rn(1.0f, ex));
 }
 
-// (value, index) argmax: larger value wins, equal values -> lower index
-__device__ __forceinline__ void better(float& v, int& i, float v2, int i2) {
-    if (i2 >= 0 && (i < 0 || v2 > v || (v2 == v && i2 < i))) { v = v2; i = i2; }
+// Order-preserving map of a finite fp32 value to uint32 (0 is below every
+// finite value and marks "not available").
+__device__ __forceinline__ uint32_t ord_key(float f) {
+    const uint32_t b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
-__device__ __forceinline__ int warp_argmax(float v, int i) {
-#pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-        const float v2 = __shfl_xor_sync(kFull, v, off);
-        const int i2 = __shfl_xor_sync(kFull, i, off);
-        better(v, i, v2, i2);
-    }
-    return i;
+// Warp argmax over one candidate per lane: largest key, then lowest index.
+__device__ __forceinline__ int warp_argmax_key(uint32_t key, int idx) {
+    const uint32_t kmax = __reduce_max_sync(kFull, key);
+    return (int)__reduce_min_sync(kFull, key == kmax ? (uint32_t)idx : 0xffffffffu);
 }
 
 // One warp routes one token.  Lane l holds experts l, l+32, ... (E <= 256).
 // uw: per-warp scratch of E floats; g_sh: per-warp scratch of G floats.
-__device__ __forceinline__ void route_token(const float* __restrict__ z, const float* __restrict__ bias, const Dims& d,
-                                            int t, float* uw, float* g_sh, int32_t* __restrict__ idx,
-                                            float* __restrict__ wts) {
+__device__ __forceinline__ void route_token(const float* __restrict__ z, const float* __restrict__ bias, int E,
+                                            int G, int Gk, int K, float routed_scale, int t, float* uw,
+                                            float* g_sh, int32_t* __restrict__ idx, float* __restrict__ wts) {
     const int lane = threadIdx.x & 31;
-    const int E = d.E, G = d.G, gs = E / G;
+    const int gs = E / G;
     float s[8], u[8];
+    int grp[8];
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
         const int e = lane + 32 * m;
-        s[m] = 0.0f; u[m] = -INFINITY;
+        s[m] = 0.0f; u[m] = 0.0f; grp[m] = 0;
         if (e < E) {
             s[m] = canonical_sigmoid(z[(size_t)t * E + e]);
             u[m] = __fadd_rn(s[m], bias ? bias[e] : 0.0f);
+            grp[m] = e / gs;
+            uw[e] = u[m];
         }
     }
-    // group score = sum of the two largest u of the group (scan in index order)
-#pragma unroll
-    for (int m = 0; m < 8; ++m) if (lane + 32 * m < E) uw[lane + 32 * m] = u[m];
     __syncwarp();
+    // group score = sum of the two largest u of the group (scan in index order)
     for (int g = lane; g < G; g += 32) {
         float top1 = -INFINITY, top2 = -INFINITY;
+        const float* ug = uw + g * gs;
+#pragma unroll 8
         for (int i = 0; i < gs; ++i) {
-            const float v = uw[g * gs + i];
+            const float v = ug[i];
             if (v > top1) { top2 = top1; top1 = v; }
             else if (v > top2) top2 = v;
         }
@@ -175,44 +182,43 @@ __device__ __forceinline__ void route_token(const float* __restrict__ z, const f
     __syncwarp();
     // keep topk_group groups: repeated argmax, ties to the lower index
     uint64_t kept = 0;
-    float gv0 = lane < G ? g_sh[lane] : 0.0f, gv1 = lane + 32 < G ? g_sh[lane + 32] : 0.0f;
-    for (int r = 0; r < d.Gk; ++r) {
-        float bv = 0.0f; int bi = -1;
-        if (lane < G && !((kept >> lane) & 1)) better(bv, bi, gv0, lane);
-        if (lane + 32 < G && !((kept >> (lane + 32)) & 1)) better(bv, bi, gv1, lane + 32);
-        bi = warp_argmax(bv, bi);
-        kept |= 1ull << bi;
+    const uint32_t gk0 = lane < G ? ord_key(g_sh[lane]) : 0u;
+    const uint32_t gk1 = lane + 32 < G ? ord_key(g_sh[lane + 32]) : 0u;
+    for (int r = 0; r < Gk; ++r) {
+        uint32_t k = 0u;
+        int i = 0x7fffffff;
+        if (lane < G && !((kept >> lane) & 1)) { k = gk0; i = lane; }
+        if (lane + 32 < G && !((kept >> (lane + 32)) & 1) && gk1 > k) { k = gk1; i = lane + 32; }
+        kept |= 1ull << warp_argmax_key(k, i);
     }
     // top_k experts by u among the kept groups, descending, ties to the lower id
-    uint32_t avail = 0;
+    uint32_t key[8];
 #pragma unroll
-    for (int m = 0; m < 8; ++m) {
-        const int e = lane + 32 * m;
-        if (e < E && ((kept >> (e / gs)) & 1)) avail |= 1u << m;
-    }
+    for (int m = 0; m < 8; ++m) key[m] = (lane + 32 * m < E && ((kept >> grp[m]) & 1)) ? ord_key(u[m]) : 0u;
     int sel = 0;
     float ssum = 0.0f, mys = 0.0f;
-    for (int j = 0; j < d.K; ++j) {
-        float bv = 0.0f; int bi = -1;
+    for (int j = 0; j < K; ++j) {
+        uint32_t bk = 0u;
+        int bm = 0;
 #pragma unroll
-        for (int m = 0; m < 8; ++m) if ((avail >> m) & 1) better(bv, bi, u[m], lane + 32 * m);
-        bi = warp_argmax(bv, bi);
+        for (int m = 0; m < 8; ++m)
+            if (key[m] > bk) { bk = key[m]; bm = m; }   // strict: the lower expert id wins a tie
+        const int bi = warp_argmax_key(bk, lane + 32 * bm);
         float win = 0.0f;
         if ((bi & 31) == lane) {
             const int m = bi >> 5;
-            avail &= ~(1u << m);
-            win = s[0];
 #pragma unroll
-            for (int mm = 1; mm < 8; ++mm) if (mm == m) win = s[mm];
+            for (int mm = 0; mm < 8; ++mm)
+                if (mm == m) { key[mm] = 0u; win = s[mm]; }
         }
         const float sv = __shfl_sync(kFull, win, bi & 31);
         ssum = __fadd_rn(ssum, sv);   // slot order, identical on every lane
         if (lane == j) { sel = bi; mys = sv; }   // lane j keeps slot j
     }
     // weights: s_j / sum(s), summed in slot order, times routed_scale
-    if (lane < d.K) {
-        idx[(size_t)t * d.K + lane] = sel;
-        wts[(size_t)t * d.K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), d.routed_scale);
+    if (lane < K) {
+        idx[(size_t)t * K + lane] = sel;
+        wts[(size_t)t * K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), routed_scale);
     }
 }
 
@@ -224,20 +230,24 @@ __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __re
                                                                float* __restrict__ wts) {
     __shared__ float u_sh[kTopkWarps][kMaxExperts];
     __shared__ float g_sh[kTopkWarps][kMaxGroups];
+    pdl_wait();
+    pdl_launch();
     const int w = threadIdx.x >> 5;
     const int t = blockIdx.x * kTopkWarps + w;
     if (t >= d.T) return;
-    route_token(z, bias, d, t, u_sh[w], g_sh[w], idx, wts);
+    route_token(z, bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, u_sh[w], g_sh[w], idx, wts);
 }
 
 // ---------------------------------------------------------------------------
 // permutation: one CTA; stable counting sort of entries a = t*K + j by expert
 // ---------------------------------------------------------------------------
-constexpr int kPermThreads = 1024;
+constexpr int kPermThreads = 512;
 constexpr int kPermWarps = kPermThreads / 32;
 
 // With `z` given, the same CTA first routes every token (one warp per token,
-// decode-sized batches) and then permutes.
+// decode-sized batches) and then permutes.  Offsets and the active list are
+// kept in shared memory as well, so nothing written here is read back from
+// global memory.
 __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restrict__ idx, Dims d,
                                                                int32_t* __restrict__ offsets,
                                                                int32_t* __restrict__ perm,
@@ -247,14 +257,18 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
                                                                const float* __restrict__ z,
                                                                const float* __restrict__ bias,
                                                                float* __restrict__ wts) {
+    pdl_wait();
+    pdl_launch();
     const int n = d.T * d.K, E = d.E;
     __shared__ int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
-    __shared__ int32_t total[kMaxExperts + 1];
+    __shared__ int32_t s_off[kMaxExperts + 1];
+    __shared__ int32_t s_act[kMaxExperts + 1];
     __shared__ float g_sh[kPermWarps][kMaxGroups];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (z != nullptr) {
         for (int t = warp; t < d.T; t += kPermWarps)
-            route_token(z, bias, d, t, reinterpret_cast<float*>(cnt[warp]), g_sh[warp], idx, wts);
+            route_token(z, bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
+                        g_sh[warp], idx, wts);
         __syncthreads();
     }
     for (int i = threadIdx.x; i < kPermWarps * kMaxExperts; i += kPermThreads) (&cnt[0][0])[i] = 0;
@@ -267,8 +281,9 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
     if (threadIdx.x < E) {
         const int e = threadIdx.x;
         int run = 0;
+#pragma unroll
         for (int wv = 0; wv < kPermWarps; ++wv) { const int c = cnt[wv][e]; cnt[wv][e] = run; run += c; }
-        total[e] = run;
+        s_off[e] = run;
     }
     __syncthreads();
     if (warp == 0) {
@@ -277,7 +292,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             const int e = lane * 8 + q;
-            local[q] = e < E ? total[e] : 0;
+            local[q] = e < E ? s_off[e] : 0;
             sum += local[q];
         }
         int incl = sum;
@@ -287,18 +302,19 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
             if (lane >= off) incl += v;
         }
         int run = incl - sum;
+        __syncwarp();
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             const int e = lane * 8 + q;
-            if (e < E) { offsets[e] = run; total[e] = run; }
+            if (e < E) { offsets[e] = run; s_off[e] = run; }
             run += local[q];
         }
-        if (lane == 31) { offsets[E] = run; }
+        if (lane == 31) { offsets[E] = run; s_off[E] = run; }
     }
     __syncthreads();
     for (int i = threadIdx.x; i < kPermWarps * E; i += kPermThreads) {
-        const int wv = i / E, e = i % E;
-        cnt[wv][e] += total[e];
+        const int wv = i / E, e = i - wv * E;
+        cnt[wv][e] += s_off[e];
     }
     __syncthreads();
     // stable scatter: each warp walks its segment in order, 32 entries a step
@@ -317,14 +333,13 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         if (ok && rank == 0) cnt[warp][e] += __popc(peers);
         __syncwarp();
     }
-    __syncthreads();
     // active expert list (ascending ids), active[0] = count
     if (warp == 0) {
         int flags = 0, c = 0;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             const int e = lane * 8 + q;
-            const int f = (e < E && offsets[e + 1] > offsets[e]) ? 1 : 0;
+            const int f = (e < E && s_off[e + 1] > s_off[e]) ? 1 : 0;
             flags |= f << q;
             c += f;
         }
@@ -337,14 +352,14 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         int pos = incl - c;
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (flags & (1 << q)) active[1 + pos++] = lane * 8 + q;
-        if (lane == 31) active[0] = incl;
+            if (flags & (1 << q)) { active[1 + pos] = lane * 8 + q; s_act[1 + pos] = lane * 8 + q; ++pos; }
+        if (lane == 31) { active[0] = incl; s_act[0] = incl; }
     }
     if (plan == nullptr) return;
     __syncthreads();
     // decode work plan: items per expert slot (shared expert first)
     if (warp == 0) {
-        const int n_slots = active[0] + d.has_shared;
+        const int n_slots = s_act[0] + d.has_shared;
         int cg[9], cd[9], sg = 0, sd = 0, tgs = 0, tgmax = 0;
 #pragma unroll
         for (int q = 0; q < 9; ++q) {
@@ -352,7 +367,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
             int ntok = 0;
             if (p < n_slots) {
                 if (p < d.has_shared) ntok = d.T;
-                else { const int e = active[1 + p - d.has_shared]; ntok = offsets[e + 1] - offsets[e]; }
+                else { const int e = s_act[1 + p - d.has_shared]; ntok = s_off[e + 1] - s_off[e]; }
             }
             const int ntg = (ntok + kDecodeTok - 1) / kDecodeTok;
             cg[q] = (d.I / 32) * ntg;     // gate/up items: 32 rows x both tensors x full K
@@ -388,41 +403,45 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 }  // namespace
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 cudaStream_t s) {
+                                 uint32_t* zero_words, int n_zero, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
     dim3 grid(d.E, (d.T + kTok - 1) / kTok);
     prof_begin("router_logits", s);
-    router_logits_kernel<<<grid, nseg * 32, 0, s>>>(x, W, d.H, d.T, d.E, z, xq, xs);
+    const cudaError_t e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq,
+                                     xs, zero_words, n_zero);
     prof_end(s);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                         cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     prof_begin("router_topk", s);
-    topk_kernel<<<(d.T + kTopkWarps - 1) / kTopkWarps, kTopkWarps * 32, 0, s>>>(z, bias, d, idx, wts);
+    const cudaError_t e = launch_pdl(topk_kernel, dim3((d.T + kTopkWarps - 1) / kTopkWarps), dim3(kTopkWarps * 32),
+                                     0, s, z, bias, d, idx, wts);
     prof_end(s);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, Plan* plan, cudaStream_t s) {
     prof_begin("permute", s);
-    permute_kernel<<<1, kPermThreads, 0, s>>>(const_cast<int32_t*>(idx), d, offsets, perm, inv, active, plan,
-                                               nullptr, nullptr, nullptr);
+    const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, const_cast<int32_t*>(idx), d,
+                                     offsets, perm, inv, active, plan, (const float*)nullptr, (const float*)nullptr,
+                                     (float*)nullptr);
     prof_end(s);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                                  int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
                                  cudaStream_t s) {
     prof_begin("route_permute", s);
-    permute_kernel<<<1, kPermThreads, 0, s>>>(idx, d, offsets, perm, inv, active, plan, z, bias, wts);
+    const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, idx, d, offsets, perm, inv,
+                                     active, plan, z, bias, wts);
     prof_end(s);
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace mq

@@ -83,8 +83,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_pdn = take(A * d.H * 4);
     const size_t o_plan = take(sizeof(Plan));
     const size_t cnt_bytes = decode_counter_bytes(d);
-    const size_t o_cnt = take(cnt_bytes);
-    const size_t o_err = take(4);
+    const size_t o_cnt = take(cnt_bytes + 4);   // work counters, then the error word (zeroed per call)
+    const size_t o_err = o_cnt + cnt_bytes;
     if (w && base) {
         char* b = static_cast<char*>(base);
         w->z = reinterpret_cast<float*>(b + o_z);
@@ -103,6 +103,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
         w->counter_bytes = cnt_bytes;
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
+        w->zero_words = w->counters;
+        w->n_zero = (int)((cnt_bytes + 4) / 4);
     }
     return at;
 }
@@ -174,7 +176,7 @@ int check_common(const mq_layer_cfg* cfg, int32_t T, const void* x, const float*
 int run_route(const Dims& d, const void* x, const float* router_w, const float* bias, Work& w,
               cudaStream_t s, bool prep_tokens) {
     if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, prep_tokens ? w.xq : nullptr, w.xs,
-                             s) != cudaSuccess)
+                             prep_tokens ? w.zero_words : nullptr, prep_tokens ? w.n_zero : 0, s) != cudaSuccess)
         return MQ_ECUDA;
     if (d.T <= kFusedRouteTokens) {
         // decode-sized batch: top-k, permutation and work plan in one CTA
@@ -237,8 +239,6 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     workspace_plan(d, workspace, &w);
     if (topk_idx) w.idx = topk_idx;
     if (topk_w) w.wts = topk_w;
-    if (cudaMemsetAsync(w.counters, 0, w.counter_bytes, s) != cudaSuccess) return MQ_ECUDA;
-    if (cudaMemsetAsync(w.err, 0, 4, s) != cudaSuccess) return MQ_ECUDA;
     rc = run_route(d, x, router_w, bias, w, s, true);
     if (rc != MQ_OK) return rc;
     (void)path_mode();

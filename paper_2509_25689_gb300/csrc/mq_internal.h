@@ -50,19 +50,47 @@ struct Work {
     int32_t* active;   // [E + 2]: active[0] = count, active[1..] = expert ids
     Plan* plan;        // decode work plan
     __half* xq;        // [T][4][nsb(H)*256] prepared token activations (fp16 fragments)
-    float* xs;         // [T][80*nsb(H)] their statistics
+    float* xs;         // [T][32*nsb(H)] their statistics
     __half* hq;        // [A][4][nsb(I)*256] prepared SwiGLU outputs, A = T*K + T
-    float* hs;         // [A][80*nsb(I)]
+    float* hs;         // [A][32*nsb(I)]
     float* pdn;        // [A][H] down outputs per assignment (combined by a last pass)
     uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
     size_t counter_bytes;
     uint32_t* err;     // device error word (bounded waits that ran out)
+    uint32_t* zero_words; // counters + error word, cleared by the first kernel of a call
+    int n_zero;
 };
 
 size_t workspace_plan(const Dims& d, void* base, Work* w);
 
 // launch helpers; each returns cudaGetLastError() of its launch
+// Programmatic dependent launch: every kernel of the layer is launched with
+// programmatic stream serialization, waits for its predecessor's results
+// with pdl_wait() before touching global memory, and lets its successor be
+// scheduled early with pdl_launch().
+#ifdef __CUDACC__
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+#endif
+
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
+                                 uint32_t* zero_words, int n_zero,
                                  cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
