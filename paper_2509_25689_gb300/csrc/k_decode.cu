@@ -796,9 +796,13 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     err = launch_pdl(ffn_kernel<true>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
+    return launch_combine(d, w.pdn, out, s);
+}
+
+cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s) {
     prof_begin("combine", s);
-    err = launch_pdl(combine_kernel, dim3((d.H + 255) / 256, d.T < 8 ? d.T : 8), dim3(256), 0, s, d,
-                     (const float*)w.pdn, out);
+    const cudaError_t err = launch_pdl(combine_kernel, dim3((d.H + 255) / 256, d.T < 8 ? d.T : 8), dim3(256), 0, s,
+                                       d, pdn, out);
     prof_end(s);
     return err;
 }

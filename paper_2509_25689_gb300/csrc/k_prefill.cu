@@ -1,0 +1,432 @@
+// Expert FFN for prefill-sized batches: a grouped GEMM per expert on the
+// 5th-generation tensor cores (arXiv 2509.25689 Fig. 1 layer; expert tensors
+// in their own k-quant style formats, Sec. 3.3).
+//
+// Work unit = (expert slot, 128 weight rows, up to 256 of the slot's tokens).
+// The MMA is tcgen05.mma.cta_group::1.kind::f16 with M = 128 weight rows,
+// N = the unit's tokens (rounded up to 16) and K in steps of 16, fp32
+// accumulators in tensor memory (gate and up side by side for gate/up units).
+// Per 64-wide K chunk the CTA's 128 threads dequantize their weight row of
+// each tensor straight from the packed planes into fp16 (one row per thread,
+// fp16 keeps 11 significant bits of the decoded weight), and gather the
+// unit's activation rows (fp16 tokens, or the fp16 SwiGLU output h) with
+// cp.async into a 3-slot ring; thread 0 issues the MMAs of a chunk and
+// commits them to that slot's mbarrier while the threads prepare the next
+// chunks.  Operands sit in shared memory in the canonical K-major layout
+// without swizzle: 8 x 8 fp16 core matrices, 16 bytes per row, rows of a core
+// matrix contiguous, core matrices 128 bytes apart along M/N and
+// (rows x 16) bytes apart along K.
+// Epilogue (tcgen05.ld, lane = weight row): gate/up -> h = silu(g) * u * w
+// stored as fp16 per assignment; down -> one fp32 partial output row block
+// per assignment, summed in slot order by the combine kernel.
+// Every mbarrier wait is bounded (about 1 s) and reports to the error word;
+// tensor memory is released on every exit path.
+#include <cuda_fp16.h>
+
+#include "mq_internal.h"
+
+namespace mq {
+namespace {
+
+constexpr int kPThreads = 128;                 // 4 warps = the 4 TMEM lane quarters
+constexpr int kMT = 128;                       // weight rows per unit (MMA M)
+constexpr int kNT = 256;                       // tokens per unit (largest MMA N)
+constexpr int kKC = 64;                        // K per ring slot
+constexpr int kPSlots = 3;
+constexpr int kABytes = kMT * kKC * 2;         // one weight chunk, 16 KB
+constexpr int kBBytes = kNT * kKC * 2;         // one activation chunk, 32 KB
+constexpr int kSlotBytes = 2 * kABytes + kBBytes;
+constexpr uint32_t kErrMma = 4u;
+
+struct PrefillArgs {
+    Dims d;
+    const int32_t* offsets; const int32_t* perm; const int32_t* active; const float* wts;
+    const __half* x16;       // [T][H] tokens in fp16
+    __half* h16;             // [A][I] SwiGLU outputs (routing weight folded in)
+    float* pdn;              // [A][H]
+    uint32_t* err;
+};
+
+struct PSlots {
+    int32_t first[kMaxExperts + 1], ntot[kMaxExperts + 1], pre[kMaxExperts + 2];
+    const uint8_t* ptr[kMaxExperts + 1][2];
+    uint8_t fmt[kMaxExperts + 1][2];
+};
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (;;) {
+        if (mbar_try(bar, parity)) return true;
+        if (global_ns() - t0 > 1000000000ull) return false;
+    }
+}
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
+}
+// kind::f16 instruction descriptor: fp16 A and B, fp32 D, both K-major
+__device__ __forceinline__ uint32_t idesc_f16(int M, int N) {
+    return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_f16(uint32_t dtmem, uint64_t da, uint64_t db, uint32_t idesc, uint32_t acc) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+                 ::"r"(dtmem), "l"(da), "l"(db), "r"(idesc), "r"(acc) : "memory");
+}
+__device__ __forceinline__ void sts128(uint32_t a, uint32_t x, uint32_t y, uint32_t z, uint32_t w) {
+    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
+}
+__device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
+__device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
+__device__ __forceinline__ uint32_t ldg32(const uint8_t* p) { return __ldg(reinterpret_cast<const unsigned int*>(p)); }
+__device__ __forceinline__ uint4 ldg128(const uint8_t* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+__device__ __forceinline__ float ldgh(const uint8_t* p) {
+    return __half2float(__ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p))));
+}
+__device__ __forceinline__ uint32_t sub4(uint4 v, int i) { return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w; }
+
+// fp16 pair "1024 + c" for the two codes at bit offset s of each 16-bit half
+__device__ __forceinline__ __half2 code_pair(uint32_t w, int s, uint32_t mask) {
+    return u2h(((w >> s) & mask) | 0x64006400u);
+}
+
+// Row r of the unit, 64-wide chunk c of the contraction: decode the 64
+// weights of one tensor to fp16 and store them as 8 core-matrix rows.
+// Decoded values follow the format definitions of include/moeq.h; the
+// per-sub-block products d*sc and dmin*m are rounded to fp16 once.
+__device__ __forceinline__ void dequant_chunk(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R, int c,
+                                              uint32_t dst) {
+    const __half2 k1024 = __float2half2_rn(1024.0f);
+    if (fmt == kQ80) {
+#pragma unroll
+        for (int bb = 0; bb < 2; ++bb) {
+            const int64_t b = 2 * c + bb;
+            const float dv = ldgh(rec_ptr(base + L.plane[0], L, 2, R, b));
+            const __half2 d2 = __float2half2_rn(dv);
+            const uint8_t* cp = rec_ptr(base + L.plane[1], L, 32, R, b);
+            const uint4 w0 = ldg128(cp), w1 = ldg128(cp + 16);
+            const __half2 k1152 = __float2half2_rn(1152.0f);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {   // core-matrix row kc = 4 bb + q: pairs m = 4q .. 4q+3
+                uint32_t o[4];
+#pragma unroll
+                for (int mm = 0; mm < 4; ++mm) {
+                    const int m = 4 * q + mm;
+                    const uint32_t w = sub4(m < 8 ? w0 : w1, (m >> 1) & 3);
+                    o[mm] = h2u(__hmul2(d2, __hsub2(code_pair(w, 8 * (m & 1), 0x00FF00FFu), k1152)));
+                }
+                sts128(dst + ((4 * bb + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+            }
+        }
+        return;
+    }
+    const int64_t s = c >> 2;
+    const int cc = c & 3;
+    const float d = ldgh(rec_ptr(base + L.plane[0], L, 2, R, s));
+    if (fmt == kQ4K) {
+        const float dmin = ldgh(rec_ptr(base + L.plane[1], L, 2, R, s));
+        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 12, R, s);
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+            const int j = 2 * cc + jj;
+            int sc, mn;
+            q4_fields(sp, j, sc, mn);
+            const __half2 a2 = __float2half2_rn(d * (float)sc), nb2 = __float2half2_rn(-(dmin * (float)mn));
+            const uint4 w = ldg128(rec_ptr(base + L.plane[3], L, 128, R, s) + (j >> 2) * (kRowTile * 64) +
+                                   16 * (j & 3));
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint32_t o[4];
+#pragma unroll
+                for (int mm = 0; mm < 4; ++mm) {
+                    const int m = 4 * q + mm;
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(sub4(w, m >> 2), 4 * (m & 3), 0x000F000Fu), k1024), nb2));
+                }
+                sts128(dst + ((4 * jj + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+            }
+        }
+        return;
+    }
+    // Q2_K / Q3_K: sub-blocks j = 4 cc + i of 16 weights, two core-matrix rows each
+    if (fmt == kQ2K) {
+        const float dmin = ldgh(rec_ptr(base + L.plane[1], L, 2, R, s));
+        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 16, R, s);
+        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 64, R, s);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int j = 4 * cc + i;
+            const uint32_t f = sp[q16_slot(j)];
+            const __half2 a2 = __float2half2_rn(d * (float)(f & 15u)), nb2 = __float2half2_rn(-(dmin * (float)(f >> 4)));
+            const uint32_t w = ldg32(cp + 4 * (4 * i + cc));
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                uint32_t o[4];
+#pragma unroll
+                for (int mm = 0; mm < 4; ++mm) {
+                    const int m = 4 * q + mm;
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(w, 2 * m, 0x00030003u), k1024), nb2));
+                }
+                sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+            }
+        }
+        return;
+    }
+    // Q3_K
+    const uint8_t* sp = rec_ptr(base + L.plane[1], L, 12, R, s);
+    const uint8_t* lp = rec_ptr(base + L.plane[2], L, 64, R, s);
+    const uint8_t* hp = rec_ptr(base + L.plane[3], L, 32, R, s);
+    const __half2 k1028 = __float2half2_rn(1028.0f);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int j = 4 * cc + i;
+        const __half2 a2 = __float2half2_rn(d * (float)(q3_scale_field(sp, j) - 32));
+        const uint32_t wl = ldg32(lp + 4 * (4 * i + cc));
+        const uint32_t wh = ldg32(hp + 4 * (2 * i + (cc >> 1))) >> (8 * (cc & 1));
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            uint32_t o[4];
+#pragma unroll
+            for (int mm = 0; mm < 4; ++mm) {
+                const int m = 4 * q + mm;
+                const uint32_t t = ((wl >> (2 * m)) & 0x00030003u) | (((wh >> m) & 0x00010001u) << 2) | 0x64006400u;
+                o[mm] = h2u(__hmul2(a2, __hsub2(u2h(t), k1028)));
+            }
+            sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+        }
+    }
+}
+
+__device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
+
+template <bool kDown>
+__global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_constant__ ExpertTab tab,
+                                                               const __grid_constant__ PrefillArgs A) {
+    pdl_wait();
+    pdl_launch();
+    extern __shared__ __align__(1024) uint8_t smem[];
+    __shared__ PSlots sl;
+    __shared__ int32_t s_row[kNT], s_asg[kNT];
+    __shared__ float s_w[kNT];
+    __shared__ __align__(8) uint64_t bars[kPSlots];
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    const Dims& d = A.d;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n_mt = (kDown ? d.H : d.I) / kMT;
+    const int K = kDown ? d.I : d.H;
+    const int n_slots = A.active[0] + d.has_shared;
+    // slot table: shared expert first, then the active routed experts
+    for (int i = tid; i < n_slots; i += kPThreads) {
+        int e;
+        if (i < d.has_shared) { e = d.E; sl.first[i] = 0; sl.ntot[i] = d.T; }
+        else {
+            e = A.active[1 + i - d.has_shared];
+            sl.first[i] = A.offsets[e]; sl.ntot[i] = A.offsets[e + 1] - A.offsets[e];
+        }
+        sl.ptr[i][0] = tab.p[e][kDown ? 2 : 0];
+        sl.ptr[i][1] = tab.p[e][1];
+        sl.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
+        sl.fmt[i][1] = tab.fmt[e][1];
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int run = 0;
+        for (int i = 0; i < n_slots; ++i) { sl.pre[i] = run; run += n_mt * ((sl.ntot[i] + kNT - 1) / kNT); }
+        sl.pre[n_slots] = run;
+        s_fail = 0;
+        for (int i = 0; i < kPSlots; ++i)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"((uint32_t)__cvta_generic_to_shared(&bars[i]))
+                         : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    constexpr int kCols = kDown ? 256 : 512;
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     ::"r"((uint32_t)__cvta_generic_to_shared(&s_tmem)), "r"(kCols) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tbase = s_tmem;
+    const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
+    const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
+    const int n_units = sl.pre[n_slots];
+    const int nC = K / kKC;
+    int gchunk = 0;        // chunks issued by this CTA so far (ring position and parities)
+    int last_committed = -1;
+    bool failed = false;
+    int cursor = 0;
+
+    for (int u = blockIdx.x; u < n_units && !failed; u += gridDim.x) {
+        while (cursor + 1 < n_slots && sl.pre[cursor + 1] <= u) ++cursor;
+        const int p = cursor, local = u - sl.pre[p];
+        const int tt = local / n_mt, mt = local - tt * n_mt;
+        const int n0 = tt * kNT, N = min(kNT, sl.ntot[p] - n0), Npad = (N + 15) & ~15;
+        const bool shared = p < d.has_shared;
+        // the unit's activation rows, assignments and weights
+        for (int n = tid; n < kNT; n += kPThreads) {
+            int a = -1, row = 0;
+            float w = 0.0f;
+            if (n < N) {
+                const int q = n0 + n;
+                if (shared) { a = d.T * d.K + q; row = q; w = 1.0f; }
+                else { a = A.perm[sl.first[p] + q]; row = a / d.K; w = A.wts[a]; }
+                if (kDown) row = a;
+            }
+            s_row[n] = row; s_asg[n] = a; s_w[n] = w;
+        }
+        const int f0 = sl.fmt[p][0], f1 = sl.fmt[p][1];
+        const TensorLayout L0 = tensor_layout(f0, kDown ? d.H : d.I, K);
+        const TensorLayout L1 = tensor_layout(f1, d.I, K);
+        const uint8_t* b0 = sl.ptr[p][0];
+        const uint8_t* b1 = sl.ptr[p][1];
+        const int64_t R = (int64_t)mt * kMT + tid;   // this thread's weight row
+        const __half* src = kDown ? A.h16 : A.x16;
+        const int src_ld = K;
+        __syncthreads();
+
+        // B gather of chunk c into ring slot s (cp.async, zero rows past N)
+        auto gather = [&](int c, int s) {
+            const uint32_t bdst = ring + s * kSlotBytes + 2 * kABytes;
+            for (int i = tid; i < Npad * 8; i += kPThreads) {
+                const int n = i >> 3, kc = i & 7;
+                const uint32_t dst = bdst + (kc * kNT + n) * 16;
+                if (n < N) {
+                    const __half* g = src + (size_t)s_row[n] * src_ld + c * kKC + kc * 8;
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(g) : "memory");
+                } else {
+                    sts128(dst, 0u, 0u, 0u, 0u);
+                }
+            }
+        };
+        gather(0, gchunk % kPSlots);
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        for (int c = 0; c < nC; ++c) {
+            const int g = gchunk + c, s = g % kPSlots;
+            bool bad = false;
+            if (c + 1 < nC) {
+                const int g1 = g + 1, s1 = g1 % kPSlots;
+                // slot s1 was last used by chunk g1 - kPSlots: its MMAs must be done
+                if (g1 >= kPSlots) bad = !mbar_wait(bar0 + 8 * s1, ((g1 - kPSlots) / kPSlots) & 1);
+                if (!bad) gather(c + 1, s1);
+            }
+            asm volatile("cp.async.commit_group;" ::: "memory");
+            const uint32_t sbase = ring + s * kSlotBytes;
+            dequant_chunk(f0, b0, L0, R, c, sbase + tid * 16);
+            if (!kDown) dequant_chunk(f1, b1, L1, R, c, sbase + kABytes + tid * 16);
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            if (__syncthreads_or(bad)) { failed = true; break; }
+            if (tid == 0) {
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t idesc = idesc_f16(kMT, Npad);
+                const uint32_t bsm = sbase + 2 * kABytes;
+#pragma unroll
+                for (int ks = 0; ks < kKC / 16; ++ks) {
+                    const uint32_t acc = (c > 0 || ks > 0) ? 1u : 0u;
+                    const uint64_t db = sdesc(bsm + 2 * ks * kNT * 16, kNT * 16, 128);
+                    mma_f16(tbase, sdesc(sbase + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
+                    if (!kDown) mma_f16(tbase + kNT, sdesc(sbase + kABytes + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
+                }
+                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                             ::"r"(bar0 + 8 * s) : "memory");
+            }
+            last_committed = g;
+        }
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        if (failed) break;
+        // all MMAs of the unit are done once the last chunk's commit arrived
+        const int glast = gchunk + nC - 1;
+        const bool ok = mbar_wait(bar0 + 8 * (glast % kPSlots), (glast / kPSlots) & 1);
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        gchunk += nC;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        // epilogue: TMEM lane 32 warp + lane = weight row, columns = tokens
+        const int row = mt * kMT + 32 * warp + lane;
+        for (int n = 0; n < Npad; n += 8) {
+            uint32_t g8[8], u8[8];
+            const uint32_t ta = tbase + ((uint32_t)(32 * warp) << 16) + (uint32_t)n;
+            asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                         : "=r"(g8[0]), "=r"(g8[1]), "=r"(g8[2]), "=r"(g8[3]), "=r"(g8[4]), "=r"(g8[5]), "=r"(g8[6]),
+                           "=r"(g8[7]) : "r"(ta));
+            if (!kDown)
+                asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                             : "=r"(u8[0]), "=r"(u8[1]), "=r"(u8[2]), "=r"(u8[3]), "=r"(u8[4]), "=r"(u8[5]),
+                               "=r"(u8[6]), "=r"(u8[7]) : "r"(ta + kNT));
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int nn = n + j;
+                if (nn >= N) break;
+                const int a = s_asg[nn];
+                if (kDown) {
+                    A.pdn[(size_t)a * d.H + row] = __uint_as_float(g8[j]);
+                } else {
+                    const float gv = __uint_as_float(g8[j]), uv = __uint_as_float(u8[j]);
+                    A.h16[(size_t)a * d.I + row] = __float2half_rn(silu(gv) * uv * s_w[nn]);
+                }
+            }
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    }
+    if (failed && tid == 0) { atomicOr(A.err, kErrMma); s_fail = 1; }
+    __syncthreads();
+    if (s_fail && last_committed >= 0) {
+        // wait (bounded) for the MMAs still in flight before giving TMEM back
+        mbar_wait(bar0 + 8 * (last_committed % kPSlots), (last_committed / kPSlots) & 1);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(kCols) : "memory");
+    }
+}
+
+int g_psms = 0;
+
+}  // namespace
+
+cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
+    if (d.T == 0) return cudaSuccess;
+    const int smem = kPSlots * kSlotBytes;
+    if (g_psms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_psms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_psms <= 0) g_psms = 148;
+        cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    }
+    PrefillArgs A;
+    A.d = d;
+    A.offsets = w.offsets; A.perm = w.perm; A.active = w.active; A.wts = w.wts;
+    A.x16 = w.x16; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
+    prof_begin("gateup_tc", s);
+    cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(kPThreads), smem, s, tab, A);
+    prof_end(s);
+    if (err != cudaSuccess) return err;
+    prof_begin("down_tc", s);
+    err = launch_pdl(prefill_kernel<true>, dim3(g_psms), dim3(kPThreads), smem, s, tab, A);
+    prof_end(s);
+    if (err != cudaSuccess) return err;
+    return launch_combine(d, w.pdn, out, s);
+}
+
+}  // namespace mq

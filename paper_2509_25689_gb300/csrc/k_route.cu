@@ -37,6 +37,7 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
                                                              const float* __restrict__ W, int H, int T,
                                                              int E, float* __restrict__ z,
                                                              __half* __restrict__ xq, float* __restrict__ xs,
+                                                             __half* __restrict__ x16,
                                                              uint32_t* __restrict__ zero_words, int n_zero) {
     pdl_wait();
     pdl_launch();
@@ -88,6 +89,15 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
             float r = part[0][threadIdx.x];
             for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
             z[(size_t)t * E + e] = r;
+        }
+    }
+    // fp16 copy of the tokens for the prefill GEMM, spread over the CTAs
+    if (x16 != nullptr) {
+        for (int j = 0; j < kTok; ++j) {
+            const int t = t0 + j;
+            if (t >= T) break;
+            for (int k = e * blockDim.x + threadIdx.x; k < H; k += E * blockDim.x)
+                x16[(size_t)t * H + k] = __float2half_rn(bf16_lo(x[(size_t)t * H + k]));
         }
     }
     // The CTAs also prepare the tokens' activations for the expert-FFN
@@ -403,13 +413,13 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 }  // namespace
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 uint32_t* zero_words, int n_zero, cudaStream_t s) {
+                                 __half* x16, uint32_t* zero_words, int n_zero, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
     dim3 grid(d.E, (d.T + kTok - 1) / kTok);
     prof_begin("router_logits", s);
     const cudaError_t e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq,
-                                     xs, zero_words, n_zero);
+                                     xs, x16, zero_words, n_zero);
     prof_end(s);
     return e;
 }

@@ -103,6 +103,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
         w->counter_bytes = cnt_bytes;
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
+        w->x16 = w->xq;   // the prefill path uses these bytes instead of the decode preparation
+        w->h16 = w->hq;
         w->zero_words = w->counters;
         w->n_zero = (int)((cnt_bytes + 4) / 4);
     }
@@ -173,21 +175,26 @@ int check_common(const mq_layer_cfg* cfg, int32_t T, const void* x, const float*
     return MQ_OK;
 }
 
+// Routing, permutation and the per-call set-up of the expert-FFN path:
+// mode 0 = routing only, 1 = decode (prepared tokens + work plan),
+// 2 = prefill (fp16 tokens for the grouped GEMM).
 int run_route(const Dims& d, const void* x, const float* router_w, const float* bias, Work& w,
-              cudaStream_t s, bool prep_tokens) {
-    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, prep_tokens ? w.xq : nullptr, w.xs,
-                             prep_tokens ? w.zero_words : nullptr, prep_tokens ? w.n_zero : 0, s) != cudaSuccess)
+              cudaStream_t s, int mode) {
+    const bool fwd = mode != 0;
+    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, mode == 1 ? w.xq : nullptr, w.xs,
+                             mode == 2 ? w.x16 : nullptr, fwd ? w.zero_words : nullptr, fwd ? w.n_zero : 0,
+                             s) != cudaSuccess)
         return MQ_ECUDA;
+    Plan* plan = mode == 1 ? w.plan : nullptr;
     if (d.T <= kFusedRouteTokens) {
         // decode-sized batch: top-k, permutation and work plan in one CTA
-        if (launch_route_permute(d, w.z, bias, w.idx, w.wts, w.offsets, w.perm, w.inv, w.active,
-                                 prep_tokens ? w.plan : nullptr, s) != cudaSuccess)
+        if (launch_route_permute(d, w.z, bias, w.idx, w.wts, w.offsets, w.perm, w.inv, w.active, plan, s) !=
+            cudaSuccess)
             return MQ_ECUDA;
         return MQ_OK;
     }
     if (launch_topk(d, w.z, bias, w.idx, w.wts, s) != cudaSuccess) return MQ_ECUDA;
-    if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, prep_tokens ? w.plan : nullptr, s) != cudaSuccess)
-        return MQ_ECUDA;
+    if (launch_permute(d, w.idx, w.offsets, w.perm, w.inv, w.active, plan, s) != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
 }
 
@@ -207,7 +214,7 @@ extern "C" int moe_quant_route(const mq_layer_cfg* cfg, int32_t n_tokens, const 
     if (offsets) w.offsets = offsets;
     if (perm) w.perm = perm;
     if (inv) w.inv = inv;
-    return run_route(d, x, router_w, bias, w, static_cast<cudaStream_t>(stream), false);
+    return run_route(d, x, router_w, bias, w, static_cast<cudaStream_t>(stream), 0);
 }
 
 extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x, const float* router_w,
@@ -239,9 +246,14 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     workspace_plan(d, workspace, &w);
     if (topk_idx) w.idx = topk_idx;
     if (topk_w) w.wts = topk_w;
-    rc = run_route(d, x, router_w, bias, w, s, true);
+    const int pm = path_mode();
+    const bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
+    rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1);
     if (rc != MQ_OK) return rc;
-    (void)path_mode();
+    if (prefill) {
+        if (launch_prefill(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
+        return MQ_OK;
+    }
     if (launch_decode_mma(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
 }

@@ -57,6 +57,8 @@ struct Work {
     uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
     size_t counter_bytes;
     uint32_t* err;     // device error word (bounded waits that ran out)
+    __half* x16;       // [T][H] tokens in fp16 for the prefill GEMM (shares xq's bytes)
+    __half* h16;       // [A][I] fp16 SwiGLU outputs for the prefill GEMM (shares hq's bytes)
     uint32_t* zero_words; // counters + error word, cleared by the first kernel of a call
     int n_zero;
 };
@@ -90,7 +92,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 #endif
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 uint32_t* zero_words, int n_zero,
+                                 __half* x16, uint32_t* zero_words, int n_zero,
                                  cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
@@ -98,6 +100,8 @@ cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, 
 cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                                  int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
                                  cudaStream_t s);
+cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s);
+cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 size_t decode_counter_bytes(const Dims& d);
 cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);
