@@ -63,7 +63,27 @@ def draw_formats(spec: LayerSpec, seed: int) -> np.ndarray:
     return f
 
 
-def draw_router(spec: LayerSpec, seed: int):
+def zipf_ranks(spec: LayerSpec, seed: int) -> np.ndarray:
+    """Seeded popularity rank of every expert (0 = most popular)."""
+    return rng_for(seed + 5).permutation(spec.n_experts).astype(np.int64)
+
+
+def zipf_bias_shape(spec: LayerSpec, seed: int) -> np.ndarray:
+    """-s * ln(rank + 1): the bias direction that skews expert counts towards
+    a Zipf(s) law; its scale gamma is fitted once (tests/golden/zipf_gamma.json)."""
+    return (-float(spec.zipf_s) * np.log(zipf_ranks(spec, seed) + 1.0)).astype(np.float32)
+
+
+def zipf_gamma() -> float:
+    import json
+    import os
+    path = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "tests", "golden",
+                        "zipf_gamma.json")
+    with open(path) as f:
+        return float(json.load(f)["gamma"])
+
+
+def draw_router(spec: LayerSpec, seed: int, gamma: float | None = None):
     r = rng_for(seed + 1)
     w = (r.standard_normal((spec.n_experts, spec.hidden), dtype=np.float32)
          * np.float32(spec.router_std)).astype(np.float32)
@@ -71,6 +91,9 @@ def draw_router(spec: LayerSpec, seed: int):
         b = (r.standard_normal(spec.n_experts, dtype=np.float32) * np.float32(spec.bias_std)).astype(np.float32)
     else:
         b = np.zeros(spec.n_experts, np.float32)
+    if spec.zipf_s is not None:
+        g = zipf_gamma() if gamma is None else gamma
+        b = (b + np.float32(g) * zipf_bias_shape(spec, seed)).astype(np.float32)
     return w, b
 
 
