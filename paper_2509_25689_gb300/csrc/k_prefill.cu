@@ -103,81 +103,138 @@ __device__ __forceinline__ __half2 code_pair(uint32_t w, int s, uint32_t mask) {
     return u2h(((w >> s) & mask) | 0x64006400u);
 }
 
-// Row r of the unit, 64-wide chunk c of the contraction: decode the 64
-// weights of one tensor to fp16 and store them as 8 core-matrix rows.
-// Decoded values follow the format definitions of include/moeq.h; the
-// per-sub-block products d*sc and dmin*m are rounded to fp16 once.
-__device__ __forceinline__ void dequant_chunk(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R, int c,
-                                              uint32_t dst) {
-    const __half2 k1024 = __float2half2_rn(1024.0f);
+// Raw packed fields of one weight row for one 64-wide chunk of the
+// contraction, loaded one chunk ahead of their use.
+struct Packed {
+    uint32_t w[16];   // code words (Q8_0: two blocks x 8; Q4_K: two sub-blocks x 4; Q2_K/Q3_K: 4 low + 4 high)
+    uint32_t sc[4];   // scale record (Q2_K 16 B, Q3_K / Q4_K 12 B)
+    uint32_t dd;      // d | dmin << 16 (Q8_0: d of the two blocks)
+};
+
+__device__ __forceinline__ uint32_t ldg16u(const uint8_t* p) { return __ldg(reinterpret_cast<const unsigned short*>(p)); }
+
+__device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R, int c,
+                                           Packed& P) {
     if (fmt == kQ80) {
 #pragma unroll
         for (int bb = 0; bb < 2; ++bb) {
             const int64_t b = 2 * c + bb;
-            const float dv = ldgh(rec_ptr(base + L.plane[0], L, 2, R, b));
-            const __half2 d2 = __float2half2_rn(dv);
             const uint8_t* cp = rec_ptr(base + L.plane[1], L, 32, R, b);
             const uint4 w0 = ldg128(cp), w1 = ldg128(cp + 16);
-            const __half2 k1152 = __float2half2_rn(1152.0f);
+            P.w[8 * bb + 0] = w0.x; P.w[8 * bb + 1] = w0.y; P.w[8 * bb + 2] = w0.z; P.w[8 * bb + 3] = w0.w;
+            P.w[8 * bb + 4] = w1.x; P.w[8 * bb + 5] = w1.y; P.w[8 * bb + 6] = w1.z; P.w[8 * bb + 7] = w1.w;
+        }
+        P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c)) |
+               (ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c + 1)) << 16);
+        return;
+    }
+    const int64_t s = c >> 2;
+    const int cc = c & 3;
+    P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, s));
+    if (fmt == kQ4K) {
+        P.dd |= ldg16u(rec_ptr(base + L.plane[1], L, 2, R, s)) << 16;
+        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 12, R, s);
+        P.sc[0] = ldg32(sp); P.sc[1] = ldg32(sp + 4); P.sc[2] = ldg32(sp + 8);
+        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 128, R, s);
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+            const int j = 2 * cc + jj;
+            const uint4 w = ldg128(cp + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
+            P.w[4 * jj + 0] = w.x; P.w[4 * jj + 1] = w.y; P.w[4 * jj + 2] = w.z; P.w[4 * jj + 3] = w.w;
+        }
+        return;
+    }
+    if (fmt == kQ2K) {
+        P.dd |= ldg16u(rec_ptr(base + L.plane[1], L, 2, R, s)) << 16;
+        const uint4 sv = ldg128(rec_ptr(base + L.plane[2], L, 16, R, s));
+        P.sc[0] = sv.x; P.sc[1] = sv.y; P.sc[2] = sv.z; P.sc[3] = sv.w;
+        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 64, R, s);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) P.w[i] = ldg32(cp + 4 * (4 * i + cc));
+        return;
+    }
+    // Q3_K
+    const uint8_t* sp = rec_ptr(base + L.plane[1], L, 12, R, s);
+    P.sc[0] = ldg32(sp); P.sc[1] = ldg32(sp + 4); P.sc[2] = ldg32(sp + 8);
+    const uint8_t* lp = rec_ptr(base + L.plane[2], L, 64, R, s);
+    const uint8_t* hp = rec_ptr(base + L.plane[3], L, 32, R, s);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        P.w[i] = ldg32(lp + 4 * (4 * i + cc));
+        P.w[4 + i] = ldg32(hp + 4 * (2 * i + (cc >> 1)));
+    }
+}
+
+__device__ __forceinline__ float half_lo(uint32_t v) { return __half2float(__ushort_as_half((unsigned short)(v & 0xffffu))); }
+__device__ __forceinline__ float half_hi(uint32_t v) { return __half2float(__ushort_as_half((unsigned short)(v >> 16))); }
+// byte i (0..15) of a 4-word record, with a runtime i kept in registers
+__device__ __forceinline__ uint32_t byte_of(const uint32_t (&w)[4], int i) {
+    const int k = i >> 2;
+    const uint32_t v = k == 0 ? w[0] : k == 1 ? w[1] : k == 2 ? w[2] : w[3];
+    return (v >> (8 * (i & 3))) & 0xffu;
+}
+
+// Decode the 64 weights of chunk c of one row (fields in P) to fp16 and store
+// them as 8 core-matrix rows at dst, dst + 128*16, ...  Values follow the
+// format definitions of include/moeq.h; the per-sub-block products d*sc and
+// dmin*m are rounded to fp16 once.
+__device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, uint32_t dst) {
+    const __half2 k1024 = __float2half2_rn(1024.0f);
+    if (fmt == kQ80) {
+        const __half2 k1152 = __float2half2_rn(1152.0f);
+#pragma unroll
+        for (int bb = 0; bb < 2; ++bb) {
+            const __half2 d2 = __float2half2_rn(bb ? half_hi(P.dd) : half_lo(P.dd));
 #pragma unroll
             for (int q = 0; q < 4; ++q) {   // core-matrix row kc = 4 bb + q: pairs m = 4q .. 4q+3
                 uint32_t o[4];
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    const uint32_t w = sub4(m < 8 ? w0 : w1, (m >> 1) & 3);
-                    o[mm] = h2u(__hmul2(d2, __hsub2(code_pair(w, 8 * (m & 1), 0x00FF00FFu), k1152)));
+                    o[mm] = h2u(__hmul2(d2, __hsub2(code_pair(P.w[8 * bb + (m >> 1)], 8 * (m & 1), 0x00FF00FFu), k1152)));
                 }
                 sts128(dst + ((4 * bb + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
         }
         return;
     }
-    const int64_t s = c >> 2;
     const int cc = c & 3;
-    const float d = ldgh(rec_ptr(base + L.plane[0], L, 2, R, s));
+    const float d = half_lo(P.dd);
     if (fmt == kQ4K) {
-        const float dmin = ldgh(rec_ptr(base + L.plane[1], L, 2, R, s));
-        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 12, R, s);
+        const float dmin = half_hi(P.dd);
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
             const int j = 2 * cc + jj;
-            int sc, mn;
-            q4_fields(sp, j, sc, mn);
+            const uint32_t lo = byte_of(P.sc, j), high = P.sc[2] >> (4 * j);
+            const int sc = (int)(lo & 15u) | (int)((high & 3u) << 4), mn = (int)(lo >> 4) | (int)(((high >> 2) & 3u) << 4);
             const __half2 a2 = __float2half2_rn(d * (float)sc), nb2 = __float2half2_rn(-(dmin * (float)mn));
-            const uint4 w = ldg128(rec_ptr(base + L.plane[3], L, 128, R, s) + (j >> 2) * (kRowTile * 64) +
-                                   16 * (j & 3));
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 uint32_t o[4];
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(sub4(w, m >> 2), 4 * (m & 3), 0x000F000Fu), k1024), nb2));
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[4 * jj + (m >> 2)], 4 * (m & 3), 0x000F000Fu), k1024), nb2));
                 }
                 sts128(dst + ((4 * jj + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
         }
         return;
     }
-    // Q2_K / Q3_K: sub-blocks j = 4 cc + i of 16 weights, two core-matrix rows each
     if (fmt == kQ2K) {
-        const float dmin = ldgh(rec_ptr(base + L.plane[1], L, 2, R, s));
-        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 16, R, s);
-        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 64, R, s);
+        const float dmin = half_hi(P.dd);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int j = 4 * cc + i;
-            const uint32_t f = sp[q16_slot(j)];
+            const uint32_t f = byte_of(P.sc, q16_slot(j));
             const __half2 a2 = __float2half2_rn(d * (float)(f & 15u)), nb2 = __float2half2_rn(-(dmin * (float)(f >> 4)));
-            const uint32_t w = ldg32(cp + 4 * (4 * i + cc));
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
                 uint32_t o[4];
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(w, 2 * m, 0x00030003u), k1024), nb2));
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[i], 2 * m, 0x00030003u), k1024), nb2));
                 }
                 sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
@@ -185,16 +242,15 @@ __device__ __forceinline__ void dequant_chunk(int fmt, const uint8_t* base, cons
         return;
     }
     // Q3_K
-    const uint8_t* sp = rec_ptr(base + L.plane[1], L, 12, R, s);
-    const uint8_t* lp = rec_ptr(base + L.plane[2], L, 64, R, s);
-    const uint8_t* hp = rec_ptr(base + L.plane[3], L, 32, R, s);
     const __half2 k1028 = __float2half2_rn(1028.0f);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int j = 4 * cc + i;
-        const __half2 a2 = __float2half2_rn(d * (float)(q3_scale_field(sp, j) - 32));
-        const uint32_t wl = ldg32(lp + 4 * (4 * i + cc));
-        const uint32_t wh = ldg32(hp + 4 * (2 * i + (cc >> 1))) >> (8 * (cc & 1));
+        const int u = q16_slot(j);
+        const int sfield = (int)((byte_of(P.sc, u >> 1) >> (4 * (u & 1))) & 15u) |
+                           (int)(((byte_of(P.sc, 8 + (u >> 2)) >> (2 * (u & 3))) & 3u) << 4);
+        const __half2 a2 = __float2half2_rn(d * (float)(sfield - 32));
+        const uint32_t wl = P.w[i], wh = P.w[4 + i] >> (8 * (cc & 1));
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
             uint32_t o[4];
@@ -315,7 +371,15 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         };
         gather(0, gchunk % kPSlots);
         asm volatile("cp.async.commit_group;" ::: "memory");
+        Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
+        load_chunk(f0, b0, L0, R, 0, P0);
+        if (!kDown) load_chunk(f1, b1, L1, R, 0, P1);
         for (int c = 0; c < nC; ++c) {
+            Packed N0, N1;             // the next chunk's, loaded while this one is decoded
+            if (c + 1 < nC) {
+                load_chunk(f0, b0, L0, R, c + 1, N0);
+                if (!kDown) load_chunk(f1, b1, L1, R, c + 1, N1);
+            }
             const int g = gchunk + c, s = g % kPSlots;
             bool bad = false;
             if (c + 1 < nC) {
@@ -326,8 +390,10 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
             const uint32_t sbase = ring + s * kSlotBytes;
-            dequant_chunk(f0, b0, L0, R, c, sbase + tid * 16);
-            if (!kDown) dequant_chunk(f1, b1, L1, R, c, sbase + kABytes + tid * 16);
+            dequant_store(f0, P0, c, sbase + tid * 16);
+            if (!kDown) dequant_store(f1, P1, c, sbase + kABytes + tid * 16);
+            P0 = N0;
+            if (!kDown) P1 = N1;
             asm volatile("cp.async.wait_group 1;" ::: "memory");
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             if (__syncthreads_or(bad)) { failed = true; break; }

@@ -78,3 +78,18 @@ def test_prefill_v3_layer_sampled(torch_cuda, orc, prefill_path):
         ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
         np.testing.assert_array_equal(idx[t:t + 1], ridx)
         assert_close(y[t:t + 1], ry)
+
+
+def test_prefill_v3_zipf_t2048_sampled(torch_cuda, orc):
+    """The Zipf-skewed V3 prefill workload (T = 2048, mixed formats) through
+    the automatic path choice; a few tokens against the oracle."""
+    spec = get_config("v3_prefill_t2048_zipf")
+    layer = DeviceLayer(spec, 0)
+    x = tokens(spec, 0)
+    y, idx, w = layer.forward(x)
+    counts = np.bincount(idx.reshape(-1), minlength=spec.n_experts)
+    assert counts.max() >= 4 * counts[counts > 0].mean()   # skewed towards a few experts
+    for t in (0, 1337, 2047):
+        ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
+        np.testing.assert_array_equal(idx[t:t + 1], ridx)
+        assert_close(y[t:t + 1], ry)
