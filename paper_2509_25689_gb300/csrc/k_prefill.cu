@@ -28,7 +28,7 @@
 namespace mq {
 namespace {
 
-constexpr int kPThreads = 128;                 // 4 warps = the 4 TMEM lane quarters
+constexpr int kPThreads = 256;                 // 8 warps: two per TMEM lane quarter
 constexpr int kMT = 128;                       // weight rows per unit (MMA M)
 constexpr int kNT = 256;                       // tokens per unit (largest MMA N)
 constexpr int kKC = 64;                        // K per ring slot
@@ -114,18 +114,17 @@ struct Packed {
 __device__ __forceinline__ uint32_t ldg16u(const uint8_t* p) { return __ldg(reinterpret_cast<const unsigned short*>(p)); }
 
 __device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R, int c,
-                                           Packed& P) {
+                                           int hf, Packed& P) {
     if (fmt == kQ80) {
-#pragma unroll
-        for (int bb = 0; bb < 2; ++bb) {
+        {
+            const int bb = hf;
             const int64_t b = 2 * c + bb;
             const uint8_t* cp = rec_ptr(base + L.plane[1], L, 32, R, b);
             const uint4 w0 = ldg128(cp), w1 = ldg128(cp + 16);
-            P.w[8 * bb + 0] = w0.x; P.w[8 * bb + 1] = w0.y; P.w[8 * bb + 2] = w0.z; P.w[8 * bb + 3] = w0.w;
-            P.w[8 * bb + 4] = w1.x; P.w[8 * bb + 5] = w1.y; P.w[8 * bb + 6] = w1.z; P.w[8 * bb + 7] = w1.w;
+            P.w[0] = w0.x; P.w[1] = w0.y; P.w[2] = w0.z; P.w[3] = w0.w;
+            P.w[4] = w1.x; P.w[5] = w1.y; P.w[6] = w1.z; P.w[7] = w1.w;
         }
-        P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c)) |
-               (ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c + 1)) << 16);
+        P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c + hf));
         return;
     }
     const int64_t s = c >> 2;
@@ -136,11 +135,10 @@ __device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const T
         const uint8_t* sp = rec_ptr(base + L.plane[2], L, 12, R, s);
         P.sc[0] = ldg32(sp); P.sc[1] = ldg32(sp + 4); P.sc[2] = ldg32(sp + 8);
         const uint8_t* cp = rec_ptr(base + L.plane[3], L, 128, R, s);
-#pragma unroll
-        for (int jj = 0; jj < 2; ++jj) {
-            const int j = 2 * cc + jj;
+        {
+            const int jj = hf, j = 2 * cc + jj;
             const uint4 w = ldg128(cp + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
-            P.w[4 * jj + 0] = w.x; P.w[4 * jj + 1] = w.y; P.w[4 * jj + 2] = w.z; P.w[4 * jj + 3] = w.w;
+            P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
         }
         return;
     }
@@ -150,7 +148,7 @@ __device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const T
         P.sc[0] = sv.x; P.sc[1] = sv.y; P.sc[2] = sv.z; P.sc[3] = sv.w;
         const uint8_t* cp = rec_ptr(base + L.plane[3], L, 64, R, s);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) P.w[i] = ldg32(cp + 4 * (4 * i + cc));
+        for (int ii = 0; ii < 2; ++ii) { const int i = 2 * hf + ii; P.w[ii] = ldg32(cp + 4 * (4 * i + cc)); }
         return;
     }
     // Q3_K
@@ -159,9 +157,10 @@ __device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const T
     const uint8_t* lp = rec_ptr(base + L.plane[2], L, 64, R, s);
     const uint8_t* hp = rec_ptr(base + L.plane[3], L, 32, R, s);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        P.w[i] = ldg32(lp + 4 * (4 * i + cc));
-        P.w[4 + i] = ldg32(hp + 4 * (2 * i + (cc >> 1)));
+    for (int ii = 0; ii < 2; ++ii) {
+        const int i = 2 * hf + ii;
+        P.w[ii] = ldg32(lp + 4 * (4 * i + cc));
+        P.w[4 + ii] = ldg32(hp + 4 * (2 * i + (cc >> 1)));
     }
 }
 
@@ -178,20 +177,20 @@ __device__ __forceinline__ uint32_t byte_of(const uint32_t (&w)[4], int i) {
 // them as 8 core-matrix rows at dst, dst + 128*16, ...  Values follow the
 // format definitions of include/moeq.h; the per-sub-block products d*sc and
 // dmin*m are rounded to fp16 once.
-__device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, uint32_t dst) {
+__device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
     const __half2 k1024 = __float2half2_rn(1024.0f);
     if (fmt == kQ80) {
         const __half2 k1152 = __float2half2_rn(1152.0f);
-#pragma unroll
-        for (int bb = 0; bb < 2; ++bb) {
-            const __half2 d2 = __float2half2_rn(bb ? half_hi(P.dd) : half_lo(P.dd));
+        {
+            const int bb = hf;
+            const __half2 d2 = __float2half2_rn(half_lo(P.dd));
 #pragma unroll
             for (int q = 0; q < 4; ++q) {   // core-matrix row kc = 4 bb + q: pairs m = 4q .. 4q+3
                 uint32_t o[4];
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    o[mm] = h2u(__hmul2(d2, __hsub2(code_pair(P.w[8 * bb + (m >> 1)], 8 * (m & 1), 0x00FF00FFu), k1152)));
+                    o[mm] = h2u(__hmul2(d2, __hsub2(code_pair(P.w[m >> 1], 8 * (m & 1), 0x00FF00FFu), k1152)));
                 }
                 sts128(dst + ((4 * bb + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
@@ -202,9 +201,8 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, u
     const float d = half_lo(P.dd);
     if (fmt == kQ4K) {
         const float dmin = half_hi(P.dd);
-#pragma unroll
-        for (int jj = 0; jj < 2; ++jj) {
-            const int j = 2 * cc + jj;
+        {
+            const int jj = hf, j = 2 * cc + jj;
             const uint32_t lo = byte_of(P.sc, j), high = P.sc[2] >> (4 * j);
             const int sc = (int)(lo & 15u) | (int)((high & 3u) << 4), mn = (int)(lo >> 4) | (int)(((high >> 2) & 3u) << 4);
             const __half2 a2 = __float2half2_rn(d * (float)sc), nb2 = __float2half2_rn(-(dmin * (float)mn));
@@ -214,7 +212,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, u
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[4 * jj + (m >> 2)], 4 * (m & 3), 0x000F000Fu), k1024), nb2));
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[m >> 2], 4 * (m & 3), 0x000F000Fu), k1024), nb2));
                 }
                 sts128(dst + ((4 * jj + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
@@ -224,8 +222,8 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, u
     if (fmt == kQ2K) {
         const float dmin = half_hi(P.dd);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int j = 4 * cc + i;
+        for (int ii = 0; ii < 2; ++ii) {
+            const int i = 2 * hf + ii, j = 4 * cc + i;
             const uint32_t f = byte_of(P.sc, q16_slot(j));
             const __half2 a2 = __float2half2_rn(d * (float)(f & 15u)), nb2 = __float2half2_rn(-(dmin * (float)(f >> 4)));
 #pragma unroll
@@ -234,7 +232,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, u
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[i], 2 * m, 0x00030003u), k1024), nb2));
+                    o[mm] = h2u(__hfma2(a2, __hsub2(code_pair(P.w[ii], 2 * m, 0x00030003u), k1024), nb2));
                 }
                 sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
@@ -244,13 +242,13 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, u
     // Q3_K
     const __half2 k1028 = __float2half2_rn(1028.0f);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int j = 4 * cc + i;
+    for (int ii = 0; ii < 2; ++ii) {
+        const int i = 2 * hf + ii, j = 4 * cc + i;
         const int u = q16_slot(j);
         const int sfield = (int)((byte_of(P.sc, u >> 1) >> (4 * (u & 1))) & 15u) |
                            (int)(((byte_of(P.sc, 8 + (u >> 2)) >> (2 * (u & 3))) & 3u) << 4);
         const __half2 a2 = __float2half2_rn(d * (float)(sfield - 32));
-        const uint32_t wl = P.w[i], wh = P.w[4 + i] >> (8 * (cc & 1));
+        const uint32_t wl = P.w[ii], wh = P.w[4 + ii] >> (8 * (cc & 1));
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
             uint32_t o[4];
@@ -350,7 +348,8 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         const TensorLayout L1 = tensor_layout(f1, d.I, K);
         const uint8_t* b0 = sl.ptr[p][0];
         const uint8_t* b1 = sl.ptr[p][1];
-        const int64_t R = (int64_t)mt * kMT + tid;   // this thread's weight row
+        const int rr = tid & (kMT - 1), hf = tid >> 7;   // weight row of the unit, half of each chunk
+        const int64_t R = (int64_t)mt * kMT + rr;
         const __half* src = kDown ? A.h16 : A.x16;
         const int src_ld = K;
         __syncthreads();
@@ -372,13 +371,13 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         gather(0, gchunk % kPSlots);
         asm volatile("cp.async.commit_group;" ::: "memory");
         Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
-        load_chunk(f0, b0, L0, R, 0, P0);
-        if (!kDown) load_chunk(f1, b1, L1, R, 0, P1);
+        load_chunk(f0, b0, L0, R, 0, hf, P0);
+        if (!kDown) load_chunk(f1, b1, L1, R, 0, hf, P1);
         for (int c = 0; c < nC; ++c) {
             Packed N0, N1;             // the next chunk's, loaded while this one is decoded
             if (c + 1 < nC) {
-                load_chunk(f0, b0, L0, R, c + 1, N0);
-                if (!kDown) load_chunk(f1, b1, L1, R, c + 1, N1);
+                load_chunk(f0, b0, L0, R, c + 1, hf, N0);
+                if (!kDown) load_chunk(f1, b1, L1, R, c + 1, hf, N1);
             }
             const int g = gchunk + c, s = g % kPSlots;
             bool bad = false;
@@ -390,8 +389,8 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
             const uint32_t sbase = ring + s * kSlotBytes;
-            dequant_store(f0, P0, c, sbase + tid * 16);
-            if (!kDown) dequant_store(f1, P1, c, sbase + kABytes + tid * 16);
+            dequant_store(f0, P0, c, hf, sbase + rr * 16);
+            if (!kDown) dequant_store(f1, P1, c, hf, sbase + kABytes + rr * 16);
             P0 = N0;
             if (!kDown) P1 = N1;
             asm volatile("cp.async.wait_group 1;" ::: "memory");
@@ -422,10 +421,11 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         gchunk += nC;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         // epilogue: TMEM lane 32 warp + lane = weight row, columns = tokens
-        const int row = mt * kMT + 32 * warp + lane;
-        for (int n = 0; n < Npad; n += 8) {
+        const int quarter = warp & 3;
+        const int row = mt * kMT + 32 * quarter + lane;
+        for (int n = 8 * (warp >> 2); n < Npad; n += 16) {
             uint32_t g8[8], u8[8];
-            const uint32_t ta = tbase + ((uint32_t)(32 * warp) << 16) + (uint32_t)n;
+            const uint32_t ta = tbase + ((uint32_t)(32 * quarter) << 16) + (uint32_t)n;
             asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                          : "=r"(g8[0]), "=r"(g8[1]), "=r"(g8[2]), "=r"(g8[3]), "=r"(g8[4]), "=r"(g8[5]), "=r"(g8[6]),
                            "=r"(g8[7]) : "r"(ta));
