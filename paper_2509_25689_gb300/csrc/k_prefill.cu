@@ -113,49 +113,55 @@ struct Packed {
 
 __device__ __forceinline__ uint32_t ldg16u(const uint8_t* p) { return __ldg(reinterpret_cast<const unsigned short*>(p)); }
 
-__device__ __forceinline__ void load_chunk(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R, int c,
-                                           int hf, Packed& P) {
+// Start of one weight row's records in each plane; the record of
+// superblock (Q8_0: block) b is at row[p] + b * 32 * record_bytes[p].
+struct RowPtrs {
+    const uint8_t* row[4];
+};
+__device__ __forceinline__ RowPtrs row_ptrs(int fmt, const uint8_t* base, const TensorLayout& L, int64_t R) {
+    RowPtrs P;
+    const PlaneBytes pb = plane_bytes(fmt);
+#pragma unroll
+    for (int p = 0; p < 4; ++p) P.row[p] = p < pb.n ? rec_ptr(base + L.plane[p], L, pb.b[p], R, 0) : nullptr;
+    return P;
+}
+
+__device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, int hf, Packed& P) {
     if (fmt == kQ80) {
-        {
-            const int bb = hf;
-            const int64_t b = 2 * c + bb;
-            const uint8_t* cp = rec_ptr(base + L.plane[1], L, 32, R, b);
-            const uint4 w0 = ldg128(cp), w1 = ldg128(cp + 16);
-            P.w[0] = w0.x; P.w[1] = w0.y; P.w[2] = w0.z; P.w[3] = w0.w;
-            P.w[4] = w1.x; P.w[5] = w1.y; P.w[6] = w1.z; P.w[7] = w1.w;
-        }
-        P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, 2 * c + hf));
+        const int64_t b = 2 * c + hf;
+        const uint8_t* cp = RP.row[1] + b * (32 * 32);
+        const uint4 w0 = ldg128(cp), w1 = ldg128(cp + 16);
+        P.w[0] = w0.x; P.w[1] = w0.y; P.w[2] = w0.z; P.w[3] = w0.w;
+        P.w[4] = w1.x; P.w[5] = w1.y; P.w[6] = w1.z; P.w[7] = w1.w;
+        P.dd = ldg16u(RP.row[0] + b * (32 * 2));
         return;
     }
     const int64_t s = c >> 2;
     const int cc = c & 3;
-    P.dd = ldg16u(rec_ptr(base + L.plane[0], L, 2, R, s));
+    P.dd = ldg16u(RP.row[0] + s * (32 * 2));
     if (fmt == kQ4K) {
-        P.dd |= ldg16u(rec_ptr(base + L.plane[1], L, 2, R, s)) << 16;
-        const uint8_t* sp = rec_ptr(base + L.plane[2], L, 12, R, s);
+        P.dd |= ldg16u(RP.row[1] + s * (32 * 2)) << 16;
+        const uint8_t* sp = RP.row[2] + s * (32 * 12);
         P.sc[0] = ldg32(sp); P.sc[1] = ldg32(sp + 4); P.sc[2] = ldg32(sp + 8);
-        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 128, R, s);
-        {
-            const int jj = hf, j = 2 * cc + jj;
-            const uint4 w = ldg128(cp + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
-            P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
-        }
+        const int j = 2 * cc + hf;
+        const uint4 w = ldg128(RP.row[3] + s * (32 * 128) + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
+        P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
         return;
     }
     if (fmt == kQ2K) {
-        P.dd |= ldg16u(rec_ptr(base + L.plane[1], L, 2, R, s)) << 16;
-        const uint4 sv = ldg128(rec_ptr(base + L.plane[2], L, 16, R, s));
+        P.dd |= ldg16u(RP.row[1] + s * (32 * 2)) << 16;
+        const uint4 sv = ldg128(RP.row[2] + s * (32 * 16));
         P.sc[0] = sv.x; P.sc[1] = sv.y; P.sc[2] = sv.z; P.sc[3] = sv.w;
-        const uint8_t* cp = rec_ptr(base + L.plane[3], L, 64, R, s);
+        const uint8_t* cp = RP.row[3] + s * (32 * 64);
 #pragma unroll
         for (int ii = 0; ii < 2; ++ii) { const int i = 2 * hf + ii; P.w[ii] = ldg32(cp + 4 * (4 * i + cc)); }
         return;
     }
     // Q3_K
-    const uint8_t* sp = rec_ptr(base + L.plane[1], L, 12, R, s);
+    const uint8_t* sp = RP.row[1] + s * (32 * 12);
     P.sc[0] = ldg32(sp); P.sc[1] = ldg32(sp + 4); P.sc[2] = ldg32(sp + 8);
-    const uint8_t* lp = rec_ptr(base + L.plane[2], L, 64, R, s);
-    const uint8_t* hp = rec_ptr(base + L.plane[3], L, 32, R, s);
+    const uint8_t* lp = RP.row[2] + s * (32 * 64);
+    const uint8_t* hp = RP.row[3] + s * (32 * 32);
 #pragma unroll
     for (int ii = 0; ii < 2; ++ii) {
         const int i = 2 * hf + ii;
@@ -350,34 +356,42 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         const uint8_t* b1 = sl.ptr[p][1];
         const int rr = tid & (kMT - 1), hf = tid >> 7;   // weight row of the unit, half of each chunk
         const int64_t R = (int64_t)mt * kMT + rr;
-        const __half* src = kDown ? A.h16 : A.x16;
-        const int src_ld = K;
+        const RowPtrs RP0 = row_ptrs(f0, b0, L0, R);
+        const RowPtrs RP1 = kDown ? RP0 : row_ptrs(f1, b1, L1, R);
         __syncthreads();
-
-        // B gather of chunk c into ring slot s (cp.async, zero rows past N)
+        // B gather: this thread always moves the 16-byte piece kc = tid % 8 of
+        // rows n = tid / 8 + 32 j; the row pointers are fixed for the unit
+        const __half* src = kDown ? A.h16 : A.x16;
+        const int kcg = tid & 7, n_base = tid >> 3;
+        const __half* gsrc[kNT / 32];
+#pragma unroll
+        for (int j = 0; j < kNT / 32; ++j) {
+            const int n = n_base + 32 * j;
+            gsrc[j] = n < N ? src + (size_t)s_row[n] * K + kcg * 8 : nullptr;
+        }
         auto gather = [&](int c, int s) {
-            const uint32_t bdst = ring + s * kSlotBytes + 2 * kABytes;
-            for (int i = tid; i < Npad * 8; i += kPThreads) {
-                const int n = i >> 3, kc = i & 7;
-                const uint32_t dst = bdst + (kc * kNT + n) * 16;
-                if (n < N) {
-                    const __half* g = src + (size_t)s_row[n] * src_ld + c * kKC + kc * 8;
-                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(g) : "memory");
-                } else {
+            const uint32_t bdst = ring + s * kSlotBytes + 2 * kABytes + (kcg * kNT + n_base) * 16;
+#pragma unroll
+            for (int j = 0; j < kNT / 32; ++j) {
+                const int n = n_base + 32 * j;
+                if (n >= Npad) break;
+                const uint32_t dst = bdst + 32 * j * 16;
+                if (gsrc[j] != nullptr)
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(gsrc[j] + c * kKC) : "memory");
+                else
                     sts128(dst, 0u, 0u, 0u, 0u);
-                }
             }
         };
         gather(0, gchunk % kPSlots);
         asm volatile("cp.async.commit_group;" ::: "memory");
         Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
-        load_chunk(f0, b0, L0, R, 0, hf, P0);
-        if (!kDown) load_chunk(f1, b1, L1, R, 0, hf, P1);
+        load_chunk(f0, RP0, 0, hf, P0);
+        if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
         for (int c = 0; c < nC; ++c) {
             Packed N0, N1;             // the next chunk's, loaded while this one is decoded
             if (c + 1 < nC) {
-                load_chunk(f0, b0, L0, R, c + 1, hf, N0);
-                if (!kDown) load_chunk(f1, b1, L1, R, c + 1, hf, N1);
+                load_chunk(f0, RP0, c + 1, hf, N0);
+                if (!kDown) load_chunk(f1, RP1, c + 1, hf, N1);
             }
             const int g = gchunk + c, s = g % kPSlots;
             bool bad = false;
