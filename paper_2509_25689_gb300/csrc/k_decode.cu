@@ -148,6 +148,9 @@ __device__ __forceinline__ uint32_t lds8(uint32_t a) {
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
 constexpr int kConsumers = 8;                       // consumer warps
+constexpr int kNT = kConsumers >= 16 ? 1 : 2;       // 16-row MMA tiles per warp (of the stage's two)
+constexpr int kCols = kConsumers * kNT / 2;         // superblock columns the warps are spread over
+constexpr int kRedBufs = kConsumers >= 16 ? 1 : 2;  // item-end reduction buffers (smem budget)
 constexpr int kThreads = (kConsumers + 1) * 32;     // + one producer warp
 constexpr int kProducerWarp = kConsumers;
 constexpr int kNST = 3;                             // ring stages
@@ -284,36 +287,39 @@ __device__ __forceinline__ void ld_frag8(uint32_t a, uint32_t (&X)[8]) {
     X[0] = u.x; X[1] = u.y; X[2] = u.z; X[3] = u.w; X[4] = v.x; X[5] = v.y; X[6] = v.z; X[7] = v.w;
 }
 
-template <int FMT>
-__device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, int half, int tk, uint32_t zaddr,
-                                           float (&acc)[4]) {
+template <int FMT, int NT>
+__device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, int half, int rt0, int tk,
+                                           uint32_t zaddr, float (&acc)[4]) {
+    // rows of this warp: i = 0 .. 2 NT - 1 -> row 16 (rt0 + i / 2) + 8 (i % 2) + g
+    constexpr int NR = 2 * NT;
     const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
     const bool own0 = g == t, own1 = g == t + 4;
     const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
     const uint32_t tb = st + h.tok0 + tk * h.tstride;
     const uint32_t xb = tb + h.tx + jj * 512, sb = tb + h.ts + jj * (kStatFloats * 4);
-    const int rbase = jj * 32 + g;   // record index of row g of tile 0
+    const int rbase = jj * 32 + 16 * rt0 + g;   // record index of this lane's first row
+    auto rec_of = [&](int i) { return rbase + 16 * (i >> 1) + 8 * (i & 1); };
 
     if (FMT == kQ2K || FMT == kQ3K) {
         const uint32_t cp = FMT == kQ2K ? w3 : w2;   // 2-bit code plane
-        uint4 c[4];                                   // rows g, g+8, 16+g, 24+g
-        uint2 hv[4];
+        uint4 c[NR];
+        uint2 hv[NR];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            c[i] = lds128(st + cp + (rbase + 8 * i) * 64 + 16 * t);
-            if (FMT == kQ3K) hv[i] = lds64(st + w3 + (rbase + 8 * i) * 32 + 8 * t);
+        for (int i = 0; i < NR; ++i) {
+            c[i] = lds128(st + cp + rec_of(i) * 64 + 16 * t);
+            if (FMT == kQ3K) hv[i] = lds64(st + w3 + rec_of(i) * 32 + 8 * t);
         }
-        float DD[2][2][2][4];   // [tile][group][pair parity]
+        float DD[NT][2][2][4];   // [tile][group][pair parity]
 #pragma unroll
-        for (int i = 0; i < 32; ++i) (&DD[0][0][0][0])[i] = 0.0f;
+        for (int i = 0; i < NT * 16; ++i) (&DD[0][0][0][0])[i] = 0.0f;
 #pragma unroll
         for (int gm = 0; gm < 2; ++gm) {
             uint32_t XA[8], XB[8];
             ld_frag8(own0 ? xb + 32 * (8 * gm + t) : zaddr, XA);
             ld_frag8(own1 ? xb + 32 * (8 * gm + 4 + t) : zaddr, XB);
-            uint32_t qa[4], qb[4], sa[4], sbb[4];   // per row: sub-blocks t (a0/a1) and t+4 (a2/a3)
+            uint32_t qa[NR], qb[NR], sa[NR], sbb[NR];   // per row: sub-blocks t (a0/a1) and t+4 (a2/a3)
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
+            for (int i = 0; i < NR; ++i) {
                 qa[i] = sub4(c[i], 2 * gm); qb[i] = sub4(c[i], 2 * gm + 1);
                 sa[i] = qa[i] >> 10; sbb[i] = qb[i] >> 10;
             }
@@ -322,7 +328,7 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
                 const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
                 const bool sh = m > 4;
 #pragma unroll
-                for (int tl = 0; tl < 2; ++tl)
+                for (int tl = 0; tl < NT; ++tl)
                     mma16816(DD[tl][gm][m & 1], (sh ? sa[2 * tl] : qa[2 * tl]) & mk,
                              (sh ? sa[2 * tl + 1] : qa[2 * tl + 1]) & mk, (sh ? sbb[2 * tl] : qb[2 * tl]) & mk,
                              (sh ? sbb[2 * tl + 1] : qb[2 * tl + 1]) & mk, XA[m], XB[m]);
@@ -330,14 +336,14 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             if (FMT == kQ3K) {
                 ld_frag8(own0 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + t) : zaddr, XA);
                 ld_frag8(own1 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + 4 + t) : zaddr, XB);
-                uint32_t ha[4], hb[4];
+                uint32_t ha[NR], hb[NR];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) { ha[i] = gm ? hv[i].y : hv[i].x; hb[i] = ha[i] >> 8; }
+                for (int i = 0; i < NR; ++i) { ha[i] = gm ? hv[i].y : hv[i].x; hb[i] = ha[i] >> 8; }
 #pragma unroll
                 for (int m = 0; m < 8; ++m) {
                     const uint32_t mk = 0x00010001u << m;
 #pragma unroll
-                    for (int tl = 0; tl < 2; ++tl)
+                    for (int tl = 0; tl < NT; ++tl)
                         mma16816(DD[tl][gm][m & 1], ha[2 * tl] & mk, ha[2 * tl + 1] & mk, hb[2 * tl] & mk,
                                  hb[2 * tl + 1] & mk, XA[m], XB[m]);
                 }
@@ -349,14 +355,14 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
         const float S[4] = {__uint_as_float(Su.x), __uint_as_float(Su.y), __uint_as_float(Su.z),
                             __uint_as_float(Su.w)};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {   // row g + 8 i = tile i / 2, half i % 2
+        for (int i = 0; i < NR; ++i) {
             const int tl = i >> 1, hl = i & 1;
             float D[2][2];
 #pragma unroll
             for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
                 for (int cc = 0; cc < 2; ++cc) D[gm][cc] = DD[tl][gm][0][2 * hl + cc] + DD[tl][gm][1][2 * hl + cc];
-            const int rec = rbase + 8 * i;
+            const int rec = rec_of(i);
             const float d = h2f(lds16(st + w0 + rec * 2));
             if (FMT == kQ2K) {
                 const float dm = h2f(lds16(st + w1 + rec * 2));
@@ -380,16 +386,16 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             }
         }
     } else if (FMT == kQ4K) {
-        uint4 cA[4], cB[4];   // rows g + 8 i: sub-blocks t (unit 0) and t+4 (unit 1)
+        uint4 cA[NR], cB[NR];   // rows: sub-blocks t (unit 0) and t+4 (unit 1)
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int rec = rbase + 8 * i;
-            cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + (rec - jj * 32)) * 64 + 16 * t);
-            cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + (rec - jj * 32)) * 64 + 16 * t);
+        for (int i = 0; i < NR; ++i) {
+            const int r = rec_of(i) - jj * 32;
+            cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t);
+            cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t);
         }
-        float DD[2][2][4];   // [tile][pair parity]
+        float DD[NT][2][4];   // [tile][pair parity]
 #pragma unroll
-        for (int i = 0; i < 16; ++i) (&DD[0][0][0])[i] = 0.0f;
+        for (int i = 0; i < NT * 8; ++i) (&DD[0][0][0])[i] = 0.0f;
 #pragma unroll
         for (int hm = 0; hm < 2; ++hm) {   // pairs 8 hm .. 8 hm + 7
             uint32_t XA[8], XB[8];
@@ -401,7 +407,7 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
                 const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
                 const int sh = j < 2 ? 0 : 8;
 #pragma unroll
-                for (int tl = 0; tl < 2; ++tl)
+                for (int tl = 0; tl < NT; ++tl)
                     mma16816(DD[tl][m & 1], (sub4(cA[2 * tl], wi) >> sh) & mk, (sub4(cA[2 * tl + 1], wi) >> sh) & mk,
                              (sub4(cB[2 * tl], wi) >> sh) & mk, (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[mm], XB[mm]);
             }
@@ -410,8 +416,8 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
         const float cf0 = __uint_as_float(Cu.x), cf1 = __uint_as_float(Cu.y);
         const float S0 = __uint_as_float(Su.x), S1 = __uint_as_float(Su.y);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int tl = i >> 1, hl = i & 1, rec = rbase + 8 * i;
+        for (int i = 0; i < NR; ++i) {
+            const int tl = i >> 1, hl = i & 1, rec = rec_of(i);
             const float d = h2f(lds16(st + w0 + rec * 2));
             const float dm = h2f(lds16(st + w1 + rec * 2));
             const uint32_t sp = st + w2 + rec * 12;
@@ -426,24 +432,24 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             acc[i] += fmaf(d, a_sc, -dm * a_m);
         }
     } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7
-        uint4 cA[4], cB[4];   // rows g + 8 i: blocks t and t+4
+        uint4 cA[NR], cB[NR];   // rows: blocks t and t+4
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int r = g + 8 * i;
+        for (int i = 0; i < NR; ++i) {
+            const int r = rec_of(i) - jj * 32;
             cA[i] = lds128(st + w1 + ((8 * jj + t) * 32 + r) * 32 + 16 * half);
             cB[i] = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r) * 32 + 16 * half);
         }
         uint32_t XA[8], XB[8];
         ld_frag8(own0 ? xb + 64 * t + 32 * half : zaddr, XA);
         ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * half : zaddr, XB);
-        float DD[2][2][4];
+        float DD[NT][2][4];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) (&DD[0][0][0])[i] = 0.0f;
+        for (int i = 0; i < NT * 8; ++i) (&DD[0][0][0])[i] = 0.0f;
 #pragma unroll
         for (int mm = 0; mm < 8; ++mm) {
             const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0;
 #pragma unroll
-            for (int tl = 0; tl < 2; ++tl)
+            for (int tl = 0; tl < NT; ++tl)
                 mma16816(DD[tl][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
                          (sub4(cA[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, (sub4(cB[2 * tl], wi) >> sh) & 0x00FF00FFu,
                          (sub4(cB[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, XA[mm], XB[mm]);
@@ -454,8 +460,8 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
         const float o0 = half ? 0.0f : 128.0f * __uint_as_float(Su.x);
         const float o1 = half ? 0.0f : 128.0f * __uint_as_float(Su.y);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int tl = i >> 1, hl = i & 1, r = g + 8 * i;
+        for (int i = 0; i < NR; ++i) {
+            const int tl = i >> 1, hl = i & 1, r = rec_of(i) - jj * 32;
             const float d0 = h2f(lds16(st + w0 + ((8 * jj + 2 * t) * 32 + r) * 2));
             const float d1 = h2f(lds16(st + w0 + ((8 * jj + 2 * t + 1) * 32 + r) * 2));
             const float D0 = DD[tl][0][2 * hl] + DD[tl][1][2 * hl], D1 = DD[tl][0][2 * hl + 1] + DD[tl][1][2 * hl + 1];
@@ -474,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     __shared__ int32_t s_perm[kMaxCachedAssign];
     __shared__ __align__(8) uint64_t bars[2 * kNST];
     __shared__ Hdr hdr[kNST];
-    __shared__ float red[2][kConsumers][2][kDecodeTok][32];   // double-buffered by item parity
+    __shared__ float red[kRedBufs][kConsumers][2][kDecodeTok][32];
     __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
@@ -626,8 +632,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         }
     } else {
         // ============================ consumer warps =============================
-        // warp w: all 32 rows of the stage, superblocks w, w + 8, ... (Q8_0:
-        // both halves of the code pairs of each)
+        // warp w: row tiles rt0 .. rt0 + kNT - 1 of the stage's 32 rows and
+        // superblocks col, col + kCols, ... (Q8_0: both halves of the code
+        // pairs of each)
+        const int rt0 = kNT == 2 ? 0 : (warp & 1), col = kNT == 2 ? warp : (warp >> 1);
         float acc[2][kDecodeTok][4];   // [0] gate (or down), [1] up; rows g + 8 i
         float cur[kDecodeTok][4];      // the tensor being streamed
 #pragma unroll
@@ -657,16 +665,16 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             for (int tk = 0; tk < kDecodeTok; ++tk) {
                 if (tk >= ntok) break;
                 if (fmt == kQ80) {
-                    for (int jj = warp; jj < ks; jj += kConsumers) {
-                        tile_block<kQ80>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
-                        tile_block<kQ80>(GS, stage, jj, 1, tk, zaddr, cur[tk]);
+                    for (int jj = col; jj < ks; jj += kCols) {
+                        tile_block<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
+                        tile_block<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, zaddr, cur[tk]);
                     }
                 } else if (fmt == kQ2K) {
-                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ2K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ2K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
                 } else if (fmt == kQ3K) {
-                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ3K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ3K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
                 } else {
-                    for (int jj = warp; jj < ks; jj += kConsumers) tile_block<kQ4K>(GS, stage, jj, 0, tk, zaddr, cur[tk]);
+                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ4K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
                 }
             }
             // fields needed after the slot is released to the producer
@@ -684,17 +692,20 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 
             // ---- item done: the streamed tensor's sums go to acc[1] (up) or acc[0]
             const int g = lane >> 2, t4 = lane & 3;
-            const int buf = n_done & 1;
+            const int buf = kRedBufs == 2 ? (n_done & 1) : 0;
 #pragma unroll
             for (int u = 0; u < (kDown ? 1 : 2); ++u)
 #pragma unroll
                 for (int tk = 0; tk < kDecodeTok; ++tk)
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
+                    for (int i = 0; i < 2 * kNT; ++i) {
                         float v = (u == (kDown ? 0 : 1)) ? acc[u][tk][i] + cur[tk][i] : acc[u][tk][i];
                         v += __shfl_xor_sync(kFull, v, 1);
                         v += __shfl_xor_sync(kFull, v, 2);
-                        if (t4 == 0) red[buf][warp][u][tk][8 * i + g] = v;
+                        if (t4 == 0) {
+                            red[buf][warp][u][tk][16 * rt0 + 8 * i + g] = v;
+                            if (kNT == 1) red[buf][warp][u][tk][16 * (1 - rt0) + 8 * i + g] = 0.0f;
+                        }
                     }
 #pragma unroll
             for (int tk = 0; tk < kDecodeTok; ++tk)
@@ -729,8 +740,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         for (int jb = n_rb; jb < 8 * A.nsbi; ++jb) prep_block32(0.0f, jb, fam, hq, hs, A.nsbi);
                 }
             }
-            // no barrier here: the next item end writes the other reduction buffer,
-            // and its barrier orders these reads before the buffer is reused
+            // with two buffers the next item end writes the other one and its
+            // barrier orders these reads before reuse; with one, wait here
+            if (kRedBufs == 1) consumer_sync();
             ++n_done;
         }
     }
