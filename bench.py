@@ -135,7 +135,8 @@ def step_bytes(spec, fmts, idx_steps):
         b_rt = E * H * 4 + T * H * 2 + T * E * 4
         quant = sum(gu(e) + dn(e) for e in touched) + ((gu(sh) + dn(sh)) if sh is not None else 0)
         out.append({"gateup_mma": b_gu, "down_mma": b_dn, "router_logits": b_rt, "quantized": quant,
-                    "total": b_gu + b_dn + b_rt, "gateup_tc": b_gu, "down_tc": b_dn})
+                    "total": b_gu + b_dn + b_rt, "gateup_tc": b_gu, "down_tc": b_dn,
+                    "gateup_tgemv": b_gu, "down_tgemv": b_dn})
     return out
 
 

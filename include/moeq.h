@@ -194,9 +194,13 @@ int moe_quant_route(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
 const char* mq_strerror(int status);
 
 /* Path selection: 0 = automatic (n_tokens >= threshold -> prefill grouped
- * GEMM, else decode GEMV), 1 = force decode, 2 = force prefill.  Process
- * wide; the MQ_FORCE_PATH environment variable ("decode"/"prefill") sets the
- * initial value.  threshold <= 0 keeps the current one (default 64). */
+ * GEMM, else decode GEMV), 1 = force decode, 2 = force prefill, 3 = force
+ * decode on the alternative tcgen05 GEMV kernels (A operand in tensor
+ * memory; slower than the default mma.sync GEMV at decode sizes, kept as a
+ * second implementation).  Process wide; the MQ_FORCE_PATH environment
+ * variable ("decode"/"prefill"/"decode_tc") sets the initial value.
+ * threshold <= 0 keeps the current one (default 64).  Returns MQ_EINVAL for
+ * another mode. */
 int mq_set_path(int mode, int32_t prefill_threshold);
 
 /* Kernel timing for measurement tools.  mq_profile_enable(n) makes the next

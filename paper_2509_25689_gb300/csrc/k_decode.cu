@@ -287,18 +287,28 @@ __device__ __forceinline__ void ld_frag8(uint32_t a, uint32_t (&X)[8]) {
     X[0] = u.x; X[1] = u.y; X[2] = u.z; X[3] = u.w; X[4] = v.x; X[5] = v.y; X[6] = v.z; X[7] = v.w;
 }
 
+// A tile's MMA sums: [tile][sub-block group][pair parity][D fragment]
+// (Q2_K / Q3_K use both groups, Q4_K / Q8_0 only group 0).
+template <int NT> struct TileAcc { float DD[NT][2][2][4]; };
+
+// Loads one (superblock, token) tile of the warp's rows and issues its MMAs
+// into T; tile_epi applies the scales once the sums are in.  Callers issue the
+// MMAs of the next tile before the epilogue of the current one, so the MMA
+// latency of one tile runs under the other's epilogue.
 template <int FMT, int NT>
-__device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, int half, int rt0, int tk,
-                                           uint32_t zaddr, float (&acc)[4]) {
+__device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int half, int rt0, int tk,
+                                         uint32_t zaddr, TileAcc<NT>& T) {
     // rows of this warp: i = 0 .. 2 NT - 1 -> row 16 (rt0 + i / 2) + 8 (i % 2) + g
     constexpr int NR = 2 * NT;
     const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
     const bool own0 = g == t, own1 = g == t + 4;
-    const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
+    const int w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
     const uint32_t tb = st + h.tok0 + tk * h.tstride;
-    const uint32_t xb = tb + h.tx + jj * 512, sb = tb + h.ts + jj * (kStatFloats * 4);
+    const uint32_t xb = tb + h.tx + jj * 512;
     const int rbase = jj * 32 + 16 * rt0 + g;   // record index of this lane's first row
     auto rec_of = [&](int i) { return rbase + 16 * (i >> 1) + 8 * (i & 1); };
+#pragma unroll
+    for (int i = 0; i < NT * 16; ++i) (&T.DD[0][0][0][0])[i] = 0.0f;
 
     if (FMT == kQ2K || FMT == kQ3K) {
         const uint32_t cp = FMT == kQ2K ? w3 : w2;   // 2-bit code plane
@@ -309,9 +319,6 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             c[i] = lds128(st + cp + rec_of(i) * 64 + 16 * t);
             if (FMT == kQ3K) hv[i] = lds64(st + w3 + rec_of(i) * 32 + 8 * t);
         }
-        float DD[NT][2][2][4];   // [tile][group][pair parity]
-#pragma unroll
-        for (int i = 0; i < NT * 16; ++i) (&DD[0][0][0][0])[i] = 0.0f;
 #pragma unroll
         for (int gm = 0; gm < 2; ++gm) {
             uint32_t XA[8], XB[8];
@@ -329,7 +336,7 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
                 const bool sh = m > 4;
 #pragma unroll
                 for (int tl = 0; tl < NT; ++tl)
-                    mma16816(DD[tl][gm][m & 1], (sh ? sa[2 * tl] : qa[2 * tl]) & mk,
+                    mma16816(T.DD[tl][gm][m & 1], (sh ? sa[2 * tl] : qa[2 * tl]) & mk,
                              (sh ? sa[2 * tl + 1] : qa[2 * tl + 1]) & mk, (sh ? sbb[2 * tl] : qb[2 * tl]) & mk,
                              (sh ? sbb[2 * tl + 1] : qb[2 * tl + 1]) & mk, XA[m], XB[m]);
             }
@@ -344,12 +351,72 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
                     const uint32_t mk = 0x00010001u << m;
 #pragma unroll
                     for (int tl = 0; tl < NT; ++tl)
-                        mma16816(DD[tl][gm][m & 1], ha[2 * tl] & mk, ha[2 * tl + 1] & mk, hb[2 * tl] & mk,
+                        mma16816(T.DD[tl][gm][m & 1], ha[2 * tl] & mk, ha[2 * tl + 1] & mk, hb[2 * tl] & mk,
                                  hb[2 * tl + 1] & mk, XA[m], XB[m]);
                 }
             }
         }
-        // ---- epilogue: slot-ordered scale word of each row: bytes b = 2*group + col
+    } else if (FMT == kQ4K) {
+        uint4 cA[NR], cB[NR];   // rows: sub-blocks t (unit 0) and t+4 (unit 1)
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int r = rec_of(i) - jj * 32;
+            cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t);
+            cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t);
+        }
+#pragma unroll
+        for (int hm = 0; hm < 2; ++hm) {   // pairs 8 hm .. 8 hm + 7
+            uint32_t XA[8], XB[8];
+            ld_frag8(own0 ? xb + 64 * t + 32 * hm : zaddr, XA);
+            ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * hm : zaddr, XB);
+#pragma unroll
+            for (int mm = 0; mm < 8; ++mm) {
+                const int m = 8 * hm + mm, wi = m >> 2, j = m & 3;
+                const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
+                const int sh = j < 2 ? 0 : 8;
+#pragma unroll
+                for (int tl = 0; tl < NT; ++tl)
+                    mma16816(T.DD[tl][0][m & 1], (sub4(cA[2 * tl], wi) >> sh) & mk,
+                             (sub4(cA[2 * tl + 1], wi) >> sh) & mk, (sub4(cB[2 * tl], wi) >> sh) & mk,
+                             (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[mm], XB[mm]);
+            }
+        }
+    } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7
+        uint4 cA[NR], cB[NR];   // rows: blocks t and t+4
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int r = rec_of(i) - jj * 32;
+            cA[i] = lds128(st + w1 + ((8 * jj + t) * 32 + r) * 32 + 16 * half);
+            cB[i] = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r) * 32 + 16 * half);
+        }
+        uint32_t XA[8], XB[8];
+        ld_frag8(own0 ? xb + 64 * t + 32 * half : zaddr, XA);
+        ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * half : zaddr, XB);
+#pragma unroll
+        for (int mm = 0; mm < 8; ++mm) {
+            const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0;
+#pragma unroll
+            for (int tl = 0; tl < NT; ++tl)
+                mma16816(T.DD[tl][0][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
+                         (sub4(cA[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, (sub4(cB[2 * tl], wi) >> sh) & 0x00FF00FFu,
+                         (sub4(cB[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, XA[mm], XB[mm]);
+        }
+    }
+}
+
+template <int FMT, int NT>
+__device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int half, int rt0, int tk,
+                                         const TileAcc<NT>& T, float (&acc)[4]) {
+    constexpr int NR = 2 * NT;
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2];
+    const uint32_t tb = st + h.tok0 + tk * h.tstride;
+    const uint32_t sb = tb + h.ts + jj * (kStatFloats * 4);
+    const int rbase = jj * 32 + 16 * rt0 + g;
+    auto rec_of = [&](int i) { return rbase + 16 * (i >> 1) + 8 * (i & 1); };
+
+    if (FMT == kQ2K || FMT == kQ3K) {
+        // slot-ordered scale word of each row: bytes b = 2*group + col
         const float cf0 = ldsf(sb + 4 * (kStatC + t)), cf1 = ldsf(sb + 4 * (kStatC + 4 + t));
         const uint4 Su = lds128(sb + 4 * (kStatS16 + 4 * t));
         const float S[4] = {__uint_as_float(Su.x), __uint_as_float(Su.y), __uint_as_float(Su.z),
@@ -361,7 +428,8 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
 #pragma unroll
             for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
-                for (int cc = 0; cc < 2; ++cc) D[gm][cc] = DD[tl][gm][0][2 * hl + cc] + DD[tl][gm][1][2 * hl + cc];
+                for (int cc = 0; cc < 2; ++cc)
+                    D[gm][cc] = T.DD[tl][gm][0][2 * hl + cc] + T.DD[tl][gm][1][2 * hl + cc];
             const int rec = rec_of(i);
             const float d = h2f(lds16(st + w0 + rec * 2));
             if (FMT == kQ2K) {
@@ -386,32 +454,6 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             }
         }
     } else if (FMT == kQ4K) {
-        uint4 cA[NR], cB[NR];   // rows: sub-blocks t (unit 0) and t+4 (unit 1)
-#pragma unroll
-        for (int i = 0; i < NR; ++i) {
-            const int r = rec_of(i) - jj * 32;
-            cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t);
-            cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t);
-        }
-        float DD[NT][2][4];   // [tile][pair parity]
-#pragma unroll
-        for (int i = 0; i < NT * 8; ++i) (&DD[0][0][0])[i] = 0.0f;
-#pragma unroll
-        for (int hm = 0; hm < 2; ++hm) {   // pairs 8 hm .. 8 hm + 7
-            uint32_t XA[8], XB[8];
-            ld_frag8(own0 ? xb + 64 * t + 32 * hm : zaddr, XA);
-            ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * hm : zaddr, XB);
-#pragma unroll
-            for (int mm = 0; mm < 8; ++mm) {
-                const int m = 8 * hm + mm, wi = m >> 2, j = m & 3;
-                const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
-                const int sh = j < 2 ? 0 : 8;
-#pragma unroll
-                for (int tl = 0; tl < NT; ++tl)
-                    mma16816(DD[tl][m & 1], (sub4(cA[2 * tl], wi) >> sh) & mk, (sub4(cA[2 * tl + 1], wi) >> sh) & mk,
-                             (sub4(cB[2 * tl], wi) >> sh) & mk, (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[mm], XB[mm]);
-            }
-        }
         const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
         const float cf0 = __uint_as_float(Cu.x), cf1 = __uint_as_float(Cu.y);
         const float S0 = __uint_as_float(Su.x), S1 = __uint_as_float(Su.y);
@@ -426,34 +468,13 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             const float m0 = (float)(((f >> 4) & 15u) | (((hi >> 2) & 3u) << 4));
             const float sc1 = (float)(((f >> 8) & 15u) | (((hi >> 4) & 3u) << 4));
             const float m1 = (float)(((f >> 12) & 15u) | (((hi >> 6) & 3u) << 4));
-            const float D0 = DD[tl][0][2 * hl] + DD[tl][1][2 * hl], D1 = DD[tl][0][2 * hl + 1] + DD[tl][1][2 * hl + 1];
+            const float D0 = T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl];
+            const float D1 = T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1];
             const float a_sc = fmaf(sc1 * cf1, D1, sc0 * cf0 * D0);
             const float a_m = fmaf(m1, S1, m0 * S0);
             acc[i] += fmaf(d, a_sc, -dm * a_m);
         }
-    } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7
-        uint4 cA[NR], cB[NR];   // rows: blocks t and t+4
-#pragma unroll
-        for (int i = 0; i < NR; ++i) {
-            const int r = rec_of(i) - jj * 32;
-            cA[i] = lds128(st + w1 + ((8 * jj + t) * 32 + r) * 32 + 16 * half);
-            cB[i] = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r) * 32 + 16 * half);
-        }
-        uint32_t XA[8], XB[8];
-        ld_frag8(own0 ? xb + 64 * t + 32 * half : zaddr, XA);
-        ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * half : zaddr, XB);
-        float DD[NT][2][4];
-#pragma unroll
-        for (int i = 0; i < NT * 8; ++i) (&DD[0][0][0])[i] = 0.0f;
-#pragma unroll
-        for (int mm = 0; mm < 8; ++mm) {
-            const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0;
-#pragma unroll
-            for (int tl = 0; tl < NT; ++tl)
-                mma16816(DD[tl][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
-                         (sub4(cA[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, (sub4(cB[2 * tl], wi) >> sh) & 0x00FF00FFu,
-                         (sub4(cB[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, XA[mm], XB[mm]);
-        }
+    } else {
         const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
         const float cf0 = __uint_as_float(Cu.x), cf1 = __uint_as_float(Cu.y);
         // codes are stored q + 128: one half removes 128 * sum(x) per block
@@ -464,17 +485,40 @@ __device__ __forceinline__ void tile_block(const Geo& h, uint32_t st, int jj, in
             const int tl = i >> 1, hl = i & 1, r = rec_of(i) - jj * 32;
             const float d0 = h2f(lds16(st + w0 + ((8 * jj + 2 * t) * 32 + r) * 2));
             const float d1 = h2f(lds16(st + w0 + ((8 * jj + 2 * t + 1) * 32 + r) * 2));
-            const float D0 = DD[tl][0][2 * hl] + DD[tl][1][2 * hl], D1 = DD[tl][0][2 * hl + 1] + DD[tl][1][2 * hl + 1];
+            const float D0 = T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl];
+            const float D1 = T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1];
             acc[i] += fmaf(d1, fmaf(D1, cf1, -o1), d0 * fmaf(D0, cf0, -o0));
         }
     }
 }
 
-template <bool kDown>
+// The warp's superblocks col, col + kCols, ... of a stage.  PAIR: two at a
+// time, the second tile's MMAs issued before the first tile's epilogue.
+template <int FMT, bool PAIR>
+__device__ __forceinline__ void tile_pairs(const Geo& h, uint32_t st, int col, int ks, int rt0, int tk,
+                                           uint32_t zaddr, float (&acc)[4]) {
+    if (PAIR) {
+        for (int jj = col; jj < ks; jj += 2 * kCols) {
+            const bool two = jj + kCols < ks;
+            TileAcc<kNT> T0, T1;
+            tile_mma<FMT, kNT>(h, st, jj, 0, rt0, tk, zaddr, T0);
+            if (two) tile_mma<FMT, kNT>(h, st, jj + kCols, 0, rt0, tk, zaddr, T1);
+            tile_epi<FMT, kNT>(h, st, jj, 0, rt0, tk, T0, acc);
+            if (two) tile_epi<FMT, kNT>(h, st, jj + kCols, 0, rt0, tk, T1, acc);
+        }
+    } else {
+        for (int jj = col; jj < ks; jj += kCols) {
+            TileAcc<kNT> T0;
+            tile_mma<FMT, kNT>(h, st, jj, 0, rt0, tk, zaddr, T0);
+            tile_epi<FMT, kNT>(h, st, jj, 0, rt0, tk, T0, acc);
+        }
+    }
+}
+
+// MT: most tokens an item of this launch carries (1 when the call has one token)
+template <bool kDown, int MT>
 __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant__ ExpertTab tab,
                                                           const __grid_constant__ DecodeArgs A) {
-    pdl_wait();
-    pdl_launch();
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
@@ -484,25 +528,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
-    const Dims& d = A.d;
-    const int n_slots = A.plan->n_slots;
     __shared__ Geo geo[4][kDecodeTok];
-    for (int i = threadIdx.x; i <= n_slots; i += blockDim.x) {
-        sc.pre[i] = kDown ? A.plan->pre_dn[i] : A.plan->pre_gu[i];
-        if (i < n_slots) {
-            int e;
-            if (i < d.has_shared) { e = d.E; sc.first[i] = 0; sc.ntot[i] = d.T; }
-            else {
-                e = A.active[1 + i - d.has_shared];
-                sc.first[i] = A.offsets[e]; sc.ntot[i] = A.offsets[e + 1] - A.offsets[e];
-            }
-            sc.e[i] = e;
-            sc.ptr[i] = tab.p[e][kDown ? 2 : 0];
-            sc.ptr_up[i] = tab.p[e][1];
-            sc.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
-            sc.fmt[i][1] = tab.fmt[e][1];
-        }
-    }
+    const Dims& d = A.d;
+    // ---- set-up that does not depend on the routing result runs before the
+    // wait for the previous kernel (overlapping its tail)
     if (threadIdx.x < 4 * kDecodeTok) {
         const int fmt = 1 + threadIdx.x / kDecodeTok, ntok = 1 + threadIdx.x % kDecodeTok;
         Geo& G = geo[fmt - 1][ntok - 1];
@@ -524,8 +553,6 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         const TokLay tl = tok_lay(fmt, G.per);
         G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.tx1 = tl.x1; G.ts = tl.s;
     }
-    const int n_routed = min(d.T * d.K, kMaxCachedAssign);
-    for (int i = threadIdx.x; i < n_routed; i += blockDim.x) s_perm[i] = A.perm[i];
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
     if (threadIdx.x < kNST) s_posted[threadIdx.x] = -1;
     if (threadIdx.x < 8) zero_blk[threadIdx.x] = 0u;
@@ -538,8 +565,20 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
+    // The shared expert's gate/up items (item ids 0 .. n_sh_items - 1) need no
+    // routing result: its slot is known from the shapes, so they start before
+    // the wait for the routing kernel.  (The tokens' prepared activations come
+    // from the logits kernel, which completed before the routing kernel let
+    // this grid launch.)
+    const int n_sh_items = (!kDown && d.has_shared) ? (d.I / 32) * ((d.T + kDecodeTok - 1) / kDecodeTok) : 0;
+    if (threadIdx.x == 0 && n_sh_items > 0) {
+        sc.pre[0] = 0; sc.pre[1] = n_sh_items;
+        sc.e[0] = d.E; sc.first[0] = 0; sc.ntot[0] = d.T;
+        sc.ptr[0] = tab.p[d.E][0]; sc.ptr_up[0] = tab.p[d.E][1];
+        sc.fmt[0][0] = tab.fmt[d.E][0]; sc.fmt[0][1] = tab.fmt[d.E][1];
+    }
     __syncthreads();
-    const int n_items = sc.pre[n_slots];
+    pdl_launch();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
 
@@ -556,9 +595,50 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         const int p_nsb = vs.nsb;
         ItemDesc P;
         int pslot = 0;
+        // the routing result: slot table (one level of independent loads; the
+        // plan holds each slot's expert, first entry and token count) and the
+        // cached permutation
+        int n_slots = n_sh_items > 0 ? 1 : 0, n_items = n_sh_items;
+        bool routed = false;
+        auto wait_routing = [&]() {
+            pdl_wait();
+            n_slots = A.plan->n_slots;
+            for (int i = lane; i < kMaxExperts + 2; i += 32) {
+                const int pre = kDown ? A.plan->pre_dn[i] : A.plan->pre_gu[i];
+                const int e = A.plan->slot_e[i], first = A.plan->slot_first[i], ntot = A.plan->slot_ntot[i];
+                if (i <= n_slots) sc.pre[i] = pre;
+                if (i < n_slots) {
+                    sc.e[i] = e;
+                    sc.first[i] = first;
+                    sc.ntot[i] = ntot;
+                    sc.ptr[i] = tab.p[e][kDown ? 2 : 0];
+                    sc.ptr_up[i] = tab.p[e][1];
+                    sc.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
+                    sc.fmt[i][1] = tab.fmt[e][1];
+                }
+            }
+            const int n_routed = min(d.T * d.K, kMaxCachedAssign);
+            for (int i = lane; i < n_routed; i += 32) s_perm[i] = A.perm[i];
+            __syncwarp();
+            n_items = sc.pre[n_slots];
+            routed = true;
+        };
+        if (n_sh_items == 0) wait_routing();
+        // items are handed out by a global counter (zeroed per call), in slot
+        // order: the shared expert's (Q8_0, the heaviest) first, so the CTAs
+        // even out on the lighter routed items that follow
+        int id_next = 0;
+        if (lane == 0) id_next = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+        id_next = __shfl_sync(kFull, id_next, 0);
         for (int k = 0;; ++k) {
-            const int id = blockIdx.x + k * gridDim.x;
+            const int id = id_next;
+            if (!routed && id >= n_sh_items) wait_routing();
             const int item = id < n_items ? id : -1;
+            if (item >= 0) {
+                // claim the following item now; the atomic's latency hides behind this item's stages
+                if (lane == 0) id_next = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+                id_next = __shfl_sync(kFull, id_next, 0);
+            }
             if (item >= 0) decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
             const int nst = item >= 0 ? P.nst : 1;
             bool failed = false;
@@ -636,10 +716,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // superblocks col, col + kCols, ... (Q8_0: both halves of the code
         // pairs of each)
         const int rt0 = kNT == 2 ? 0 : (warp & 1), col = kNT == 2 ? warp : (warp >> 1);
-        float acc[2][kDecodeTok][4];   // [0] gate (or down), [1] up; rows g + 8 i
-        float cur[kDecodeTok][4];      // the tensor being streamed
+        float acc[2][MT][4];   // [0] gate (or down), [1] up; rows g + 8 i
+        float cur[MT][4];      // the tensor being streamed
 #pragma unroll
-        for (int tk = 0; tk < kDecodeTok; ++tk)
+        for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
             for (int i = 0; i < 4; ++i) acc[0][tk][i] = acc[1][tk][i] = cur[tk][i] = 0.0f;
         int n_done = 0;   // items finished by this CTA (selects the reduction buffer and the owner warps)
@@ -657,24 +737,31 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             if (!kDown && H.tensor == 1 && H.s0 == 0) {
                 // first stage of the up tensor: the gate sums are complete
 #pragma unroll
-                for (int tk = 0; tk < kDecodeTok; ++tk)
+                for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
                     for (int i = 0; i < 4; ++i) { acc[0][tk][i] += cur[tk][i]; cur[tk][i] = 0.0f; }
             }
 #pragma unroll
-            for (int tk = 0; tk < kDecodeTok; ++tk) {
+            for (int tk = 0; tk < MT; ++tk) {
                 if (tk >= ntok) break;
+                // one-token items have the registers to keep two tiles of MMA sums
+                // in flight (Q3_K's second code plane does not fit them)
+                constexpr bool kPair = MT == 1;
                 if (fmt == kQ80) {
                     for (int jj = col; jj < ks; jj += kCols) {
-                        tile_block<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
-                        tile_block<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, zaddr, cur[tk]);
+                        TileAcc<kNT> T0, T1;
+                        tile_mma<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, T0);
+                        if (!kPair) tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
+                        tile_mma<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, zaddr, T1);
+                        if (kPair) tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
+                        tile_epi<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, T1, cur[tk]);
                     }
                 } else if (fmt == kQ2K) {
-                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ2K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ2K, kPair>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
                 } else if (fmt == kQ3K) {
-                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ3K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ3K, false>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
                 } else {
-                    for (int jj = col; jj < ks; jj += kCols) tile_block<kQ4K, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ4K, kPair>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
                 }
             }
             // fields needed after the slot is released to the producer
@@ -696,7 +783,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 #pragma unroll
             for (int u = 0; u < (kDown ? 1 : 2); ++u)
 #pragma unroll
-                for (int tk = 0; tk < kDecodeTok; ++tk)
+                for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
                     for (int i = 0; i < 2 * kNT; ++i) {
                         float v = (u == (kDown ? 0 : 1)) ? acc[u][tk][i] + cur[tk][i] : acc[u][tk][i];
@@ -708,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         }
                     }
 #pragma unroll
-            for (int tk = 0; tk < kDecodeTok; ++tk)
+            for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) acc[0][tk][i] = acc[1][tk][i] = cur[tk][i] = 0.0f;
             consumer_sync();
@@ -729,6 +816,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
                 } else {
                     // SwiGLU (routing weight folded in), then prepare h for the down projection
+                    if (!e_shared) pdl_wait();   // routing weights come from the routing kernel
                     const float w = e_shared ? 1.0f : A.wts[a];
                     const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
                     const int fam = families_of(tab.fmt[e_e][2]);
@@ -786,8 +874,10 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
         if (g_num_sms <= 0) g_num_sms = 148;
-        cudaFuncSetAttribute(ffn_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        cudaFuncSetAttribute(ffn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(ffn_kernel<false, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(ffn_kernel<true, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(ffn_kernel<false, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(ffn_kernel<true, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     }
     DecodeArgs A;
     A.d = d;
@@ -800,12 +890,16 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.next = w.counters;
     A.err = w.err;
     A.out = out;
+    // one token: every item carries one, and the accumulators shrink to one token's
+    const bool one = d.T == 1;
     prof_begin("gateup_mma", s);
-    cudaError_t err = launch_pdl(ffn_kernel<false>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
+    cudaError_t err = one ? launch_pdl(ffn_kernel<false, 1>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A)
+                          : launch_pdl(ffn_kernel<false, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     prof_begin("down_mma", s);
-    err = launch_pdl(ffn_kernel<true>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
+    err = one ? launch_pdl(ffn_kernel<true, 1>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A)
+              : launch_pdl(ffn_kernel<true, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);

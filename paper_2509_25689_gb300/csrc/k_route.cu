@@ -374,10 +374,13 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 #pragma unroll
         for (int q = 0; q < 9; ++q) {
             const int p = lane * 9 + q;
-            int ntok = 0;
+            int ntok = 0, e = d.E, first = 0;
             if (p < n_slots) {
                 if (p < d.has_shared) ntok = d.T;
-                else { const int e = s_act[1 + p - d.has_shared]; ntok = s_off[e + 1] - s_off[e]; }
+                else { e = s_act[1 + p - d.has_shared]; first = s_off[e]; ntok = s_off[e + 1] - first; }
+                plan->slot_e[p] = e;
+                plan->slot_first[p] = first;
+                plan->slot_ntot[p] = ntok;
             }
             const int ntg = (ntok + kDecodeTok - 1) / kDecodeTok;
             cg[q] = (d.I / 32) * ntg;     // gate/up items: 32 rows x both tensors x full K

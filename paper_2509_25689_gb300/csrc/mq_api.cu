@@ -29,6 +29,7 @@ int path_mode() {
         g_path_mode = 0;
         if (env && std::strcmp(env, "decode") == 0) g_path_mode = 1;
         if (env && std::strcmp(env, "prefill") == 0) g_path_mode = 2;
+        if (env && std::strcmp(env, "decode_tc") == 0) g_path_mode = 3;
     }
     return g_path_mode;
 }
@@ -148,7 +149,7 @@ extern "C" const char* mq_strerror(int status) {
 }
 
 extern "C" int mq_set_path(int mode, int32_t prefill_threshold) {
-    if (mode < 0 || mode > 2) return MQ_EINVAL;
+    if (mode < 0 || mode > 3) return MQ_EINVAL;
     path_mode();
     g_path_mode = mode;
     if (prefill_threshold > 0) g_prefill_threshold = prefill_threshold;
@@ -254,7 +255,9 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
         if (launch_prefill(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
         return MQ_OK;
     }
-    if (launch_decode_mma(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
+    const cudaError_t e = (pm == 3 && decode_tc_fits(d)) ? launch_decode_tc(d, tab, w, out, s)
+                                                         : launch_decode_mma(d, tab, w, out, s);
+    if (e != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
 }
 

@@ -37,6 +37,10 @@ struct Plan {
     int32_t pad;
     int32_t pre_gu[kMaxExperts + 2];
     int32_t pre_dn[kMaxExperts + 2];
+    // per slot: expert id (E = shared), first entry of its tokens in perm, token count
+    int32_t slot_e[kMaxExperts + 2];
+    int32_t slot_first[kMaxExperts + 2];
+    int32_t slot_ntot[kMaxExperts + 2];
 };
 
 // Carved out of the caller's workspace (see workspace_plan).
@@ -103,6 +107,9 @@ cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bia
 cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s);
 cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
+// tcgen05 decode kernels: need hidden and inter to be multiples of 128
+bool decode_tc_fits(const Dims& d);
+cudaError_t launch_decode_tc(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 size_t decode_counter_bytes(const Dims& d);
 cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);
 

@@ -97,7 +97,16 @@ def test_routing_tie_break_on_device(torch_cuda, orc):
 
 
 # --------------------------------------------------------------- forward ---
-def test_forward_tiny_layer(torch_cuda, orc):
+@pytest.fixture(params=[1, 3], ids=["mma", "tc"])
+def decode_kernel(request):
+    """Decode path on the mma.sync GEMV kernels (1) or the tcgen05 ones (3)."""
+    mq = mq_lib()
+    mq.mq_set_path(request.param)
+    yield request.param
+    mq.mq_set_path(0)
+
+
+def test_forward_tiny_layer(torch_cuda, orc, decode_kernel):
     spec = get_config("tiny")
     layer = DeviceLayer(spec, 0, orc=orc)
     x = tokens(spec, 0)
@@ -109,7 +118,7 @@ def test_forward_tiny_layer(torch_cuda, orc):
 
 
 @pytest.mark.parametrize("T", [1, 3, 5, 9])
-def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T):
+def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T, decode_kernel):
     spec = LayerSpec(name="small_mixed", hidden=512, inter=256, n_experts=12, n_groups=4, topk_group=2,
                      top_k=3, tokens=T, has_shared=True, mixed=True, router_std=1 / 22.6, bias_std=0.01)
     fm = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
@@ -121,7 +130,7 @@ def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T):
     assert_close(y, ry)
 
 
-def test_forward_v3_decode_t1(torch_cuda, orc):
+def test_forward_v3_decode_t1(torch_cuda, orc, decode_kernel):
     spec = get_config("v3_decode_t1")
     layer = DeviceLayer(spec, 0)
     x = tokens(spec, 0)
@@ -131,7 +140,7 @@ def test_forward_v3_decode_t1(torch_cuda, orc):
     assert_close(y, ry)
 
 
-def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc):
+def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc, decode_kernel):
     spec = get_config("v3_decode_t32_mixed")
     layer = DeviceLayer(spec, 0)
     x = tokens(spec, 0)
