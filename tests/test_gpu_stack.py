@@ -1,0 +1,54 @@
+"""The layer-stack workload: independent V3-shaped layers (each with its own
+mixed-format experts and shared expert) called back to back and captured in
+one CUDA graph, as the stack benchmark runs them.  Two full-size layers at
+T = 8; the graph replay must give the same bytes as eager calls, and sampled
+tokens of every layer match the oracle."""
+import numpy as np
+import pytest
+
+from tests.gpu_helpers import DeviceLayer, assert_close, mq_lib, tokens
+from workloads import get_config
+from dataclasses import replace
+
+pytestmark = pytest.mark.gpu
+
+
+def test_stack_graph_replay_matches_eager_and_oracle(orc):
+    import torch
+    mq = mq_lib()
+    base = get_config("v3_stack20")
+    T, L = 8, 2
+    spec = replace(base, tokens=T)
+    layers = [DeviceLayer(spec, l) for l in range(L)]
+    xs = [tokens(spec, 40 + l, T) for l in range(L)]
+    xbuf = torch.from_numpy(np.stack(xs).view(np.int16)).cuda()
+    outs = torch.full((L, T, spec.hidden), float("nan"), device="cuda")
+    idxs = torch.full((L, T, spec.top_k), -1, dtype=torch.int32, device="cuda")
+    wts = torch.zeros((L, T, spec.top_k), dtype=torch.float32, device="cuda")
+    wsb = mq.moe_quant_workspace_size(layers[0].cfg, T)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")   # shared by the layers (stream-ordered)
+
+    def calls():
+        for l, lay in enumerate(layers):
+            mq.moe_quant_forward(lay.cfg, T, xbuf[l], lay.router_w, lay.bias, lay.table, lay.fmts, outs[l],
+                                 idxs[l], wts[l], ws, wsb)
+
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        calls()
+    torch.cuda.synchronize()
+    eager_out, eager_idx = outs.cpu().numpy().copy(), idxs.cpu().numpy().copy()
+    outs.fill_(float("nan"))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        calls()
+    graph.replay()
+    torch.cuda.synchronize()
+    g_out, g_idx = outs.cpu().numpy(), idxs.cpu().numpy()
+    np.testing.assert_array_equal(g_idx, eager_idx)
+    np.testing.assert_array_equal(g_out.view(np.uint32), eager_out.view(np.uint32))   # deterministic kernels
+    for l, lay in enumerate(layers):
+        for t in (0, T - 1):
+            ry, ridx, _ = lay.oracle_forward(orc, xs[l][t:t + 1], idx_hint=g_idx[l, t])
+            np.testing.assert_array_equal(g_idx[l, t:t + 1], ridx)
+            assert_close(g_out[l, t:t + 1], ry)
