@@ -44,6 +44,7 @@ struct PrefillArgs {
     const __half* x16;       // [T][H] tokens in fp16
     __half* h16;             // [A][I] SwiGLU outputs (routing weight folded in)
     float* pdn;              // [A][H]
+    uint32_t* next;          // unit counters (gate/up, down), zeroed per call
     uint32_t* err;
 };
 
@@ -283,6 +284,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
     __shared__ __align__(8) uint64_t bars[kPSlots];
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
+    __shared__ int s_unit;
     const Dims& d = A.d;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n_mt = (kDown ? d.H : d.I) / kMT;
@@ -331,7 +333,13 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
     bool failed = false;
     int cursor = 0;
 
-    for (int u = blockIdx.x; u < n_units && !failed; u += gridDim.x) {
+    // units are claimed from a global counter (their cost varies with the
+    // number of tokens of the expert, up to 16x between full and small tiles)
+    for (;;) {
+        if (tid == 0) s_unit = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+        __syncthreads();
+        const int u = s_unit;
+        if (u >= n_units || failed) break;
         while (cursor + 1 < n_slots && sl.pre[cursor + 1] <= u) ++cursor;
         const int p = cursor, local = u - sl.pre[p];
         const int tt = local / n_mt, mt = local - tt * n_mt;
@@ -384,10 +392,32 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         };
         gather(0, gchunk % kPSlots);
         asm volatile("cp.async.commit_group;" ::: "memory");
+        // L2 prefetch duty: lanes 0..7 of warps 0..3 (the unit's four 32-row
+        // tiles): lane = plane (0..3) of tensor lane / 4; a superblock's records
+        // of a tile are one contiguous range per plane
+        const uint8_t* pf_src = nullptr;
+        uint32_t pf_bytes = 0;
+        int pf_nsb = 0;   // whole superblocks of records a row has (Q8_0: groups of 8 blocks)
+        if (hf == 0 && lane < 8 && (!kDown || lane < 4)) {
+            const int pl = lane & 3, fmt = lane < 4 ? f0 : f1;
+            const PlaneBytes pb = plane_bytes(fmt);
+            if (pl < pb.n) {
+                const TensorLayout& Lx = lane < 4 ? L0 : L1;
+                pf_src = rec_ptr((lane < 4 ? b0 : b1) + Lx.plane[pl], Lx, pb.b[pl], (int64_t)mt * kMT + 32 * warp, 0);
+                pf_bytes = (uint32_t)(32 * pb.b[pl] * (fmt == kQ80 ? 8 : 1));
+                pf_nsb = (int)(fmt == kQ80 ? Lx.blocks_per_row / 8 : Lx.blocks_per_row);
+                if ((reinterpret_cast<uintptr_t>(pf_src) & 15u) != 0 || (pf_bytes & 15u) != 0) pf_src = nullptr;
+            }
+        }
         Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
         load_chunk(f0, RP0, 0, hf, P0);
         if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
         for (int c = 0; c < nC; ++c) {
+            // pull the records of this warp's 32-row tile for the next superblock
+            // into L2, so the per-thread loads of the coming chunks hit L2
+            if ((c & 3) == 0 && pf_src != nullptr && (c >> 2) + 1 < pf_nsb)
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                             ::"l"(pf_src + (int64_t)((c >> 2) + 1) * pf_bytes), "r"(pf_bytes) : "memory");
             Packed N0, N1;             // the next chunk's, loaded while this one is decoded
             if (c + 1 < nC) {
                 load_chunk(f0, RP0, c + 1, hf, N0);
@@ -498,6 +528,7 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     A.d = d;
     A.offsets = w.offsets; A.perm = w.perm; A.active = w.active; A.wts = w.wts;
     A.x16 = w.x16; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
+    A.next = w.counters;
     prof_begin("gateup_tc", s);
     cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(kPThreads), smem, s, tab, A);
     prof_end(s);
