@@ -257,7 +257,7 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
             if (it.shared) { t = q; a = d.T * d.K + q; }
             else {
                 const int idx = sc.first[p] + q;
-                a = idx < kMaxCachedAssign ? s_perm[idx] : A.perm[idx];
+                a = idx < kMaxCachedAssign ? s_perm[idx] : __ldcg(A.perm + idx);
                 t = a / d.K;
             }
         }
@@ -578,7 +578,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         sc.fmt[0][0] = tab.fmt[d.E][0]; sc.fmt[0][1] = tab.fmt[d.E][1];
     }
     __syncthreads();
-    pdl_launch();
+    // The down kernel lets its successor (the combine) launch right away; the
+    // gate/up kernel only once it holds the routing result (below), so that
+    // the down kernel, launched after that, may read the routing result
+    // before its own wait.
+    if (kDown) pdl_launch();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
 
@@ -600,12 +604,20 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // cached permutation
         int n_slots = n_sh_items > 0 ? 1 : 0, n_items = n_sh_items;
         bool routed = false;
+        // gate/up: the routing kernel is the predecessor, wait for it.  down:
+        // the routing result is two kernels back (complete before the gate/up
+        // kernel let this grid launch); only h, from the gate/up kernel, needs
+        // the wait, taken before the first copy of h (deps below).
+        bool deps = !kDown;
         auto wait_routing = [&]() {
-            pdl_wait();
-            n_slots = A.plan->n_slots;
+            if (!kDown) pdl_wait();
+            // read through L2 (ld.global.cg): the down kernel reads before its
+            // wait, and an SM's L1 may still hold lines of an earlier call
+            n_slots = __ldcg(&A.plan->n_slots);
             for (int i = lane; i < kMaxExperts + 2; i += 32) {
-                const int pre = kDown ? A.plan->pre_dn[i] : A.plan->pre_gu[i];
-                const int e = A.plan->slot_e[i], first = A.plan->slot_first[i], ntot = A.plan->slot_ntot[i];
+                const int pre = __ldcg(kDown ? &A.plan->pre_dn[i] : &A.plan->pre_gu[i]);
+                const int e = __ldcg(&A.plan->slot_e[i]), first = __ldcg(&A.plan->slot_first[i]);
+                const int ntot = __ldcg(&A.plan->slot_ntot[i]);
                 if (i <= n_slots) sc.pre[i] = pre;
                 if (i < n_slots) {
                     sc.e[i] = e;
@@ -618,10 +630,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 }
             }
             const int n_routed = min(d.T * d.K, kMaxCachedAssign);
-            for (int i = lane; i < n_routed; i += 32) s_perm[i] = A.perm[i];
+            for (int i = lane; i < n_routed; i += 32) s_perm[i] = __ldcg(A.perm + i);
             __syncwarp();
             n_items = sc.pre[n_slots];
             routed = true;
+            if (!kDown) pdl_launch();
         };
         if (n_sh_items == 0) wait_routing();
         // items are handed out by a global counter (zeroed per call), in slot
@@ -704,7 +717,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     mbar_arrive_tx(full, total);
                 }
                 __syncwarp();
-                if (bytes) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
+                // weight planes (lanes 0..3) first; the down kernel's first copy
+                // of h waits for the gate/up kernel, while its weights stream
+                if (bytes && lane < 4) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
+                if (!deps) { pdl_wait(); deps = true; }
+                if (bytes && lane >= 4) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
                 ++p_q;
             }
             if (failed) { if (lane == 0) { atomicOr(A.err, kErrEmpty); s_fail = 1; } break; }

@@ -39,21 +39,24 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
                                                              __half* __restrict__ xq, float* __restrict__ xs,
                                                              __half* __restrict__ x16,
                                                              uint32_t* __restrict__ zero_words, int n_zero) {
-    pdl_wait();
-    pdl_launch();
-    // per-call words that must start at zero (work counters, error word)
-    if (blockIdx.x == 0 && blockIdx.y == 0)
-        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
     __shared__ float part[32][kTok];
     const int e = blockIdx.x, t0 = blockIdx.y * kTok;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
     const int c0 = seg * 8, nc = min(8, nchunk - c0);
     const float* wrow = W + (size_t)e * H;
+    // The router weights are an input no kernel of this library writes, so
+    // their loads go out before the wait for the previous kernel (which may
+    // be the previous layer's combine, writing this call's x).
     float4 wv[8];
 #pragma unroll
     for (int c = 0; c < 8; ++c)
         if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(wrow + (c0 + c) * 128 + 4 * lane));
+    pdl_wait();
+    pdl_launch();
+    // per-call words that must start at zero (work counters, error word)
+    if (blockIdx.x == 0 && blockIdx.y == 0)
+        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
     float acc[kTok];
 #pragma unroll
     for (int j = 0; j < kTok; ++j) acc[j] = 0.0f;
@@ -267,17 +270,23 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
                                                                const float* __restrict__ z,
                                                                const float* __restrict__ bias,
                                                                float* __restrict__ wts) {
-    pdl_wait();
-    pdl_launch();
     const int n = d.T * d.K, E = d.E;
     __shared__ int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
     __shared__ int32_t s_off[kMaxExperts + 1];
     __shared__ int32_t s_act[kMaxExperts + 1];
     __shared__ float g_sh[kPermWarps][kMaxGroups];
+    __shared__ float s_bias[kMaxExperts];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // the selection bias is an input no kernel of this library writes: staged
+    // before the wait for the logits kernel
+    if (z != nullptr)
+        for (int i = threadIdx.x; i < E; i += kPermThreads) s_bias[i] = bias ? bias[i] : 0.0f;
+    __syncthreads();
+    pdl_wait();
+    pdl_launch();
     if (z != nullptr) {
         for (int t = warp; t < d.T; t += kPermWarps)
-            route_token(z, bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
+            route_token(z, s_bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
                         g_sh[warp], idx, wts);
         __syncthreads();
     }
