@@ -171,6 +171,60 @@ __device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, in
     }
 }
 
+// One superblock's packed fields of one weight row for this thread's half of
+// each of its four 64-wide chunks (Q2_K, Q3_K, Q4_K): codes, scales and d /
+// dmin are read once per superblock, with wide loads, one superblock ahead.
+struct SBlk {
+    uint4 cw[4];      // Q2_K / Q3_K low bits: words 4i..4i+3 for i = 2 hf, 2 hf + 1; Q4_K: the 4 chunks' 16 bytes
+    uint2 hw[2];      // Q3_K high bits: words 2i, 2i+1
+    uint32_t sc[4];   // scale record
+    uint32_t dd;      // d | dmin << 16
+};
+__device__ __forceinline__ uint2 ldg64u(const uint8_t* p) { return __ldg(reinterpret_cast<const uint2*>(p)); }
+__device__ __forceinline__ void load_sblk(int fmt, const RowPtrs& RP, int sb, int hf, SBlk& B) {
+    const int64_t s = sb;
+    B.dd = ldg16u(RP.row[0] + s * (32 * 2));
+    if (fmt == kQ4K) {
+        B.dd |= ldg16u(RP.row[1] + s * (32 * 2)) << 16;
+        const uint8_t* sp = RP.row[2] + s * (32 * 12);
+        B.sc[0] = ldg32(sp); B.sc[1] = ldg32(sp + 4); B.sc[2] = ldg32(sp + 8);
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            const int j = 2 * cc + hf;
+            B.cw[cc] = ldg128(RP.row[3] + s * (32 * 128) + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
+        }
+    } else if (fmt == kQ2K) {
+        B.dd |= ldg16u(RP.row[1] + s * (32 * 2)) << 16;
+        const uint4 sv = ldg128(RP.row[2] + s * (32 * 16));
+        B.sc[0] = sv.x; B.sc[1] = sv.y; B.sc[2] = sv.z; B.sc[3] = sv.w;
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) B.cw[ii] = ldg128(RP.row[3] + s * (32 * 64) + 16 * (2 * hf + ii));
+    } else {   // Q3_K
+        const uint8_t* sp = RP.row[1] + s * (32 * 12);
+        B.sc[0] = ldg32(sp); B.sc[1] = ldg32(sp + 4); B.sc[2] = ldg32(sp + 8);
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            B.cw[ii] = ldg128(RP.row[2] + s * (32 * 64) + 16 * (2 * hf + ii));
+            B.hw[ii] = ldg64u(RP.row[3] + s * (32 * 32) + 8 * (2 * hf + ii));
+        }
+    }
+}
+// the chunk's fields (chunk cc of the superblock) in the per-chunk form dequant_store reads
+__device__ __forceinline__ void make_packed(int fmt, const SBlk& B, int cc, Packed& P) {
+    P.dd = B.dd;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) P.sc[i] = B.sc[i];
+    if (fmt == kQ4K) {
+        P.w[0] = B.cw[cc].x; P.w[1] = B.cw[cc].y; P.w[2] = B.cw[cc].z; P.w[3] = B.cw[cc].w;
+    } else {
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            P.w[ii] = sub4(B.cw[ii], cc);
+            P.w[4 + ii] = (cc >> 1) ? B.hw[ii].y : B.hw[ii].x;
+        }
+    }
+}
+
 __device__ __forceinline__ float half_lo(uint32_t v) { return __half2float(__ushort_as_half((unsigned short)(v & 0xffffu))); }
 __device__ __forceinline__ float half_hi(uint32_t v) { return __half2float(__ushort_as_half((unsigned short)(v >> 16))); }
 // byte i (0..15) of a 4-word record, with a runtime i kept in registers
@@ -409,20 +463,9 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
                 if ((reinterpret_cast<uintptr_t>(pf_src) & 15u) != 0 || (pf_bytes & 15u) != 0) pf_src = nullptr;
             }
         }
-        Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
-        load_chunk(f0, RP0, 0, hf, P0);
-        if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
-        for (int c = 0; c < nC; ++c) {
-            // pull the records of this warp's 32-row tile for the next superblock
-            // into L2, so the per-thread loads of the coming chunks hit L2
-            if ((c & 3) == 0 && pf_src != nullptr && (c >> 2) + 1 < pf_nsb)
-                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
-                             ::"l"(pf_src + (int64_t)((c >> 2) + 1) * pf_bytes), "r"(pf_bytes) : "memory");
-            Packed N0, N1;             // the next chunk's, loaded while this one is decoded
-            if (c + 1 < nC) {
-                load_chunk(f0, RP0, c + 1, hf, N0);
-                if (!kDown) load_chunk(f1, RP1, c + 1, hf, N1);
-            }
+        // one 64-wide chunk: gather the next chunk's rows, decode this one's
+        // weights, then thread 0 issues its MMAs
+        auto chunk_body = [&](int c, const Packed& Q0, const Packed& Q1) -> bool {
             const int g = gchunk + c, s = g % kPSlots;
             bool bad = false;
             if (c + 1 < nC) {
@@ -433,13 +476,11 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
             const uint32_t sbase = ring + s * kSlotBytes;
-            dequant_store(f0, P0, c, hf, sbase + rr * 16);
-            if (!kDown) dequant_store(f1, P1, c, hf, sbase + kABytes + rr * 16);
-            P0 = N0;
-            if (!kDown) P1 = N1;
+            dequant_store(f0, Q0, c, hf, sbase + rr * 16);
+            if (!kDown) dequant_store(f1, Q1, c, hf, sbase + kABytes + rr * 16);
             asm volatile("cp.async.wait_group 1;" ::: "memory");
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            if (__syncthreads_or(bad)) { failed = true; break; }
+            if (__syncthreads_or(bad)) return false;
             if (tid == 0) {
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t idesc = idesc_f16(kMT, Npad);
@@ -455,6 +496,58 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
                              ::"r"(bar0 + 8 * s) : "memory");
             }
             last_committed = g;
+            return true;
+        };
+        if (f0 != kQ80 && (kDown || f1 != kQ80)) {
+            // superblock-granular fields (Q2_K, Q3_K, Q4_K), one superblock ahead
+            const int nS = (nC + 3) / 4;
+            SBlk Sa0, Sa1, Sb0, Sb1;
+            load_sblk(f0, RP0, 0, hf, Sa0);
+            if (!kDown) load_sblk(f1, RP1, 0, hf, Sa1);
+            auto sblock = [&](int sb, const SBlk& C0, const SBlk& C1, SBlk& N0, SBlk& N1) -> bool {
+                if (sb + 1 < nS) {
+                    load_sblk(f0, RP0, sb + 1, hf, N0);
+                    if (!kDown) load_sblk(f1, RP1, sb + 1, hf, N1);
+                }
+                // the records of the superblock after that into L2
+                if (pf_src != nullptr && sb + 2 < pf_nsb)
+                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                                 ::"l"(pf_src + (int64_t)(sb + 2) * pf_bytes), "r"(pf_bytes) : "memory");
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) {
+                    const int c = 4 * sb + cc;
+                    if (c >= nC) break;
+                    Packed Q0, Q1;
+                    make_packed(f0, C0, cc, Q0);
+                    if (!kDown) make_packed(f1, C1, cc, Q1);
+                    if (!chunk_body(c, Q0, Q1)) return false;
+                }
+                return true;
+            };
+            for (int sb = 0; sb < nS; sb += 2) {
+                if (!sblock(sb, Sa0, Sa1, Sb0, Sb1)) { failed = true; break; }
+                if (sb + 1 < nS && !sblock(sb + 1, Sb0, Sb1, Sa0, Sa1)) { failed = true; break; }
+            }
+        } else {
+            // Q8_0 in the unit: per-chunk fields (blocks of 32), one chunk ahead
+            Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
+            load_chunk(f0, RP0, 0, hf, P0);
+            if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
+            for (int c = 0; c < nC; ++c) {
+                // pull the records of this warp's 32-row tile for the next superblock
+                // into L2, so the per-thread loads of the coming chunks hit L2
+                if ((c & 3) == 0 && pf_src != nullptr && (c >> 2) + 1 < pf_nsb)
+                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                                 ::"l"(pf_src + (int64_t)((c >> 2) + 1) * pf_bytes), "r"(pf_bytes) : "memory");
+                Packed N0, N1;             // the next chunk's, loaded while this one is decoded
+                if (c + 1 < nC) {
+                    load_chunk(f0, RP0, c + 1, hf, N0);
+                    if (!kDown) load_chunk(f1, RP1, c + 1, hf, N1);
+                }
+                if (!chunk_body(c, P0, P1)) { failed = true; break; }
+                P0 = N0;
+                if (!kDown) P1 = N1;
+            }
         }
         asm volatile("cp.async.wait_group 0;" ::: "memory");
         if (failed) break;
