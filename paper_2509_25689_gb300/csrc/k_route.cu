@@ -123,6 +123,100 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
 }
 
 // ---------------------------------------------------------------------------
+// logits for larger batches (no activation preparation): grid
+// (ceil(E / kEB), ceil(T / kTokT)); a CTA keeps its 4 tokens' segments in
+// registers as fp32 and runs through 16 experts, so the tokens are read and
+// converted once per 16 experts instead of once per expert.  Same canonical
+// order as router_logits_kernel (lane chains over the segment's chunks, xor
+// butterfly, segments left to right), so z is bit-identical.
+// ---------------------------------------------------------------------------
+constexpr int kEB = 16;
+constexpr int kTokT = 4;
+
+__global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t* __restrict__ x,
+                                                                  const float* __restrict__ W, int H, int T,
+                                                                  int E, float* __restrict__ z,
+                                                                  __half* __restrict__ x16,
+                                                                  uint32_t* __restrict__ zero_words, int n_zero) {
+    __shared__ float part[32][kTokT];
+    const int e0 = blockIdx.x * kEB, t0 = blockIdx.y * kTokT;
+    const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
+    const int c0 = seg * 8, nc = min(8, nchunk - c0);
+    // the first expert's weights go out before the wait (an input no kernel of this library writes)
+    float4 wv[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        if (c < nc && e0 < E) wv[c] = __ldg(reinterpret_cast<const float4*>(W + (size_t)e0 * H + (c0 + c) * 128 + 4 * lane));
+    pdl_wait();
+    pdl_launch();
+    if (blockIdx.x == 0 && blockIdx.y == 0)
+        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
+    float4 xf[kTokT][8];   // the tokens' segment elements 4 lane + 0..3 of each chunk, as fp32
+#pragma unroll
+    for (int j = 0; j < kTokT; ++j)
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            uint2 v = make_uint2(0u, 0u);
+            if (c < nc && t0 + j < T)
+                v = __ldg(reinterpret_cast<const uint2*>(x + (size_t)(t0 + j) * H + (c0 + c) * 128 + 4 * lane));
+            xf[j][c] = make_float4(bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y));
+            if (x16 != nullptr && blockIdx.x == 0 && c < nc && t0 + j < T) {
+                // fp16 copy of the tokens for the prefill GEMM
+                const __half2 h0 = __floats2half2_rn(xf[j][c].x, xf[j][c].y);
+                const __half2 h1 = __floats2half2_rn(xf[j][c].z, xf[j][c].w);
+                uint2 hv;
+                hv.x = *reinterpret_cast<const uint32_t*>(&h0);
+                hv.y = *reinterpret_cast<const uint32_t*>(&h1);
+                *reinterpret_cast<uint2*>(x16 + (size_t)(t0 + j) * H + (c0 + c) * 128 + 4 * lane) = hv;
+            }
+        }
+    for (int el = 0; el < kEB; ++el) {
+        const int e = e0 + el;
+        if (e >= E) break;
+        float acc[kTokT];
+#pragma unroll
+        for (int j = 0; j < kTokT; ++j) {
+            acc[j] = 0.0f;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                if (c < nc) {
+                    acc[j] = __fmaf_rn(xf[j][c].x, wv[c].x, acc[j]);
+                    acc[j] = __fmaf_rn(xf[j][c].y, wv[c].y, acc[j]);
+                    acc[j] = __fmaf_rn(xf[j][c].z, wv[c].z, acc[j]);
+                    acc[j] = __fmaf_rn(xf[j][c].w, wv[c].w, acc[j]);
+                }
+            }
+        }
+        // the next expert's weights, loaded while this one's sums are reduced
+        if (e + 1 < E && el + 1 < kEB) {
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(W + (size_t)(e + 1) * H + (c0 + c) * 128 + 4 * lane));
+        }
+#pragma unroll
+        for (int j = 0; j < kTokT; ++j) {
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) acc[j] = __fadd_rn(acc[j], __shfl_xor_sync(kFull, acc[j], off));
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int j = 0; j < kTokT; ++j) part[seg][j] = acc[j];
+        }
+        __syncthreads();
+        if (threadIdx.x < kTokT) {
+            const int t = t0 + threadIdx.x;
+            if (t < T) {
+                float r = part[0][threadIdx.x];
+                for (int s2 = 1; s2 < nseg; ++s2) r = __fadd_rn(r, part[s2][threadIdx.x]);
+                z[(size_t)t * E + e] = r;
+            }
+        }
+        __syncthreads();
+    }
+}
+
+// ---------------------------------------------------------------------------
 // scores + group-limited top-k: one warp per token
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float canonical_sigmoid(float z) {
@@ -428,10 +522,18 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
                                  __half* x16, uint32_t* zero_words, int n_zero, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
-    dim3 grid(d.E, (d.T + kTok - 1) / kTok);
     prof_begin("router_logits", s);
-    const cudaError_t e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq,
-                                     xs, x16, zero_words, n_zero);
+    cudaError_t e;
+    if (xq == nullptr && d.T >= 16 && nseg <= 8) {
+        // larger batches without activation preparation: tokens reused across 16 experts
+        dim3 grid((d.E + kEB - 1) / kEB, (d.T + kTokT - 1) / kTokT);
+        e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16,
+                       zero_words, n_zero);
+    } else {
+        dim3 grid(d.E, (d.T + kTok - 1) / kTok);
+        e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq, xs, x16,
+                       zero_words, n_zero);
+    }
     prof_end(s);
     return e;
 }
