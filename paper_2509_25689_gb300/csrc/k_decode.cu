@@ -924,8 +924,10 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
 
 cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s) {
     prof_begin("combine", s);
-    const cudaError_t err = launch_pdl(combine_kernel, dim3((d.H + 255) / 256, d.T < 8 ? d.T : 8), dim3(256), 0, s,
-                                       d, pdn, out);
+    // one CTA row per token (up to 65535; the kernel strides over the rest),
+    // so large batches stream the partial outputs at full bandwidth
+    const cudaError_t err = launch_pdl(combine_kernel, dim3((d.H + 255) / 256, d.T < 65535 ? d.T : 65535), dim3(256),
+                                       0, s, d, pdn, out);
     prof_end(s);
     return err;
 }
