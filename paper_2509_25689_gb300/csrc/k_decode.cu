@@ -243,9 +243,10 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
     slot = p;
     const int local = id - sc.pre[p];
     const Dims& d = A.d;
-    const int nrb = (kDown ? d.H : d.I) / 32;
+    // gate/up items: one 32-row block of gate and up; down items: two 32-row blocks
+    const int nrb = kDown ? d.H / 64 : d.I / 32;
     it.tg = local / nrb;
-    it.rb = local - it.tg * nrb;
+    it.rb = (local - it.tg * nrb) * (kDown ? 2 : 1);
     it.e = sc.e[p];
     it.shared = p < d.has_shared;
     it.ntok = min(kDecodeTok, sc.ntot[p] - it.tg * kDecodeTok);
@@ -265,7 +266,7 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
         it.vec[j] = kDown ? a : t;
     }
     it.nst0 = geo[sc.fmt[p][0] - 1][it.ntok - 1].nst;
-    it.nst = kDown ? it.nst0 : it.nst0 + geo[sc.fmt[p][1] - 1][it.ntok - 1].nst;
+    it.nst = kDown ? 2 * it.nst0 : it.nst0 + geo[sc.fmt[p][1] - 1][it.ntok - 1].nst;
 }
 
 // ---- consumer math: one warp = the 32 rows of the stage (two 16-row MMA
@@ -672,15 +673,16 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     ++p_q;
                     break;
                 }
-                if (pj == 0 || (!kDown && pj == P.nst0)) {
-                    tensor = kDown ? 2 : (pj == 0 ? 0 : 1);
+                if (pj == 0 || pj == P.nst0) {
+                    // phases: gate then up (gate/up items); rows rb then rb + 1 (down items, tensor 2 / 3)
+                    tensor = kDown ? (pj == 0 ? 2 : 3) : (pj == 0 ? 0 : 1);
                     phase_j = pj;
                     fmt = sc.fmt[pslot][tensor == 1 ? 1 : 0];
                     G = &geo[fmt - 1][P.ntok - 1];
                     const uint8_t* tbase = tensor == 1 ? sc.ptr_up[pslot] : sc.ptr[pslot];
                     c_src = nullptr; c_stride = 0; c_dst = 0;
                     if (lane < G->npl) {
-                        c_src = tbase + G->pl[lane] + (int64_t)P.rb * G->rbstr[lane];
+                        c_src = tbase + G->pl[lane] + (int64_t)(P.rb + (tensor == 3 ? 1 : 0)) * G->rbstr[lane];
                         c_stride = G->cstr[lane];
                         c_dst = G->woff[lane];
                     }
@@ -751,8 +753,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             const uint32_t stage = ring + slot * kStageBytes;
             const int fmt = H.fmt, ks = H.ks, ntok = H.ntok;
             const Geo& GS = geo[fmt - 1][ntok - 1];
-            if (!kDown && H.tensor == 1 && H.s0 == 0) {
-                // first stage of the up tensor: the gate sums are complete
+            if ((H.tensor == 1 || H.tensor == 3) && H.s0 == 0) {
+                // first stage of the second phase: the first phase's sums are complete
 #pragma unroll
                 for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
@@ -794,16 +796,17 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             if (lane == 0) mbar_arrive(bar0 + 8 * (kNST + slot));
             if (!item_end) continue;
 
-            // ---- item done: the streamed tensor's sums go to acc[1] (up) or acc[0]
+            // ---- item done: phase 0 (gate, or rows rb) in acc[0], phase 1 (up, or
+            // rows rb + 1) still streaming in cur
             const int g = lane >> 2, t4 = lane & 3;
             const int buf = kRedBufs == 2 ? (n_done & 1) : 0;
 #pragma unroll
-            for (int u = 0; u < (kDown ? 1 : 2); ++u)
+            for (int u = 0; u < 2; ++u)
 #pragma unroll
                 for (int tk = 0; tk < MT; ++tk)
 #pragma unroll
                     for (int i = 0; i < 2 * kNT; ++i) {
-                        float v = (u == (kDown ? 0 : 1)) ? acc[u][tk][i] + cur[tk][i] : acc[u][tk][i];
+                        float v = u == 1 ? acc[u][tk][i] + cur[tk][i] : acc[u][tk][i];
                         v += __shfl_xor_sync(kFull, v, 1);
                         v += __shfl_xor_sync(kFull, v, 2);
                         if (t4 == 0) {
@@ -827,10 +830,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 #pragma unroll
                 for (int c2 = 0; c2 < kConsumers; ++c2) {
                     v0 += red[buf][c2][0][tk][lane];
-                    if (!kDown) v1 += red[buf][c2][1][tk][lane];
+                    v1 += red[buf][c2][1][tk][lane];
                 }
                 if (kDown) {
                     A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
+                    A.pdn[(size_t)a * d.H + 32 * (e_rb + 1) + lane] = v1;
                 } else {
                     // SwiGLU (routing weight folded in), then prepare h for the down projection
                     if (!e_shared) pdl_wait();   // routing weights come from the routing kernel

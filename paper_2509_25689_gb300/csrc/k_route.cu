@@ -487,7 +487,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
             }
             const int ntg = (ntok + kDecodeTok - 1) / kDecodeTok;
             cg[q] = (d.I / 32) * ntg;     // gate/up items: 32 rows x both tensors x full K
-            cd[q] = (d.H / 32) * ntg;     // down items: 32 rows x full K
+            cd[q] = (d.H / 64) * ntg;     // down items: 64 rows (two 32-row blocks) x full K
             sg += cg[q]; sd += cd[q]; tgs += ntg; tgmax = max(tgmax, ntg);
         }
         int ig = sg, id = sd;
