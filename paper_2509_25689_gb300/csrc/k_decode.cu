@@ -161,18 +161,6 @@ constexpr uint32_t kErrFull = 1u, kErrEmpty = 2u;
 // named barrier 1: the consumer warps only
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers * 32) : "memory"); }
 
-struct DecodeArgs {
-    Dims d;
-    int nsbx, nsbi;          // superblocks along hidden / inter
-    const __half* xq; const float* xs;   // prepared tokens
-    __half* hq; float* hs;               // prepared SwiGLU outputs (per assignment)
-    const int32_t* offsets; const int32_t* perm; const int32_t* active; const float* wts;
-    const Plan* plan;
-    float* pdn;              // [A][H]
-    uint32_t* next;          // [2] item counters
-    uint32_t* err;
-    float* out;
-};
 
 // stage header written by the producer (one per ring slot); the stage's
 // byte layout is geo[fmt - 1][ntok - 1]
@@ -186,7 +174,7 @@ struct __align__(16) Hdr {
 // token pieces in a stage: the family fragments, the Q3_K high-bit fragments
 // and the per-superblock statistics, each for the stage's ks superblocks
 struct TokLay { int x, x1, s, stride; };
-__device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
+__host__ __device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
     TokLay t;
     int at = 0;
     t.x = at; at += ks * 512;
@@ -196,7 +184,7 @@ __device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
     return t;
 }
 
-__device__ __forceinline__ int weight_stage_bytes(int fmt, int ks) {
+__host__ __device__ __forceinline__ int weight_stage_bytes(int fmt, int ks) {
     const PlaneBytes pb = plane_bytes(fmt);
     const int nblk = fmt == kQ80 ? 8 * ks : ks;
     int at = 0;
@@ -204,7 +192,7 @@ __device__ __forceinline__ int weight_stage_bytes(int fmt, int ks) {
     return at;
 }
 // superblocks per stage for a format and token count (fits kStageBytes)
-__device__ __forceinline__ int stage_sb(int fmt, int ntok) {
+__host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok) {
     int ks = fmt == kQ80 ? kStageSb / 2 : kStageSb;
     while (ks > 1 && weight_stage_bytes(fmt, ks) + ntok * tok_lay(fmt, ks).stride > kStageBytes) --ks;
     return ks;
@@ -227,6 +215,42 @@ struct Geo {
     int per, nst, npl;   // superblocks per stage, stages per tensor, planes
     int woff[4], cstr[4];// plane regions in the stage, bytes per superblock
     int tok0, tstride, tx, tx1, ts;
+};
+
+// Stage geometry of (format, tokens per item) for the gate/up (down = false)
+// or down kernel; the host computes it once per launch.
+__host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int fmt, int ntok) {
+    const int nsb = down ? (d.I + 255) / 256 : (d.H + 255) / 256;
+    const TensorLayout L = tensor_layout(fmt, down ? d.H : d.I, down ? d.I : d.H);
+    const PlaneBytes pb = plane_bytes(fmt);
+    const int bmul = fmt == kQ80 ? 8 : 1;
+    G.per = stage_sb(fmt, ntok);
+    G.nst = (nsb + G.per - 1) / G.per;
+    G.npl = pb.n;
+    int at = 0;
+    for (int pl = 0; pl < 4; ++pl) {
+        G.woff[pl] = at;
+        G.cstr[pl] = pl < pb.n ? 32 * bmul * pb.b[pl] : 0;
+        G.pl[pl] = L.plane[pl];
+        G.rbstr[pl] = pl < pb.n ? L.blocks_per_row * 32 * pb.b[pl] : 0;
+        if (pl < pb.n) at += (32 * bmul * G.per * pb.b[pl] + 127) & ~127;
+    }
+    const TokLay tl = tok_lay(fmt, G.per);
+    G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.tx1 = tl.x1; G.ts = tl.s;
+}
+
+struct DecodeArgs {
+    Dims d;
+    int nsbx, nsbi;          // superblocks along hidden / inter
+    const __half* xq; const float* xs;   // prepared tokens
+    __half* hq; float* hs;               // prepared SwiGLU outputs (per assignment)
+    const int32_t* offsets; const int32_t* perm; const int32_t* active; const float* wts;
+    const Plan* plan;
+    float* pdn;              // [A][H]
+    uint32_t* next;          // [2] item counters
+    uint32_t* err;
+    float* out;
+    Geo geo[4][kDecodeTok];  // stage geometry per (format, tokens), computed on the host
 };
 
 struct ItemDesc {            // decoded item (producer side)
@@ -289,7 +313,8 @@ __device__ __forceinline__ void ld_frag8(uint32_t a, uint32_t (&X)[8]) {
 }
 
 // A tile's MMA sums: [tile][sub-block group][pair parity][D fragment]
-// (Q2_K / Q3_K use both groups, Q4_K / Q8_0 only group 0).
+// (Q2_K / Q3_K: the two sub-block groups; Q4_K / Q8_0: four accumulators
+// of the same sums, added in the epilogue).
 template <int NT> struct TileAcc { float DD[NT][2][2][4]; };
 
 // Loads one (superblock, token) tile of the warp's rows and issues its MMAs
@@ -311,6 +336,9 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
 #pragma unroll
     for (int i = 0; i < NT * 16; ++i) (&T.DD[0][0][0][0])[i] = 0.0f;
 
+    // Issue order: every MMA of a step goes to a different accumulator and an
+    // accumulator is reused only 8 MMAs later, so the in-order warp does not
+    // stall on the MMA latency inside a tile (all B fragments are loaded first).
     if (FMT == kQ2K || FMT == kQ3K) {
         const uint32_t cp = FMT == kQ2K ? w3 : w2;   // 2-bit code plane
         uint4 c[NR];
@@ -320,44 +348,57 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
             c[i] = lds128(st + cp + rec_of(i) * 64 + 16 * t);
             if (FMT == kQ3K) hv[i] = lds64(st + w3 + rec_of(i) * 32 + 8 * t);
         }
+        uint32_t XA[2][8], XB[2][8];
 #pragma unroll
         for (int gm = 0; gm < 2; ++gm) {
-            uint32_t XA[8], XB[8];
-            ld_frag8(own0 ? xb + 32 * (8 * gm + t) : zaddr, XA);
-            ld_frag8(own1 ? xb + 32 * (8 * gm + 4 + t) : zaddr, XB);
-            uint32_t qa[NR], qb[NR], sa[NR], sbb[NR];   // per row: sub-blocks t (a0/a1) and t+4 (a2/a3)
+            ld_frag8(own0 ? xb + 32 * (8 * gm + t) : zaddr, XA[gm]);
+            ld_frag8(own1 ? xb + 32 * (8 * gm + 4 + t) : zaddr, XB[gm]);
+        }
+        uint32_t qa[2][NR], qb[2][NR], sa[2][NR], sbb[2][NR];   // per row: sub-blocks t (a0/a1) and t+4 (a2/a3)
+#pragma unroll
+        for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
             for (int i = 0; i < NR; ++i) {
-                qa[i] = sub4(c[i], 2 * gm); qb[i] = sub4(c[i], 2 * gm + 1);
-                sa[i] = qa[i] >> 10; sbb[i] = qb[i] >> 10;
+                qa[gm][i] = sub4(c[i], 2 * gm); qb[gm][i] = sub4(c[i], 2 * gm + 1);
+                sa[gm][i] = qa[gm][i] >> 10; sbb[gm][i] = qb[gm][i] >> 10;
             }
 #pragma unroll
-            for (int m = 0; m < 8; ++m) {
-                const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
-                const bool sh = m > 4;
+        for (int m = 0; m < 8; ++m) {
+            const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
+            const bool sh = m > 4;
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
                 for (int tl = 0; tl < NT; ++tl)
-                    mma16816(T.DD[tl][gm][m & 1], (sh ? sa[2 * tl] : qa[2 * tl]) & mk,
-                             (sh ? sa[2 * tl + 1] : qa[2 * tl + 1]) & mk, (sh ? sbb[2 * tl] : qb[2 * tl]) & mk,
-                             (sh ? sbb[2 * tl + 1] : qb[2 * tl + 1]) & mk, XA[m], XB[m]);
+                    mma16816(T.DD[tl][gm][m & 1], (sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk,
+                             (sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk,
+                             (sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk,
+                             (sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk, XA[gm][m], XB[gm][m]);
+        }
+        if (FMT == kQ3K) {
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm) {
+                ld_frag8(own0 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + t) : zaddr, XA[gm]);
+                ld_frag8(own1 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + 4 + t) : zaddr, XB[gm]);
             }
-            if (FMT == kQ3K) {
-                ld_frag8(own0 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + t) : zaddr, XA);
-                ld_frag8(own1 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + 4 + t) : zaddr, XB);
-                uint32_t ha[NR], hb[NR];
+            uint32_t ha[2][NR], hb[2][NR];
 #pragma unroll
-                for (int i = 0; i < NR; ++i) { ha[i] = gm ? hv[i].y : hv[i].x; hb[i] = ha[i] >> 8; }
+            for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
-                for (int m = 0; m < 8; ++m) {
-                    const uint32_t mk = 0x00010001u << m;
+                for (int i = 0; i < NR; ++i) { ha[gm][i] = gm ? hv[i].y : hv[i].x; hb[gm][i] = ha[gm][i] >> 8; }
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const uint32_t mk = 0x00010001u << m;
+#pragma unroll
+                for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
                     for (int tl = 0; tl < NT; ++tl)
-                        mma16816(T.DD[tl][gm][m & 1], ha[2 * tl] & mk, ha[2 * tl + 1] & mk, hb[2 * tl] & mk,
-                                 hb[2 * tl + 1] & mk, XA[m], XB[m]);
-                }
+                        mma16816(T.DD[tl][gm][m & 1], ha[gm][2 * tl] & mk, ha[gm][2 * tl + 1] & mk, hb[gm][2 * tl] & mk,
+                                 hb[gm][2 * tl + 1] & mk, XA[gm][m], XB[gm][m]);
             }
         }
     } else if (FMT == kQ4K) {
+        // pairs 8 hm + mm accumulate into group slot hm (the epilogue adds both)
         uint4 cA[NR], cB[NR];   // rows: sub-blocks t (unit 0) and t+4 (unit 1)
 #pragma unroll
         for (int i = 0; i < NR; ++i) {
@@ -365,24 +406,27 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
             cA[i] = lds128(st + w3 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t);
             cB[i] = lds128(st + w3 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t);
         }
+        uint32_t XA[2][8], XB[2][8];
 #pragma unroll
-        for (int hm = 0; hm < 2; ++hm) {   // pairs 8 hm .. 8 hm + 7
-            uint32_t XA[8], XB[8];
-            ld_frag8(own0 ? xb + 64 * t + 32 * hm : zaddr, XA);
-            ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * hm : zaddr, XB);
+        for (int hm = 0; hm < 2; ++hm) {
+            ld_frag8(own0 ? xb + 64 * t + 32 * hm : zaddr, XA[hm]);
+            ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * hm : zaddr, XB[hm]);
+        }
 #pragma unroll
-            for (int mm = 0; mm < 8; ++mm) {
+        for (int mm = 0; mm < 8; ++mm) {
+#pragma unroll
+            for (int hm = 0; hm < 2; ++hm) {
                 const int m = 8 * hm + mm, wi = m >> 2, j = m & 3;
                 const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
                 const int sh = j < 2 ? 0 : 8;
 #pragma unroll
                 for (int tl = 0; tl < NT; ++tl)
-                    mma16816(T.DD[tl][0][m & 1], (sub4(cA[2 * tl], wi) >> sh) & mk,
+                    mma16816(T.DD[tl][hm][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & mk,
                              (sub4(cA[2 * tl + 1], wi) >> sh) & mk, (sub4(cB[2 * tl], wi) >> sh) & mk,
-                             (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[mm], XB[mm]);
+                             (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[hm][mm], XB[hm][mm]);
             }
         }
-    } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7
+    } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7, four accumulators per row tile
         uint4 cA[NR], cB[NR];   // rows: blocks t and t+4
 #pragma unroll
         for (int i = 0; i < NR; ++i) {
@@ -395,10 +439,10 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
         ld_frag8(own1 ? xb + 64 * (t + 4) + 32 * half : zaddr, XB);
 #pragma unroll
         for (int mm = 0; mm < 8; ++mm) {
-            const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0;
+            const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0, a = mm & 3;
 #pragma unroll
             for (int tl = 0; tl < NT; ++tl)
-                mma16816(T.DD[tl][0][mm & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
+                mma16816(T.DD[tl][a >> 1][a & 1], (sub4(cA[2 * tl], wi) >> sh) & 0x00FF00FFu,
                          (sub4(cA[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, (sub4(cB[2 * tl], wi) >> sh) & 0x00FF00FFu,
                          (sub4(cB[2 * tl + 1], wi) >> sh) & 0x00FF00FFu, XA[mm], XB[mm]);
         }
@@ -469,8 +513,9 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
             const float m0 = (float)(((f >> 4) & 15u) | (((hi >> 2) & 3u) << 4));
             const float sc1 = (float)(((f >> 8) & 15u) | (((hi >> 4) & 3u) << 4));
             const float m1 = (float)(((f >> 12) & 15u) | (((hi >> 6) & 3u) << 4));
-            const float D0 = T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl];
-            const float D1 = T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1];
+            const float D0 = (T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl]) + (T.DD[tl][1][0][2 * hl] + T.DD[tl][1][1][2 * hl]);
+            const float D1 = (T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1]) +
+                             (T.DD[tl][1][0][2 * hl + 1] + T.DD[tl][1][1][2 * hl + 1]);
             const float a_sc = fmaf(sc1 * cf1, D1, sc0 * cf0 * D0);
             const float a_m = fmaf(m1, S1, m0 * S0);
             acc[i] += fmaf(d, a_sc, -dm * a_m);
@@ -486,8 +531,9 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
             const int tl = i >> 1, hl = i & 1, r = rec_of(i) - jj * 32;
             const float d0 = h2f(lds16(st + w0 + ((8 * jj + 2 * t) * 32 + r) * 2));
             const float d1 = h2f(lds16(st + w0 + ((8 * jj + 2 * t + 1) * 32 + r) * 2));
-            const float D0 = T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl];
-            const float D1 = T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1];
+            const float D0 = (T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl]) + (T.DD[tl][1][0][2 * hl] + T.DD[tl][1][1][2 * hl]);
+            const float D1 = (T.DD[tl][0][0][2 * hl + 1] + T.DD[tl][0][1][2 * hl + 1]) +
+                             (T.DD[tl][1][0][2 * hl + 1] + T.DD[tl][1][1][2 * hl + 1]);
             acc[i] += fmaf(d1, fmaf(D1, cf1, -o1), d0 * fmaf(D0, cf0, -o0));
         }
     }
@@ -528,36 +574,32 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     __shared__ float red[kRedBufs][kConsumers][2][kDecodeTok][32];
     __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
+    __shared__ int s_touch;
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
     __shared__ Geo geo[4][kDecodeTok];
     const Dims& d = A.d;
     // ---- set-up that does not depend on the routing result runs before the
     // wait for the previous kernel (overlapping its tail)
-    if (threadIdx.x < 4 * kDecodeTok) {
-        const int fmt = 1 + threadIdx.x / kDecodeTok, ntok = 1 + threadIdx.x % kDecodeTok;
-        Geo& G = geo[fmt - 1][ntok - 1];
-        const int nsb = kDown ? (d.I + 255) / 256 : (d.H + 255) / 256;
-        const TensorLayout L = tensor_layout(fmt, kDown ? d.H : d.I, kDown ? d.I : d.H);
-        const PlaneBytes pb = plane_bytes(fmt);
-        const int bmul = fmt == kQ80 ? 8 : 1;
-        G.per = stage_sb(fmt, ntok);
-        G.nst = (nsb + G.per - 1) / G.per;
-        G.npl = pb.n;
-        int at = 0;
-        for (int pl = 0; pl < 4; ++pl) {
-            G.woff[pl] = at;
-            G.cstr[pl] = pl < pb.n ? 32 * bmul * pb.b[pl] : 0;
-            G.pl[pl] = L.plane[pl];
-            G.rbstr[pl] = pl < pb.n ? L.blocks_per_row * 32 * pb.b[pl] : 0;
-            if (pl < pb.n) at += (32 * bmul * G.per * pb.b[pl] + 127) & ~127;
-        }
-        const TokLay tl = tok_lay(fmt, G.per);
-        G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.tx1 = tl.x1; G.ts = tl.s;
+    {
+        // stage geometry (host-computed) into shared memory, one word per thread
+        static_assert(sizeof(geo) % 4 == 0, "geometry table");
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(&A.geo[0][0]);
+        uint32_t* dst = reinterpret_cast<uint32_t*>(&geo[0][0]);
+        for (int i = threadIdx.x; i < (int)(sizeof(geo) / 4); i += kThreads) dst[i] = src[i];
     }
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
     if (threadIdx.x < kNST) s_posted[threadIdx.x] = -1;
     if (threadIdx.x < 8) zero_blk[threadIdx.x] = 0u;
     if (threadIdx.x == 0) s_fail = 0;
+    {
+        // Touch the expert table (a kernel parameter) once on this SM, so the
+        // per-slot pointer lookups made after the routing result arrives (one
+        // distinct expert per lane) hit the constant cache.
+        uintptr_t v = 0;
+        for (int i = threadIdx.x; i < 3 * (d.E + 1); i += kThreads) v |= reinterpret_cast<uintptr_t>(tab.p[i / 3][i % 3]);
+        for (int i = threadIdx.x; i < d.E + 1; i += kThreads) v |= (uintptr_t)tab.fmt[i][0] << 8;
+        if (v == 1) s_touch = 1;   // never true (pointers are 256-byte aligned); keeps the loads
+    }
     const uint32_t zaddr = (uint32_t)__cvta_generic_to_shared(zero_blk);
     if (threadIdx.x == 0) {
         for (int s = 0; s < kNST; ++s) {
@@ -615,11 +657,17 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             // read through L2 (ld.global.cg): the down kernel reads before its
             // wait, and an SM's L1 may still hold lines of an earlier call
             n_slots = __ldcg(&A.plan->n_slots);
-            for (int i = lane; i < kMaxExperts + 2; i += 32) {
+            // one pass per 32 slots (one for a decode call): the pass's loads
+            // go out together, then the stores
+            for (int i = lane; i <= n_slots; i += 32) {
                 const int pre = __ldcg(kDown ? &A.plan->pre_dn[i] : &A.plan->pre_gu[i]);
-                const int e = __ldcg(&A.plan->slot_e[i]), first = __ldcg(&A.plan->slot_first[i]);
-                const int ntot = __ldcg(&A.plan->slot_ntot[i]);
-                if (i <= n_slots) sc.pre[i] = pre;
+                int e = 0, first = 0, ntot = 0;
+                if (i < n_slots) {
+                    e = __ldcg(&A.plan->slot_e[i]);
+                    first = __ldcg(&A.plan->slot_first[i]);
+                    ntot = __ldcg(&A.plan->slot_ntot[i]);
+                }
+                sc.pre[i] = pre;
                 if (i < n_slots) {
                     sc.e[i] = e;
                     sc.first[i] = first;
@@ -631,7 +679,19 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 }
             }
             const int n_routed = min(d.T * d.K, kMaxCachedAssign);
-            for (int i = lane; i < n_routed; i += 32) s_perm[i] = __ldcg(A.perm + i);
+            for (int i0 = 0; i0 < n_routed; i0 += 128) {
+                int v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int i = i0 + 32 * u + lane;
+                    v[u] = i < n_routed ? __ldcg(A.perm + i) : 0;
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int i = i0 + 32 * u + lane;
+                    if (i < n_routed) s_perm[i] = v[u];
+                }
+            }
             __syncwarp();
             n_items = sc.pre[n_slots];
             routed = true;
@@ -641,18 +701,18 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // items are handed out by a global counter (zeroed per call), in slot
         // order: the shared expert's (Q8_0, the heaviest) first, so the CTAs
         // even out on the lighter routed items that follow
-        int id_next = 0;
-        if (lane == 0) id_next = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
-        id_next = __shfl_sync(kFull, id_next, 0);
+        auto claim = [&]() -> int {
+            int v = 0;
+            if (lane == 0) v = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+            return __shfl_sync(kFull, v, 0);
+        };
+        int id_next = claim();
         for (int k = 0;; ++k) {
             const int id = id_next;
             if (!routed && id >= n_sh_items) wait_routing();
             const int item = id < n_items ? id : -1;
-            if (item >= 0) {
-                // claim the following item now; the atomic's latency hides behind this item's stages
-                if (lane == 0) id_next = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
-                id_next = __shfl_sync(kFull, id_next, 0);
-            }
+            // claim the following item now; the atomic's latency hides behind this item's stages
+            if (item >= 0) id_next = claim();
             if (item >= 0) decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
             const int nst = item >= 0 ? P.nst : 1;
             bool failed = false;
@@ -753,6 +813,12 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             const uint32_t stage = ring + slot * kStageBytes;
             const int fmt = H.fmt, ks = H.ks, ntok = H.ntok;
             const Geo& GS = geo[fmt - 1][ntok - 1];
+            // superblock jj of the stage goes to warp column (jj + s) % kCols, s the
+            // stage's first superblock counted over the whole item, so every warp
+            // gets the same share of an item even where a stage's count is not a
+            // multiple of kCols
+            const int s_item = H.s0 + ((H.tensor & 1) ? (kDown ? A.nsbi : A.nsbx) : 0);
+            const int wcol = (col - s_item % kCols + kCols) % kCols;
             if ((H.tensor == 1 || H.tensor == 3) && H.s0 == 0) {
                 // first stage of the second phase: the first phase's sums are complete
 #pragma unroll
@@ -765,9 +831,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 if (tk >= ntok) break;
                 // one-token items have the registers to keep two tiles of MMA sums
                 // in flight (Q3_K's second code plane does not fit them)
-                constexpr bool kPair = MT == 1;
+                constexpr bool kPair = false;
                 if (fmt == kQ80) {
-                    for (int jj = col; jj < ks; jj += kCols) {
+                    for (int jj = wcol; jj < ks; jj += kCols) {
                         TileAcc<kNT> T0, T1;
                         tile_mma<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, T0);
                         if (!kPair) tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
@@ -776,11 +842,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         tile_epi<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, T1, cur[tk]);
                     }
                 } else if (fmt == kQ2K) {
-                    tile_pairs<kQ2K, kPair>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ2K, kPair>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 } else if (fmt == kQ3K) {
-                    tile_pairs<kQ3K, false>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ3K, false>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 } else {
-                    tile_pairs<kQ4K, kPair>(GS, stage, col, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_pairs<kQ4K, kPair>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 }
             }
             // fields needed after the slot is released to the producer
@@ -911,6 +977,11 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.next = w.counters;
     A.err = w.err;
     A.out = out;
+    auto fill_geo = [&](bool down) {
+        for (int f = 1; f <= 4; ++f)
+            for (int n = 1; n <= kDecodeTok; ++n) make_geo(A.geo[f - 1][n - 1], d, down, f, n);
+    };
+    fill_geo(false);
     // one token: every item carries one, and the accumulators shrink to one token's
     const bool one = d.T == 1;
     prof_begin("gateup_mma", s);
@@ -918,6 +989,7 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
                           : launch_pdl(ffn_kernel<false, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
+    fill_geo(true);
     prof_begin("down_mma", s);
     err = one ? launch_pdl(ffn_kernel<true, 1>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A)
               : launch_pdl(ffn_kernel<true, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
@@ -927,6 +999,8 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
 }
 
 cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s) {
+    static const bool carve = (prefer_max_shared(combine_kernel), true);
+    (void)carve;
     prof_begin("combine", s);
     // one CTA row per token (up to 65535; the kernel strides over the rest),
     // so large batches stream the partial outputs at full bandwidth

@@ -19,6 +19,7 @@
 
 #include "mq_actprep.cuh"
 #include "mq_internal.h"
+#include "mq_select.cuh"
 
 namespace mq {
 namespace {
@@ -216,119 +217,6 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
     }
 }
 
-// ---------------------------------------------------------------------------
-// scores + group-limited top-k: one warp per token
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ float canonical_sigmoid(float z) {
-    const float kLog2e = 0x1.715476p+0f, kLn2Hi = 0x1.62e4p-1f, kLn2Lo = 0x1.7f7d1cp-20f;
-    float a = __fsub_rn(0.0f, z);
-    if (a > 87.0f) a = 87.0f;
-    if (a < -87.0f) a = -87.0f;
-    const float n = rintf(__fmul_rn(a, kLog2e));
-    float r = __fmaf_rn(-n, kLn2Hi, a);
-    r = __fmaf_rn(-n, kLn2Lo, r);
-    // e^r = sum r^i / i!, i <= 7
-    float p = 0x1.a01a02p-13f;
-    p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);
-    p = __fmaf_rn(p, r, 0x1.111112p-7f);
-    p = __fmaf_rn(p, r, 0x1.555556p-5f);
-    p = __fmaf_rn(p, r, 0x1.555556p-3f);
-    p = __fmaf_rn(p, r, 0.5f);
-    p = __fmaf_rn(p, r, 1.0f);
-    p = __fmaf_rn(p, r, 1.0f);
-    const float two_n = __int_as_float(((int)n + 127) << 23);
-    const float ex = __fmul_rn(p, two_n);
-    return __fdiv_rn(1.0f, __fadd_rn(1.0f, ex));
-}
-
-// Order-preserving map of a finite fp32 value to uint32 (0 is below every
-// finite value and marks "not available").
-__device__ __forceinline__ uint32_t ord_key(float f) {
-    const uint32_t b = __float_as_uint(f);
-    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-}
-// Warp argmax over one candidate per lane: largest key, then lowest index.
-__device__ __forceinline__ int warp_argmax_key(uint32_t key, int idx) {
-    const uint32_t kmax = __reduce_max_sync(kFull, key);
-    return (int)__reduce_min_sync(kFull, key == kmax ? (uint32_t)idx : 0xffffffffu);
-}
-
-// One warp routes one token.  Lane l holds experts l, l+32, ... (E <= 256).
-// uw: per-warp scratch of E floats; g_sh: per-warp scratch of G floats.
-__device__ __forceinline__ void route_token(const float* __restrict__ z, const float* __restrict__ bias, int E,
-                                            int G, int Gk, int K, float routed_scale, int t, float* uw,
-                                            float* g_sh, int32_t* __restrict__ idx, float* __restrict__ wts) {
-    const int lane = threadIdx.x & 31;
-    const int gs = E / G;
-    float s[8], u[8];
-    int grp[8];
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-        const int e = lane + 32 * m;
-        s[m] = 0.0f; u[m] = 0.0f; grp[m] = 0;
-        if (e < E) {
-            s[m] = canonical_sigmoid(z[(size_t)t * E + e]);
-            u[m] = __fadd_rn(s[m], bias ? bias[e] : 0.0f);
-            grp[m] = e / gs;
-            uw[e] = u[m];
-        }
-    }
-    __syncwarp();
-    // group score = sum of the two largest u of the group (scan in index order)
-    for (int g = lane; g < G; g += 32) {
-        float top1 = -INFINITY, top2 = -INFINITY;
-        const float* ug = uw + g * gs;
-#pragma unroll 8
-        for (int i = 0; i < gs; ++i) {
-            const float v = ug[i];
-            if (v > top1) { top2 = top1; top1 = v; }
-            else if (v > top2) top2 = v;
-        }
-        g_sh[g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
-    }
-    __syncwarp();
-    // keep topk_group groups: repeated argmax, ties to the lower index
-    uint64_t kept = 0;
-    const uint32_t gk0 = lane < G ? ord_key(g_sh[lane]) : 0u;
-    const uint32_t gk1 = lane + 32 < G ? ord_key(g_sh[lane + 32]) : 0u;
-    for (int r = 0; r < Gk; ++r) {
-        uint32_t k = 0u;
-        int i = 0x7fffffff;
-        if (lane < G && !((kept >> lane) & 1)) { k = gk0; i = lane; }
-        if (lane + 32 < G && !((kept >> (lane + 32)) & 1) && gk1 > k) { k = gk1; i = lane + 32; }
-        kept |= 1ull << warp_argmax_key(k, i);
-    }
-    // top_k experts by u among the kept groups, descending, ties to the lower id
-    uint32_t key[8];
-#pragma unroll
-    for (int m = 0; m < 8; ++m) key[m] = (lane + 32 * m < E && ((kept >> grp[m]) & 1)) ? ord_key(u[m]) : 0u;
-    int sel = 0;
-    float ssum = 0.0f, mys = 0.0f;
-    for (int j = 0; j < K; ++j) {
-        uint32_t bk = 0u;
-        int bm = 0;
-#pragma unroll
-        for (int m = 0; m < 8; ++m)
-            if (key[m] > bk) { bk = key[m]; bm = m; }   // strict: the lower expert id wins a tie
-        const int bi = warp_argmax_key(bk, lane + 32 * bm);
-        float win = 0.0f;
-        if ((bi & 31) == lane) {
-            const int m = bi >> 5;
-#pragma unroll
-            for (int mm = 0; mm < 8; ++mm)
-                if (mm == m) { key[mm] = 0u; win = s[mm]; }
-        }
-        const float sv = __shfl_sync(kFull, win, bi & 31);
-        ssum = __fadd_rn(ssum, sv);   // slot order, identical on every lane
-        if (lane == j) { sel = bi; mys = sv; }   // lane j keeps slot j
-    }
-    // weights: s_j / sum(s), summed in slot order, times routed_scale
-    if (lane < K) {
-        idx[(size_t)t * K + lane] = sel;
-        wts[(size_t)t * K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), routed_scale);
-    }
-}
-
 constexpr int kTopkWarps = 4;
 
 __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __restrict__ z,
@@ -342,7 +230,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __re
     const int w = threadIdx.x >> 5;
     const int t = blockIdx.x * kTopkWarps + w;
     if (t >= d.T) return;
-    route_token(z, bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, u_sh[w], g_sh[w], idx, wts);
+    sel::route_token(z, bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, u_sh[w], g_sh[w], idx, wts);
 }
 
 // ---------------------------------------------------------------------------
@@ -378,9 +266,68 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
     __syncthreads();
     pdl_wait();
     pdl_launch();
+    if (z != nullptr && d.T == 1 && d.K <= 32 && E <= 256) {
+        // One token: the selection holds K distinct experts, one entry each, so
+        // the counting sort reduces to ranking them.  One warp does all of it
+        // in registers (no block barriers, nothing read back from global memory).
+        if (warp != 0) return;
+        const int K = d.K;
+        int sel = 0;
+        sel::route_token(z, s_bias, d.E, d.G, d.Gk, K, d.routed_scale, 0, reinterpret_cast<float*>(cnt[0]), g_sh[0],
+                         idx, wts, &sel);
+        // the selection as a 256-bit set; an expert's rank (and offsets[e]) is
+        // the number of selected ids below it
+        uint32_t mask[8];
+#pragma unroll
+        for (int w = 0; w < 8; ++w)
+            mask[w] = __reduce_or_sync(kFull, (lane < K && (sel >> 5) == w) ? 1u << (sel & 31) : 0u);
+        auto below = [&](int e) {   // selected ids < e (e <= 256)
+            int c = 0;
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+                c += __popc(32 * w + 32 <= e ? mask[w] : (32 * w < e ? mask[w] & ((1u << (e & 31)) - 1u) : 0u));
+            return c;
+        };
+        const int rank = below(sel);
+        if (lane < K) {
+            perm[rank] = lane;   // entry a = t * K + j = j
+            inv[lane] = rank;
+            active[1 + rank] = sel;
+        }
+        if (lane == 0) active[0] = K;
+        // offsets[e] = selected experts with a lower id; offsets[E] = K
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int e = lane * 8 + q;
+            if (e < E) offsets[e] = below(e);
+        }
+        if (lane == 0) offsets[E] = K;
+        if (plan == nullptr) return;
+        // work plan: slot p (shared expert first) holds one token
+        const int n_slots = K + d.has_shared;
+        for (int p = lane; p <= kMaxExperts + 1; p += 32) {
+            const int pc = min(p, n_slots);
+            plan->pre_gu[p] = pc * (d.I / 32);
+            plan->pre_dn[p] = pc * (d.H / 64);
+        }
+        // slot of the expert of rank r: has_shared + r
+        if (lane < K) {
+            const int p = d.has_shared + rank;
+            plan->slot_e[p] = sel;
+            plan->slot_first[p] = rank;
+            plan->slot_ntot[p] = 1;
+        }
+        if (lane == 0) {
+            if (d.has_shared) { plan->slot_e[0] = d.E; plan->slot_first[0] = 0; plan->slot_ntot[0] = 1; }
+            plan->n_slots = n_slots;
+            plan->dn_target = n_slots;
+            plan->ntg_max = 1;
+        }
+        return;
+    }
     if (z != nullptr) {
         for (int t = warp; t < d.T; t += kPermWarps)
-            route_token(z, s_bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
+            sel::route_token(z, s_bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
                         g_sh[warp], idx, wts);
         __syncthreads();
     }
@@ -522,6 +469,8 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
                                  __half* x16, uint32_t* zero_words, int n_zero, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
+    static const bool carve = (prefer_max_shared(router_logits_kernel), prefer_max_shared(router_logits_tile_kernel), true);
+    (void)carve;
     prof_begin("router_logits", s);
     cudaError_t e;
     if (xq == nullptr && d.T >= 16 && nseg <= 8) {
@@ -541,6 +490,8 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                         cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
+    static const bool carve = (prefer_max_shared(topk_kernel), true);
+    (void)carve;
     prof_begin("router_topk", s);
     const cudaError_t e = launch_pdl(topk_kernel, dim3((d.T + kTopkWarps - 1) / kTopkWarps), dim3(kTopkWarps * 32),
                                      0, s, z, bias, d, idx, wts);
@@ -550,6 +501,8 @@ cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_
 
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, Plan* plan, cudaStream_t s) {
+    static const bool carve = (prefer_max_shared(permute_kernel), true);
+    (void)carve;
     prof_begin("permute", s);
     const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, const_cast<int32_t*>(idx), d,
                                      offsets, perm, inv, active, plan, (const float*)nullptr, (const float*)nullptr,
@@ -561,6 +514,8 @@ cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, 
 cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                                  int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
                                  cudaStream_t s) {
+    static const bool carve = (prefer_max_shared(permute_kernel), true);
+    (void)carve;
     prof_begin("route_permute", s);
     const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, idx, d, offsets, perm, inv,
                                      active, plan, z, bias, wts);

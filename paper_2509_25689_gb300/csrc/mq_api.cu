@@ -249,14 +249,14 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     if (topk_w) w.wts = topk_w;
     const int pm = path_mode();
     const bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
+    const bool tc = !prefill && pm == 3 && decode_tc_fits(d);
     rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1);
     if (rc != MQ_OK) return rc;
     if (prefill) {
         if (launch_prefill(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;
         return MQ_OK;
     }
-    const cudaError_t e = (pm == 3 && decode_tc_fits(d)) ? launch_decode_tc(d, tab, w, out, s)
-                                                         : launch_decode_mma(d, tab, w, out, s);
+    const cudaError_t e = tc ? launch_decode_tc(d, tab, w, out, s) : launch_decode_mma(d, tab, w, out, s);
     if (e != cudaSuccess) return MQ_ECUDA;
     return MQ_OK;
 }

@@ -93,6 +93,14 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
+
+// The small kernels of a layer call ask for the largest shared-memory
+// carveout as the FFN kernels (227 KB per CTA) need it, so an SM keeps one
+// L1/shared split across the call instead of switching between kernels.
+template <typename... KArgs>
+void prefer_max_shared(void (*kernel)(KArgs...)) {
+    cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
+}
 #endif
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
