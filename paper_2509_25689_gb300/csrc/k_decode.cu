@@ -362,25 +362,26 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
                 qa[gm][i] = sub4(c[i], 2 * gm); qb[gm][i] = sub4(c[i], 2 * gm + 1);
                 sa[gm][i] = qa[gm][i] >> 10; sbb[gm][i] = qb[gm][i] >> 10;
             }
+        if (FMT == kQ2K) {
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-            const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
-            const bool sh = m > 4;
+            for (int m = 0; m < 8; ++m) {
+                const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
+                const bool sh = m > 4;
 #pragma unroll
-            for (int gm = 0; gm < 2; ++gm)
+                for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
-                for (int tl = 0; tl < NT; ++tl)
-                    mma16816(T.DD[tl][gm][m & 1], (sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk,
-                             (sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk,
-                             (sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk,
-                             (sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk, XA[gm][m], XB[gm][m]);
-        }
-        if (FMT == kQ3K) {
-#pragma unroll
-            for (int gm = 0; gm < 2; ++gm) {
-                ld_frag8(own0 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + t) : zaddr, XA[gm]);
-                ld_frag8(own1 ? tb + h.tx1 + jj * 512 + 32 * (8 * gm + 4 + t) : zaddr, XB[gm]);
+                    for (int tl = 0; tl < NT; ++tl)
+                        mma16816(T.DD[tl][gm][m & 1], (sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk,
+                                 (sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk,
+                                 (sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk,
+                                 (sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk, XA[gm][m], XB[gm][m]);
             }
+        } else {
+            // Q3_K: the high bit of pair m (bit m of its half of the hmask word)
+            // goes right above the pair's 2-bit code, so one operand carries the
+            // 3-bit code (low2 + 4 hbit) at the code's positional power.  Bit 10
+            // of an fp16 still has the subnormal ulp (2^-24), so position 10
+            // (m = 4) stays linear.
             uint32_t ha[2][NR], hb[2][NR];
 #pragma unroll
             for (int gm = 0; gm < 2; ++gm)
@@ -388,13 +389,21 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
                 for (int i = 0; i < NR; ++i) { ha[gm][i] = gm ? hv[i].y : hv[i].x; hb[gm][i] = ha[gm][i] >> 8; }
 #pragma unroll
             for (int m = 0; m < 8; ++m) {
-                const uint32_t mk = 0x00010001u << m;
+                const int pos = m <= 4 ? 2 * m : 2 * (m - 5);
+                const uint32_t mk = 0x00030003u << pos, mh = 0x00040004u << pos;
+                const bool sh = m > 4;
+                // hbit m from bit m to bit pos + 2
+                auto hsh = [&](uint32_t w) { return (m <= 4 ? (w << (m + 2)) : (w >> (8 - m))) & mh; };
 #pragma unroll
                 for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
                     for (int tl = 0; tl < NT; ++tl)
-                        mma16816(T.DD[tl][gm][m & 1], ha[gm][2 * tl] & mk, ha[gm][2 * tl + 1] & mk, hb[gm][2 * tl] & mk,
-                                 hb[gm][2 * tl + 1] & mk, XA[gm][m], XB[gm][m]);
+                        mma16816(T.DD[tl][gm][m & 1],
+                                 ((sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk) | hsh(ha[gm][2 * tl]),
+                                 ((sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk) | hsh(ha[gm][2 * tl + 1]),
+                                 ((sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk) | hsh(hb[gm][2 * tl]),
+                                 ((sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk) | hsh(hb[gm][2 * tl + 1]),
+                                 XA[gm][m], XB[gm][m]);
             }
         }
     } else if (FMT == kQ4K) {
