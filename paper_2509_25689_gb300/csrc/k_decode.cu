@@ -153,8 +153,14 @@ constexpr int kCols = kConsumers * kNT / 2;         // superblock columns the wa
 constexpr int kRedBufs = kConsumers >= 16 ? 1 : 2;  // item-end reduction buffers (smem budget)
 constexpr int kThreads = (kConsumers + 1) * 32;     // + one producer warp
 constexpr int kProducerWarp = kConsumers;
-constexpr int kNST = 3;                             // ring stages
-constexpr int kStageBytes = 64 * 1024;
+// Ring: 3 slots of 64 KB (gate/up: Q8_0 stages of the shared expert are
+// 61 KB) or 4 of 48 KB (down: Q3_K stages are 37 KB, more of them in flight)
+constexpr int kNSTmax = 4;
+__host__ __device__ constexpr int ring_slots(bool down) { return down ? 4 : 3; }
+__host__ __device__ constexpr int slot_bytes(bool down) { return down ? 48 * 1024 : 64 * 1024; }
+constexpr int kRingBytes = 192 * 1024;
+static_assert(ring_slots(false) * slot_bytes(false) == kRingBytes && ring_slots(true) * slot_bytes(true) == kRingBytes,
+              "ring size");
 constexpr int kStageSb = 16;                        // superblocks per stage (Q8_0: 8), fewer if over budget
 constexpr int kMaxCachedAssign = 2048;              // routed assignments cached in smem
 constexpr uint32_t kErrFull = 1u, kErrEmpty = 2u;
@@ -171,14 +177,14 @@ struct __align__(16) Hdr {
     int32_t asg[kDecodeTok];
 };
 
-// token pieces in a stage: the family fragments, the Q3_K high-bit fragments
-// and the per-superblock statistics, each for the stage's ks superblocks
-struct TokLay { int x, x1, s, stride; };
+// token pieces in a stage: the family fragments and the per-superblock
+// statistics, each for the stage's ks superblocks
+struct TokLay { int x, s, stride; };
 __host__ __device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
+    (void)fmt;
     TokLay t;
     int at = 0;
     t.x = at; at += ks * 512;
-    t.x1 = at; if (fmt == kQ3K) at += ks * 512;
     t.s = at; at += ks * kStatFloats * 4;
     t.stride = (at + 127) & ~127;
     return t;
@@ -191,10 +197,10 @@ __host__ __device__ __forceinline__ int weight_stage_bytes(int fmt, int ks) {
     for (int p = 0; p < pb.n; ++p) at += (32 * nblk * pb.b[p] + 127) & ~127;
     return at;
 }
-// superblocks per stage for a format and token count (fits kStageBytes)
-__host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok) {
+// superblocks per stage for a format and token count (fits a ring slot)
+__host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok, int stage_bytes) {
     int ks = fmt == kQ80 ? kStageSb / 2 : kStageSb;
-    while (ks > 1 && weight_stage_bytes(fmt, ks) + ntok * tok_lay(fmt, ks).stride > kStageBytes) --ks;
+    while (ks > 1 && weight_stage_bytes(fmt, ks) + ntok * tok_lay(fmt, ks).stride > stage_bytes) --ks;
     return ks;
 }
 
@@ -214,7 +220,7 @@ struct Geo {
     int64_t rbstr[4];    // bytes per 32-row block in each plane
     int per, nst, npl;   // superblocks per stage, stages per tensor, planes
     int woff[4], cstr[4];// plane regions in the stage, bytes per superblock
-    int tok0, tstride, tx, tx1, ts;
+    int tok0, tstride, tx, ts;
 };
 
 // Stage geometry of (format, tokens per item) for the gate/up (down = false)
@@ -224,7 +230,7 @@ __host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int f
     const TensorLayout L = tensor_layout(fmt, down ? d.H : d.I, down ? d.I : d.H);
     const PlaneBytes pb = plane_bytes(fmt);
     const int bmul = fmt == kQ80 ? 8 : 1;
-    G.per = stage_sb(fmt, ntok);
+    G.per = stage_sb(fmt, ntok, slot_bytes(down));
     G.nst = (nsb + G.per - 1) / G.per;
     G.npl = pb.n;
     int at = 0;
@@ -236,7 +242,7 @@ __host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int f
         if (pl < pb.n) at += (32 * bmul * G.per * pb.b[pl] + 127) & ~127;
     }
     const TokLay tl = tok_lay(fmt, G.per);
-    G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.tx1 = tl.x1; G.ts = tl.s;
+    G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.ts = tl.s;
 }
 
 struct DecodeArgs {
@@ -578,10 +584,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
-    __shared__ __align__(8) uint64_t bars[2 * kNST];
-    __shared__ Hdr hdr[kNST];
+    constexpr int kNST = ring_slots(kDown), kStageBytes = slot_bytes(kDown);
+    __shared__ __align__(8) uint64_t bars[2 * kNSTmax];
+    __shared__ Hdr hdr[kNSTmax];
     __shared__ float red[kRedBufs][kConsumers][2][kDecodeTok][32];
-    __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
+    __shared__ int s_posted[kNSTmax];   // last stage index posted to each ring slot
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
     __shared__ int s_touch;
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
@@ -643,7 +650,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // The CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...  Per
         // phase (one tensor of one item) every lane owns at most one copy:
         // lanes 0..3 a weight plane, lanes 4.. one piece of one token (family
-        // fragments, Q3_K high-bit fragments, statistics).  A stage then only
+        // fragments or statistics).  A stage then only
         // advances the source by the stage's first superblock.
         const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi}
                                 : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
@@ -755,8 +762,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         c_stride = G->cstr[lane];
                         c_dst = G->woff[lane];
                     }
-                    if (lane >= 4 && lane < 4 + 3 * P.ntok) {
-                        const int tk = (lane - 4) / 3, piece = (lane - 4) - 3 * tk;
+                    if (lane >= 4 && lane < 4 + 2 * P.ntok) {
+                        const int tk = (lane - 4) / 2, piece = (lane - 4) - 2 * tk;
                         int v = P.vec[0];
 #pragma unroll
                         for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) v = P.vec[t2];
@@ -765,10 +772,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         const int fam = fmt == kQ2K || fmt == kQ3K ? kF2 : fmt == kQ4K ? kF4 : kF8;
                         const uint32_t tb = G->tok0 + tk * G->tstride;
                         if (piece == 0) { c_src = qv + (size_t)fam * vs.nsb * 512; c_stride = 512; c_dst = tb + G->tx; }
-                        if (piece == 1 && fmt == kQ3K) {
-                            c_src = qv + (size_t)kF1 * vs.nsb * 512; c_stride = 512; c_dst = tb + G->tx1;
-                        }
-                        if (piece == 2) { c_src = sv; c_stride = kStatFloats * 4; c_dst = tb + G->ts; }
+                        if (piece == 1) { c_src = sv; c_stride = kStatFloats * 4; c_dst = tb + G->ts; }
                     }
                 }
                 const int per = G->per;
@@ -964,7 +968,7 @@ size_t decode_counter_bytes(const Dims& d) {
 
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
-    const int smem = kNST * kStageBytes;
+    const int smem = kRingBytes;
     if (g_num_sms == 0) {
         int dev = 0;
         cudaGetDevice(&dev);

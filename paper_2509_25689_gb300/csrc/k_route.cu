@@ -117,7 +117,8 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
             for (int jb = 32 * seg + e; jb < 32 * seg + 32 && jb < 8 * nsb; jb += E) {
                 const int k = 32 * jb + lane;
                 const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
-                prep_block32(v, jb, 0xF, xq + (size_t)t * qstride, xs + (size_t)t * sstride, nsb);
+                prep_block32(v, jb, (1 << kF2) | (1 << kF4) | (1 << kF8), xq + (size_t)t * qstride,
+                             xs + (size_t)t * sstride, nsb);
             }
         }
     }

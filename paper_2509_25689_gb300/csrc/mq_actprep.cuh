@@ -10,14 +10,15 @@
 //   - sigma = 2^ex, ex chosen so the block maximum scales into [2^12, 2^13);
 //     xt = fp16(v / sigma) is the fp16 activation every kernel uses (exact
 //     for bf16 inputs), and c = 2^24 * sigma undoes both scalings;
-//   - four fp16 copies of xt in natural element order, one per code family,
-//     each element divided by the power of two its code carries:
-//       F2 (2-bit codes: Q2_K, low bits of Q3_K), F1 (Q3_K high bit, times
-//       4), F4 (4-bit codes: Q4_K), F8 (8-bit codes: Q8_0, none);
+//   - fp16 copies of xt in natural element order, one per code family, each
+//     element divided by the power of two its code carries: F2 (2-bit code
+//     positions: Q2_K, and Q3_K whose high bit the kernels place right above
+//     the pair's 2-bit code), F4 (4-bit codes: Q4_K), F8 (8-bit codes: Q8_0,
+//     none); slot 1 of the layout is not used;
 //   - the sums sigma * sum(xt) over every 16- and 32-element sub-block (the
 //     sub-block min terms of Q2_K / Q4_K, the -4 offset of Q3_K codes and the
 //     +128 offset of Q8_0 codes).
-// Layout per vector: halves [4 families][nsb][256] and, per superblock, a
+// Layout per vector: halves [4 family slots][nsb][256] and, per superblock, a
 // 32-float record {c[8] | S16[16] in slot order | S32[8]}.
 #pragma once
 #include <cuda_fp16.h>
@@ -25,7 +26,7 @@
 
 namespace mq {
 
-enum Family : int { kF2 = 0, kF1 = 1, kF4 = 2, kF8 = 3 };
+enum Family : int { kF2 = 0, kF4 = 2, kF8 = 3 };
 
 constexpr int kStatFloats = 32;   // floats of statistics per superblock
 constexpr int kStatC = 0, kStatS16 = 8, kStatS32 = 24;
@@ -33,7 +34,6 @@ constexpr int kStatC = 0, kStatS16 = 8, kStatS32 = 24;
 // power of two carried by the code pair m of each family (bit offset of the
 // code inside its fp16 half after the word is read, see the decode kernels)
 __host__ __device__ __forceinline__ int pair_shift2(int m) { return m <= 4 ? 2 * m : 2 * (m - 5); }   // m < 8
-__host__ __device__ __forceinline__ int pair_shift1(int m) { return m; }                              // m < 8
 __host__ __device__ __forceinline__ int pair_shift4(int m) { return 4 * (m & 1); }                    // m < 16
 
 // slot of 16-wide sub-block j (< 16): lane t of a warp owns slots 4t..4t+3,
@@ -67,7 +67,6 @@ __device__ __forceinline__ void prep_block32(float v, int jb, int fam_mask, __ha
     const size_t fam_stride = (size_t)nsb * 256;
     const int m16 = (kk & 15) >> 1, m32 = (kk & 31) >> 1;
     if (fam_mask & (1 << kF2)) qs[kF2 * fam_stride] = __float2half_rn(ldexpf(xt, -pair_shift2(m16)));
-    if (fam_mask & (1 << kF1)) qs[kF1 * fam_stride] = __float2half_rn(ldexpf(4.0f * xt, -pair_shift1(m16)));
     if (fam_mask & (1 << kF4)) qs[kF4 * fam_stride] = __float2half_rn(ldexpf(xt, -pair_shift4(m32)));
     if (fam_mask & (1 << kF8)) qs[kF8 * fam_stride] = __float2half_rn(xt);
     const float s16 = half_warp_sum(xt);
@@ -85,7 +84,7 @@ __device__ __forceinline__ void prep_block32(float v, int jb, int fam_mask, __ha
 
 // family mask needed by a weight format
 __host__ __device__ __forceinline__ int families_of(int fmt) {
-    return fmt == 1 ? (1 << kF2) : fmt == 2 ? ((1 << kF2) | (1 << kF1)) : fmt == 3 ? (1 << kF4) : (1 << kF8);
+    return fmt == 1 || fmt == 2 ? (1 << kF2) : fmt == 3 ? (1 << kF4) : (1 << kF8);
 }
 
 }  // namespace mq
