@@ -324,9 +324,7 @@ __device__ __forceinline__ void ld_frag8(uint32_t a, uint32_t (&X)[8]) {
 template <int NT> struct TileAcc { float DD[NT][2][2][4]; };
 
 // Loads one (superblock, token) tile of the warp's rows and issues its MMAs
-// into T; tile_epi applies the scales once the sums are in.  Callers issue the
-// MMAs of the next tile before the epilogue of the current one, so the MMA
-// latency of one tile runs under the other's epilogue.
+// into T; tile_epi applies the scales once the sums are in.
 template <int FMT, int NT>
 __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int half, int rt0, int tk,
                                          uint32_t zaddr, TileAcc<NT>& T) {
@@ -554,26 +552,14 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
     }
 }
 
-// The warp's superblocks col, col + kCols, ... of a stage.  PAIR: two at a
-// time, the second tile's MMAs issued before the first tile's epilogue.
-template <int FMT, bool PAIR>
-__device__ __forceinline__ void tile_pairs(const Geo& h, uint32_t st, int col, int ks, int rt0, int tk,
-                                           uint32_t zaddr, float (&acc)[4]) {
-    if (PAIR) {
-        for (int jj = col; jj < ks; jj += 2 * kCols) {
-            const bool two = jj + kCols < ks;
-            TileAcc<kNT> T0, T1;
-            tile_mma<FMT, kNT>(h, st, jj, 0, rt0, tk, zaddr, T0);
-            if (two) tile_mma<FMT, kNT>(h, st, jj + kCols, 0, rt0, tk, zaddr, T1);
-            tile_epi<FMT, kNT>(h, st, jj, 0, rt0, tk, T0, acc);
-            if (two) tile_epi<FMT, kNT>(h, st, jj + kCols, 0, rt0, tk, T1, acc);
-        }
-    } else {
-        for (int jj = col; jj < ks; jj += kCols) {
-            TileAcc<kNT> T0;
-            tile_mma<FMT, kNT>(h, st, jj, 0, rt0, tk, zaddr, T0);
-            tile_epi<FMT, kNT>(h, st, jj, 0, rt0, tk, T0, acc);
-        }
+// The warp's superblocks col, col + kCols, ... of a stage, one tile at a time.
+template <int FMT>
+__device__ __forceinline__ void tile_cols(const Geo& h, uint32_t st, int col, int ks, int rt0, int tk,
+                                          uint32_t zaddr, float (&acc)[4]) {
+    for (int jj = col; jj < ks; jj += kCols) {
+        TileAcc<kNT> T0;
+        tile_mma<FMT, kNT>(h, st, jj, 0, rt0, tk, zaddr, T0);
+        tile_epi<FMT, kNT>(h, st, jj, 0, rt0, tk, T0, acc);
     }
 }
 
@@ -842,24 +828,20 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 #pragma unroll
             for (int tk = 0; tk < MT; ++tk) {
                 if (tk >= ntok) break;
-                // one-token items have the registers to keep two tiles of MMA sums
-                // in flight (Q3_K's second code plane does not fit them)
-                constexpr bool kPair = false;
                 if (fmt == kQ80) {
-                    for (int jj = wcol; jj < ks; jj += kCols) {
+                    for (int jj = wcol; jj < ks; jj += kCols) {   // both halves of each superblock's code pairs
                         TileAcc<kNT> T0, T1;
                         tile_mma<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, zaddr, T0);
-                        if (!kPair) tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
+                        tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
                         tile_mma<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, zaddr, T1);
-                        if (kPair) tile_epi<kQ80, kNT>(GS, stage, jj, 0, rt0, tk, T0, cur[tk]);
                         tile_epi<kQ80, kNT>(GS, stage, jj, 1, rt0, tk, T1, cur[tk]);
                     }
                 } else if (fmt == kQ2K) {
-                    tile_pairs<kQ2K, kPair>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_cols<kQ2K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 } else if (fmt == kQ3K) {
-                    tile_pairs<kQ3K, false>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_cols<kQ3K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 } else {
-                    tile_pairs<kQ4K, kPair>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
+                    tile_cols<kQ4K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 }
             }
             // fields needed after the slot is released to the producer
