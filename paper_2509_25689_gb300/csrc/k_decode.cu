@@ -120,6 +120,15 @@ __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
                  ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ void bulk_copy_hint(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar, uint64_t pol) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(pol) : "memory");
+}
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
@@ -641,6 +650,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi}
                                 : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
         int p_cursor = 0, p_q = 0;
+        // weights are read once per call: evict-first in L2, so they do not
+        // displace the activations, h and partial outputs the kernels share
+        const uint64_t wpol = evict_first_policy();
         const int p_nsb = vs.nsb;
         ItemDesc P;
         int pslot = 0;
@@ -780,7 +792,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 __syncwarp();
                 // weight planes (lanes 0..3) first; the down kernel's first copy
                 // of h waits for the gate/up kernel, while its weights stream
-                if (bytes && lane < 4) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
+                if (bytes && lane < 4) bulk_copy_hint(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full, wpol);
                 if (!deps) { pdl_wait(); deps = true; }
                 if (bytes && lane >= 4) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
                 ++p_q;
