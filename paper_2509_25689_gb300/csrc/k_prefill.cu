@@ -28,7 +28,14 @@
 namespace mq {
 namespace {
 
-constexpr int kPThreads = 256;                 // 8 warps: two per TMEM lane quarter
+constexpr int kPWorkers = 256;                 // 8 worker warps: two per TMEM lane quarter
+constexpr int kMmaWarp = kPWorkers / 32;       // the down GEMM: + one warp that issues the MMAs
+// The gate/up GEMM keeps the MMA issue in worker thread 0: at 9 warps a
+// thread gets at most 168 registers, and its two tensors' prefetched fields
+// spill there (2.57 -> 2.83 ms measured), while the down GEMM gains (1.97 ->
+// 1.72 ms).
+__host__ __device__ constexpr bool mma_warp(bool down) { return down; }
+__host__ __device__ constexpr int prefill_threads(bool down) { return kPWorkers + (mma_warp(down) ? 32 : 0); }
 constexpr int kMT = 128;                       // weight rows per unit (MMA M)
 constexpr int kNT = 256;                       // tokens per unit (largest MMA N)
 constexpr int kKC = 64;                        // K per ring slot
@@ -73,6 +80,17 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
         if (mbar_try(bar, parity)) return true;
         if (global_ns() - t0 > 1000000000ull) return false;
     }
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// barrier 1 over the worker warps only (the MMA warp runs its own loop)
+__device__ __forceinline__ void workers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kPWorkers) : "memory"); }
+__device__ __forceinline__ bool workers_any(bool v) {
+    uint32_t r;
+    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.or.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+                 : "=r"(r) : "r"((uint32_t)v), "n"(kPWorkers) : "memory");
+    return r != 0;
 }
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
     return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
@@ -327,15 +345,19 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, i
 __device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
 
 template <bool kDown>
-__global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_constant__ ExpertTab tab,
-                                                               const __grid_constant__ PrefillArgs A) {
+__global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(const __grid_constant__ ExpertTab tab,
+                                                                            const __grid_constant__ PrefillArgs A) {
+    constexpr bool kWS = mma_warp(kDown);
+    constexpr int kPThreads = prefill_threads(kDown);
     pdl_wait();
     pdl_launch();
     extern __shared__ __align__(1024) uint8_t smem[];
     __shared__ PSlots sl;
     __shared__ int32_t s_row[kNT], s_asg[kNT];
     __shared__ float s_w[kNT];
-    __shared__ __align__(8) uint64_t bars[kPSlots];
+    __shared__ __align__(8) uint64_t bars[kPSlots];   // the MMAs of the slot's chunk are done
+    __shared__ __align__(8) uint64_t fbar[kPSlots];   // the slot's chunk is in shared memory (every worker)
+    __shared__ int s_info[kPSlots];                   // that chunk: N rounded to 16 | accumulate << 16, or -1 = end
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
     __shared__ int s_unit;
@@ -363,9 +385,12 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         for (int i = 0; i < n_slots; ++i) { sl.pre[i] = run; run += n_mt * ((sl.ntot[i] + kNT - 1) / kNT); }
         sl.pre[n_slots] = run;
         s_fail = 0;
-        for (int i = 0; i < kPSlots; ++i)
+        for (int i = 0; i < kPSlots; ++i) {
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"((uint32_t)__cvta_generic_to_shared(&bars[i]))
                          : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;"
+                         ::"r"((uint32_t)__cvta_generic_to_shared(&fbar[i])), "n"(kPWorkers) : "memory");
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     constexpr int kCols = kDown ? 256 : 512;
@@ -380,10 +405,47 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
     const uint32_t tbase = s_tmem;
     const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
+    const uint32_t fbar0 = (uint32_t)__cvta_generic_to_shared(fbar);
     const int n_units = sl.pre[n_slots];
     const int nC = K / kKC;
-    int gchunk = 0;        // chunks issued by this CTA so far (ring position and parities)
-    int last_committed = -1;
+    // the MMAs of the chunk in ring slot s (info: N rounded to 16 | accumulate << 16),
+    // committed to the slot's barrier, which frees the slot
+    auto issue_chunk = [&](int s, int info) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t idesc = idesc_f16(kMT, info & 0xffff);
+        const uint32_t sbase = ring + s * kSlotBytes, bsm = sbase + 2 * kABytes;
+#pragma unroll
+        for (int ks = 0; ks < kKC / 16; ++ks) {
+            const uint32_t acc = ((info >> 16) != 0 || ks > 0) ? 1u : 0u;
+            const uint64_t db = sdesc(bsm + 2 * ks * kNT * 16, kNT * 16, 128);
+            mma_f16(tbase, sdesc(sbase + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
+            if (!kDown) mma_f16(tbase + kNT, sdesc(sbase + kABytes + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
+        }
+        asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                     ::"r"(bar0 + 8 * s) : "memory");
+    };
+
+    if (kWS && warp == kMmaWarp) {
+        // ---- MMA issue: the CTA's chunk g sits in ring slot g % kPSlots once
+        // every worker has arrived on its full barrier; one lane issues its
+        // MMAs and commits them to the slot's barrier (which frees the slot)
+        int last = -1;
+        bool ok = true;
+        for (int g = 0;; ++g) {
+            const int s = g % kPSlots;
+            if (!mbar_wait(fbar0 + 8 * s, (g / kPSlots) & 1)) { ok = false; break; }
+            const int info = s_info[s];
+            if (info < 0) break;
+            if (lane == 0) issue_chunk(s, info);
+            __syncwarp();
+            last = g;
+        }
+        if (!ok && lane == 0) { atomicOr(A.err, kErrMma); s_fail = 1; }
+        // tensor memory is released only after the MMAs issued here are done
+        if (last >= 0) mbar_wait(bar0 + 8 * (last % kPSlots), (last / kPSlots) & 1);
+    } else {
+    int gchunk = 0;        // chunks posted by this CTA so far (ring position and parities)
+    int last_committed = -1;   // without the MMA warp: the last chunk thread 0 committed
     bool failed = false;
     int cursor = 0;
 
@@ -391,7 +453,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
     // number of tokens of the expert, up to 16x between full and small tiles)
     for (;;) {
         if (tid == 0) s_unit = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
-        __syncthreads();
+        workers_sync();
         const int u = s_unit;
         if (u >= n_units || failed) break;
         while (cursor + 1 < n_slots && sl.pre[cursor + 1] <= u) ++cursor;
@@ -400,7 +462,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         const int n0 = tt * kNT, N = min(kNT, sl.ntot[p] - n0), Npad = (N + 15) & ~15;
         const bool shared = p < d.has_shared;
         // the unit's activation rows, assignments and weights
-        for (int n = tid; n < kNT; n += kPThreads) {
+        for (int n = tid; n < kNT; n += kPWorkers) {
             int a = -1, row = 0;
             float w = 0.0f;
             if (n < N) {
@@ -420,7 +482,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         const int64_t R = (int64_t)mt * kMT + rr;
         const RowPtrs RP0 = row_ptrs(f0, b0, L0, R);
         const RowPtrs RP1 = kDown ? RP0 : row_ptrs(f1, b1, L1, R);
-        __syncthreads();
+        workers_sync();
         // B gather: this thread always moves the 16-byte piece kc = tid % 8 of
         // rows n = tid / 8 + 32 j; the row pointers are fixed for the unit
         const __half* src = kDown ? A.h16 : A.x16;
@@ -464,7 +526,9 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
             }
         }
         // one 64-wide chunk: gather the next chunk's rows, decode this one's
-        // weights, then thread 0 issues its MMAs
+        // weights, then post the chunk to the MMA warp (no block barrier: the
+        // workers run ahead up to the ring's depth) or, without it, meet at a
+        // barrier after which thread 0 issues the chunk's MMAs
         auto chunk_body = [&](int c, const Packed& Q0, const Packed& Q1) -> bool {
             const int g = gchunk + c, s = g % kPSlots;
             bool bad = false;
@@ -479,22 +543,18 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
             dequant_store(f0, Q0, c, hf, sbase + rr * 16);
             if (!kDown) dequant_store(f1, Q1, c, hf, sbase + kABytes + rr * 16);
             asm volatile("cp.async.wait_group 1;" ::: "memory");
+            // this thread's shared-memory writes (and landed copies) before the
+            // tensor cores read them
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            if (__syncthreads_or(bad)) return false;
-            if (tid == 0) {
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const uint32_t idesc = idesc_f16(kMT, Npad);
-                const uint32_t bsm = sbase + 2 * kABytes;
-#pragma unroll
-                for (int ks = 0; ks < kKC / 16; ++ks) {
-                    const uint32_t acc = (c > 0 || ks > 0) ? 1u : 0u;
-                    const uint64_t db = sdesc(bsm + 2 * ks * kNT * 16, kNT * 16, 128);
-                    mma_f16(tbase, sdesc(sbase + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
-                    if (!kDown) mma_f16(tbase + kNT, sdesc(sbase + kABytes + 2 * ks * kMT * 16, kMT * 16, 128), db, idesc, acc);
-                }
-                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-                             ::"r"(bar0 + 8 * s) : "memory");
+            const int info = Npad | (c > 0 ? 1 << 16 : 0);
+            if (kWS) {
+                if (tid == 0) s_info[s] = info;
+                mbar_arrive(fbar0 + 8 * s);
+                if (bad) s_fail = 1;   // checked by all workers at the unit's end
+                return true;
             }
+            if (workers_any(bad)) return false;
+            if (tid == 0) issue_chunk(s, info);
             last_committed = g;
             return true;
         };
@@ -554,7 +614,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
         // all MMAs of the unit are done once the last chunk's commit arrived
         const int glast = gchunk + nC - 1;
         const bool ok = mbar_wait(bar0 + 8 * (glast % kPSlots), (glast / kPSlots) & 1);
-        if (__syncthreads_or(!ok)) { failed = true; break; }
+        if (workers_any(!ok || s_fail)) { failed = true; break; }
         gchunk += nC;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         // epilogue: TMEM lane 32 warp + lane = weight row, columns = tokens
@@ -584,16 +644,25 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_kernel(const __grid_cons
                 }
             }
         }
+        // the accumulators are read: the next unit's MMAs (posted after this
+        // point by every worker) may overwrite them
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        workers_sync();
     }
-    if (failed && tid == 0) { atomicOr(A.err, kErrMma); s_fail = 1; }
-    __syncthreads();
-    if (s_fail && last_committed >= 0) {
+    if (failed) {
+        if (tid == 0) { atomicOr(A.err, kErrMma); s_fail = 1; }
         // wait (bounded) for the MMAs still in flight before giving TMEM back
-        mbar_wait(bar0 + 8 * (last_committed % kPSlots), (last_committed / kPSlots) & 1);
+        if (!kWS && last_committed >= 0)
+            mbar_wait(bar0 + 8 * (last_committed % kPSlots), (last_committed / kPSlots) & 1);
+    } else if (kWS) {
+        // end marker for the MMA warp in the next chunk's slot (every earlier
+        // chunk's MMAs are done, so the warp has read every earlier marker)
+        const int s = gchunk % kPSlots;
+        if (tid == 0) s_info[s] = -1;
+        mbar_arrive(fbar0 + 8 * s);
     }
+    }   // workers
+    __syncthreads();
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (warp == 0) {
@@ -623,11 +692,11 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     A.x16 = w.x16; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
     A.next = w.counters;
     prof_begin("gateup_tc", s);
-    cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(kPThreads), smem, s, tab, A);
+    cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(prefill_threads(false)), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     prof_begin("down_tc", s);
-    err = launch_pdl(prefill_kernel<true>, dim3(g_psms), dim3(kPThreads), smem, s, tab, A);
+    err = launch_pdl(prefill_kernel<true>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);
