@@ -34,22 +34,6 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 
-__device__ __forceinline__ uint32_t lop3_and_or(uint32_t a, uint32_t mask, uint32_t orv) {
-    uint32_t d;
-    asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(d) : "r"(a), "r"(mask), "r"(orv));   // (a & b) | c
-    return d;
-}
-// Q8_0: byte u -> fp16 1024 + (u ^ 0x80) in each half: M ? (a ^ K) : K
-__device__ __forceinline__ uint32_t lop3_q8(uint32_t a) {
-    uint32_t d;
-    asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(d) : "r"(a), "r"(0x00FF00FFu), "r"(0x64806480u));
-    return d;
-}
-__device__ __forceinline__ uint32_t hmul2u(uint32_t a, uint32_t b) {
-    __half2 x = *reinterpret_cast<__half2*>(&a), y = *reinterpret_cast<__half2*>(&b);
-    __half2 z = __hmul2(x, y);
-    return *reinterpret_cast<uint32_t*>(&z);
-}
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                          uint32_t b0, uint32_t b1) {
     asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
@@ -57,23 +41,7 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint4 ldg128(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
-__device__ __forceinline__ uint2 ldg64(const void* p) { return __ldg(reinterpret_cast<const uint2*>(p)); }
-__device__ __forceinline__ uint32_t ldg32(const void* p) { return __ldg(reinterpret_cast<const unsigned int*>(p)); }
-__device__ __forceinline__ uint32_t ldg16(const void* p) { return __ldg(reinterpret_cast<const unsigned short*>(p)); }
 __device__ __forceinline__ float h2f(uint32_t bits16) { return __half2float(__ushort_as_half((unsigned short)bits16)); }
-
-// 2-bit code pair at position p of word w as fp16x2 "1024 + 4^pos q"
-template <int P>
-__device__ __forceinline__ uint32_t ext2(uint32_t w, uint32_t w10) {
-    constexpr int pos = P <= 4 ? P : P - 5;
-    return lop3_and_or(P <= 4 ? w : w10, 0x00030003u << (2 * pos), 0x64006400u);
-}
-template <int P1>
-__device__ __forceinline__ uint32_t ext1(uint32_t w, uint32_t w10) {
-    constexpr int pos = P1 <= 9 ? P1 : P1 - 10;
-    return lop3_and_or(P1 <= 9 ? w : w10, 0x00010001u << pos, 0x64006400u);
-}
 
 struct VecSrc {
     const __half* q;     // prepared fp16 fragments of vector 0
