@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
                                                                   int E, float* __restrict__ z,
                                                                   __half* __restrict__ x16,
                                                                   uint32_t* __restrict__ zero_words, int n_zero) {
-    __shared__ float part[32][kTokT];
+    __shared__ float part[8][kEB][kTokT];   // per segment (warp): each expert's sums of the CTA's tokens
     const int e0 = blockIdx.x * kEB, t0 = blockIdx.y * kTokT;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
@@ -173,9 +173,18 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
                 *reinterpret_cast<uint2*>(x16 + (size_t)(t0 + j) * H + (c0 + c) * 128 + 4 * lane) = hv;
             }
         }
+    // expert el's weights in wv, expert el + 1's loading into wn while el is
+    // reduced; the per-warp sums of all 16 experts wait in shared memory and
+    // the segments are added once at the end
     for (int el = 0; el < kEB; ++el) {
         const int e = e0 + el;
         if (e >= E) break;
+        float4 wn[8] = {};
+        if (e + 1 < E && el + 1 < kEB) {
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                if (c < nc) wn[c] = __ldg(reinterpret_cast<const float4*>(W + (size_t)(e + 1) * H + (c0 + c) * 128 + 4 * lane));
+        }
         float acc[kTokT];
 #pragma unroll
         for (int j = 0; j < kTokT; ++j) {
@@ -190,12 +199,6 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
                 }
             }
         }
-        // the next expert's weights, loaded while this one's sums are reduced
-        if (e + 1 < E && el + 1 < kEB) {
-#pragma unroll
-            for (int c = 0; c < 8; ++c)
-                if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(W + (size_t)(e + 1) * H + (c0 + c) * 128 + 4 * lane));
-        }
 #pragma unroll
         for (int j = 0; j < kTokT; ++j) {
 #pragma unroll
@@ -203,18 +206,20 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
         }
         if (lane == 0) {
 #pragma unroll
-            for (int j = 0; j < kTokT; ++j) part[seg][j] = acc[j];
+            for (int j = 0; j < kTokT; ++j) part[seg][el][j] = acc[j];
         }
-        __syncthreads();
-        if (threadIdx.x < kTokT) {
-            const int t = t0 + threadIdx.x;
-            if (t < T) {
-                float r = part[0][threadIdx.x];
-                for (int s2 = 1; s2 < nseg; ++s2) r = __fadd_rn(r, part[s2][threadIdx.x]);
-                z[(size_t)t * E + e] = r;
-            }
+#pragma unroll
+        for (int c = 0; c < 8; ++c) wv[c] = wn[c];
+    }
+    __syncthreads();
+    // segments left to right, per (expert, token) of the CTA
+    for (int o = threadIdx.x; o < kEB * kTokT; o += blockDim.x) {
+        const int el = o / kTokT, j = o % kTokT, e = e0 + el, t = t0 + j;
+        if (e < E && t < T) {
+            float r = part[0][el][j];
+            for (int s2 = 1; s2 < nseg; ++s2) r = __fadd_rn(r, part[s2][el][j]);
+            z[(size_t)t * E + e] = r;
         }
-        __syncthreads();
     }
 }
 
