@@ -117,6 +117,20 @@ def test_forward_tiny_layer(torch_cuda, orc, decode_kernel):
     assert_close(y, ry)
 
 
+def test_forward_tiny_layer_one_token_no_shared(torch_cuda, orc, decode_kernel):
+    """One token and no shared expert: the one-warp routing path (no block-wide
+    sort) and the one-token FFN kernels with routed slots only."""
+    spec = get_config("tiny")
+    assert not spec.has_shared
+    layer = DeviceLayer(spec, 0, orc=orc)
+    x = tokens(spec, 0, 1)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    assert_close(y, ry)
+
+
 @pytest.mark.parametrize("T", [1, 3, 5, 9])
 def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T, decode_kernel):
     spec = LayerSpec(name="small_mixed", hidden=512, inter=256, n_experts=12, n_groups=4, topk_group=2,
