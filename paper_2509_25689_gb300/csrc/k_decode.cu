@@ -13,14 +13,16 @@
 //     per lane so nothing is masked in the loop;
 //   D (16 rows x 8 cols) = per-(row, sub-block) partial dot products, so the
 //     sub-block scales and mins are applied once per tile in fp32.
-// Work is cut into items (32 rows x all superblocks of one tensor (gate and
-// up together) of one expert x up to 4 tokens); CTA c of the persistent grid
-// (one CTA per SM) takes items c, c + grid, ...  The packed layout keeps any
-// superblock range of a 32-row tile contiguous in every plane, so a
-// dedicated producer warp streams each item through a 3-slot shared-memory
-// ring with 1D bulk (TMA) copies that complete on mbarriers; 8 consumer warps
-// (all 32 rows x every 8th superblock of a stage each) run the tensor-core
-// math.  At the end of an item the CTA reduces its warps' sums in a fixed
+// Work is cut into items (gate/up: 32 rows x all superblocks of gate and of
+// up; down: two 32-row blocks x all superblocks; of one expert x up to 4
+// tokens), claimed by the persistent CTAs (one per SM) from a per-call
+// counter.  The packed layout keeps any superblock range of a 32-row tile
+// contiguous in every plane, so a dedicated producer warp streams each item
+// through a shared-memory ring (3 x 64 KB for gate/up, 4 x 48 KB for down)
+// with 1D bulk (TMA) copies that complete on mbarriers; 8 consumer warps (all
+// 32 rows x every 8th superblock of a stage each, the columns rotated from
+// stage to stage) run the tensor-core math.  At the end of an item the CTA
+// reduces its warps' sums in a fixed
 // order (SwiGLU and the prepared h for gate/up, one partial output row block
 // per assignment for down), so results are deterministic.  Every wait on an
 // mbarrier is bounded (about 1 s) and reports to an error word.
@@ -610,11 +612,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 
     if (warp == kProducerWarp) {
         // ===================== producer (dedicated warp) =====================
-        // The CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...  Per
-        // phase (one tensor of one item) every lane owns at most one copy:
-        // lanes 0..3 a weight plane, lanes 4.. one piece of one token (family
-        // fragments or statistics).  A stage then only
-        // advances the source by the stage's first superblock.
+        // The CTA claims items from the per-call counter.  Per phase (one
+        // tensor, or one 32-row block of down, of one item) every lane owns at
+        // most one copy: lanes 0..3 a weight plane, lanes 4.. one piece of one
+        // token (family fragments or statistics).  A stage then only advances
+        // the source by the stage's first superblock.
         const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi}
                                 : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
         int p_cursor = 0, p_q = 0;
