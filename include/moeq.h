@@ -197,7 +197,10 @@ const char* mq_strerror(int status);
  * GEMM, else decode GEMV), 1 = force decode, 2 = force prefill, 3 = force
  * decode on the alternative tcgen05 GEMV kernels (A operand in tensor
  * memory; slower than the default mma.sync GEMV at decode sizes, kept as a
- * second implementation).  Process wide; the MQ_FORCE_PATH environment
+ * second implementation).  Decode on a layer whose hidden or intermediate
+ * size is not a multiple of 256 always takes the tcgen05 GEMV kernels (the
+ * mma.sync kernels stream whole 256-element superblocks).  Process wide; the
+ * MQ_FORCE_PATH environment
  * variable ("decode"/"prefill"/"decode_tc") sets the initial value.
  * threshold <= 0 keeps the current one (default 64).  Returns MQ_EINVAL for
  * another mode. */

@@ -34,6 +34,13 @@ int path_mode() {
     return g_path_mode;
 }
 
+}  // namespace
+
+// the mma.sync decode kernels (k_decode.cu) stream whole 256-element superblocks
+bool decode_mma_fits(const Dims& d) { return d.H % 256 == 0 && d.I % 256 == 0; }
+
+namespace {
+
 int check_cfg(const mq_layer_cfg* c) {
     if (!c) return MQ_EINVAL;
     if (c->hidden < 128 || c->hidden % 128 || c->hidden > 32768) return MQ_ESHAPE;
@@ -249,7 +256,7 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     if (topk_w) w.wts = topk_w;
     const int pm = path_mode();
     const bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
-    const bool tc = !prefill && pm == 3 && decode_tc_fits(d);
+    const bool tc = !prefill && decode_tc_fits(d) && (pm == 3 || !decode_mma_fits(d));
     rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1);
     if (rc != MQ_OK) return rc;
     if (prefill) {

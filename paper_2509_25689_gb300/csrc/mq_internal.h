@@ -117,6 +117,10 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 // tcgen05 decode kernels: need hidden and inter to be multiples of 128
 bool decode_tc_fits(const Dims& d);
+// mma.sync decode kernels: stream whole 256-element superblocks of every
+// format (a Q8_0 stage holds 8 blocks of 32 per superblock), so hidden and
+// inter must be multiples of 256; other shapes take the tcgen05 decode kernels
+bool decode_mma_fits(const Dims& d);
 cudaError_t launch_decode_tc(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s);
 size_t decode_counter_bytes(const Dims& d);
 cudaError_t launch_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float* dst, cudaStream_t s);

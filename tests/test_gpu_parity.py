@@ -1,6 +1,8 @@
 """GPU parity: the CUDA path through the C ABI vs the oracle on the same
 seeded inputs.  Bit-exact for unpacked weights, expert ids, routing weights
 and the permutation; max |err| <= 2e-3 * max|y| for the layer output."""
+from dataclasses import replace
+
 import numpy as np
 import pytest
 
@@ -83,6 +85,59 @@ def test_routing_bit_exact(torch_cuda, orc, name, T):
     np.testing.assert_array_equal(off, roff)
     np.testing.assert_array_equal(perm, rperm)
     np.testing.assert_array_equal(inv, rinv)
+
+
+MAX_ROUTER = LayerSpec(name="max_router", hidden=256, inter=256, n_experts=256, n_groups=64, topk_group=16,
+                       top_k=32, tokens=1, has_shared=True, mixed=True, router_std=1 / 16, bias_std=0.01)
+
+
+@pytest.mark.parametrize("T", [1, 3, 300])
+def test_routing_bit_exact_largest_shapes(torch_cuda, orc, T):
+    """256 experts, 64 groups of 4, top-32: every lane holds a selection in
+    the one-token path, the group scan takes its lane-per-group form, and
+    T = 300 goes through the separate top-k and permutation kernels."""
+    spec = replace(MAX_ROUTER, tokens=T)
+    lay = _RouterOnly(spec, 2)
+    x = tokens(spec, 2, T)
+    idx, w, off, perm, inv = _route(torch_cuda, lay, x)
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group, spec.top_k,
+                           spec.routed_scale, spec.has_shared)
+    ridx, rw, _, _ = orc.route(layer, x, lay.router_w_host, lay.bias_host)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    roff, rperm, rinv = orc.permute(ridx, spec.n_experts)
+    np.testing.assert_array_equal(off, roff)
+    np.testing.assert_array_equal(perm, rperm)
+    np.testing.assert_array_equal(inv, rinv)
+
+
+@pytest.mark.parametrize("T", [1, 3])
+def test_forward_largest_routing_shapes(torch_cuda, orc, T, decode_kernel):
+    """Top-32 of 256 mixed-format experts plus the shared one: 33 slots per
+    token through the decode kernels."""
+    spec = replace(MAX_ROUTER, tokens=T)
+    layer = DeviceLayer(spec, 5)
+    x = tokens(spec, 5, T)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x, idx_hint=idx)
+    np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
+
+
+@pytest.mark.parametrize("T", [1, 3])
+def test_forward_sizes_not_multiple_of_256(torch_cuda, orc, T, decode_kernel):
+    """Hidden 384 and inter 128 (multiples of 128 only) with every format,
+    Q8_0 included: these shapes always take the tcgen05 decode kernels (the
+    mma.sync ones stream whole 256-element superblocks)."""
+    spec = LayerSpec(name="odd_sizes", hidden=384, inter=128, n_experts=12, n_groups=4, topk_group=2, top_k=3,
+                     tokens=T, has_shared=True, mixed=True, router_std=1 / 19.6, bias_std=0.01)
+    fm = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
+    layer = DeviceLayer(spec, T, fmts=fm)
+    x = tokens(spec, T)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
 
 
 def test_routing_tie_break_on_device(torch_cuda, orc):
