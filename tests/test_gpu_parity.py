@@ -111,6 +111,26 @@ def test_routing_bit_exact_largest_shapes(torch_cuda, orc, T):
     np.testing.assert_array_equal(inv, rinv)
 
 
+@pytest.mark.parametrize("T", [1, 40])
+def test_routing_bit_exact_largest_hidden(torch_cuda, orc, T):
+    """Hidden 32768 (the largest accepted): 32 segments of 1024 per logit, so
+    the per-expert logits kernel runs with 32 warps, also for 40 tokens (the
+    tiled kernel takes at most 8 segments)."""
+    spec = LayerSpec(name="wide_router", hidden=32768, inter=128, n_experts=16, n_groups=4, topk_group=2,
+                     top_k=4, tokens=T, has_shared=False, router_std=1 / 181.0, bias_std=0.01)
+    lay = _RouterOnly(spec, 3)
+    x = tokens(spec, 3, T)
+    idx, w, off, perm, inv = _route(torch_cuda, lay, x)
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group, spec.top_k,
+                           spec.routed_scale, spec.has_shared)
+    ridx, rw, _, _ = orc.route(layer, x, lay.router_w_host, lay.bias_host)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    roff, rperm, rinv = orc.permute(ridx, spec.n_experts)
+    np.testing.assert_array_equal(off, roff)
+    np.testing.assert_array_equal(perm, rperm)
+
+
 @pytest.mark.parametrize("T", [1, 3])
 def test_forward_largest_routing_shapes(torch_cuda, orc, T, decode_kernel):
     """Top-32 of 256 mixed-format experts plus the shared one: 33 slots per
