@@ -107,3 +107,31 @@ def test_pointer_and_workspace_checks(mq):
 def test_strerror(mq):
     assert mq.mq_strerror(0) == "ok"
     assert "workspace" in mq.mq_strerror(-5)
+
+
+@pytest.mark.parametrize("fmt", [1, 2, 3, 4])
+def test_generator_sizes_match_library_and_oracle(mq, orc, fmt):
+    # the input generators and bench.py's byte accounting size packed tensors
+    # themselves; they must agree with both codecs
+    from workloads.configs import packed_bytes
+    for rows, cols in [(1, 32), (31, 256), (33, 257), (128, 2048), (2048, 7168), (7168, 2048), (96, 8192)]:
+        n = packed_bytes(fmt, rows, cols)
+        assert n == mq.mq_packed_size(fmt, rows, cols) == orc.packed_size(fmt, rows, cols), (rows, cols)
+
+
+def test_bench_step_bytes_counts_each_touched_expert_once(mq):
+    import bench
+    from workloads.configs import get_config
+    spec = get_config("v3_decode_t1")
+    E, H, I, K = spec.n_experts, spec.hidden, spec.inter, spec.top_k
+    fmts = np.tile(np.array([[1, 1, 2]], np.uint8), (E + 1, 1))
+    fmts[E] = 4
+    idx = np.array([[3, 7, 7, 11, 0, 190, 191, 3]], np.int32)   # 6 distinct experts
+    b = bench.step_bytes(spec, fmts, [idx])[0]
+    gu = 2 * mq.mq_packed_size(1, I, H)
+    dn = mq.mq_packed_size(2, H, I)
+    sh = 2 * mq.mq_packed_size(4, I, H) + mq.mq_packed_size(4, H, I)
+    assert b["quantized"] == 6 * (gu + dn) + sh
+    assert b["gateup_mma"] == 6 * gu + 2 * mq.mq_packed_size(4, I, H) + H * 2 + (K + 1) * I * 4
+    assert b["down_mma"] == 6 * dn + mq.mq_packed_size(4, H, I) + (K + 1) * I * 4 + H * 4
+    assert b["router_logits"] == E * H * 4 + H * 2 + E * 4
