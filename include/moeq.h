@@ -199,11 +199,10 @@ const char* mq_strerror(int status);
  * memory; slower than the default mma.sync GEMV at decode sizes, kept as a
  * second implementation).  Decode on a layer whose hidden or intermediate
  * size is not a multiple of 256 always takes the tcgen05 GEMV kernels (the
- * mma.sync kernels stream whole 256-element superblocks).  Process wide; the
- * MQ_FORCE_PATH environment
- * variable ("decode"/"prefill"/"decode_tc") sets the initial value.
- * threshold <= 0 keeps the current one (default 64).  Returns MQ_EINVAL for
- * another mode. */
+ * mma.sync kernels stream whole 256-element superblocks).  Process wide;
+ * the MQ_FORCE_PATH environment variable ("decode"/"prefill"/"decode_tc")
+ * sets the initial value.  threshold <= 0 keeps the current one (default
+ * 64).  Returns MQ_EINVAL for another mode. */
 int mq_set_path(int mode, int32_t prefill_threshold);
 
 /* Kernel timing for measurement tools.  mq_profile_enable(n) makes the next
