@@ -131,19 +131,35 @@ def mq_pack(fmt, w, dst=None):
     n = mq_packed_size(fmt, rows, cols)
     if dst is None:
         dst = np.empty(n, np.uint8)
-    _check("mq_pack", _lib.mq_pack(_fmt(fmt), w.ctypes.data, rows, cols, _ptr(dst), n))
+    _check("mq_pack", _lib.mq_pack(_fmt(fmt), w.ctypes.data, rows, cols, _ptr(dst), _nbytes(dst)))
     return dst
+
+
+def _nbytes(a) -> int:
+    if hasattr(a, "element_size"):
+        return a.numel() * a.element_size()
+    return a.nbytes
+
+
+def _need(fn, a, n):
+    """The C entry points take no source/destination sizes: refuse buffers
+    smaller than the tensor they describe before passing their pointers."""
+    if a is not None and not isinstance(a, int) and _nbytes(a) < n:
+        raise MoeqError(fn, MQ_EINVAL)
 
 
 def mq_unpack(fmt, src, rows: int, cols: int):
     import numpy as np
     src = np.ascontiguousarray(src, dtype=np.uint8)
+    _need("mq_unpack", src, mq_packed_size(fmt, rows, cols))
     out = np.empty((rows, cols), np.float32)
     _check("mq_unpack", _lib.mq_unpack(_fmt(fmt), src.ctypes.data, rows, cols, out.ctypes.data))
     return out
 
 
 def mq_unpack_device(fmt, src, rows: int, cols: int, dst, stream=None):
+    _need("mq_unpack_device", src, mq_packed_size(fmt, rows, cols))
+    _need("mq_unpack_device", dst, 4 * max(rows, 0) * max(cols, 0))
     _check("mq_unpack_device",
            _lib.mq_unpack_device(_fmt(fmt), _ptr(src), rows, cols, _ptr(dst), _stream(stream)))
     return dst

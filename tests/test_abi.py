@@ -135,3 +135,14 @@ def test_bench_step_bytes_counts_each_touched_expert_once(mq):
     assert b["gateup_mma"] == 6 * gu + 2 * mq.mq_packed_size(4, I, H) + H * 2 + (K + 1) * I * 4
     assert b["down_mma"] == 6 * dn + mq.mq_packed_size(4, H, I) + (K + 1) * I * 4 + H * 4
     assert b["router_logits"] == E * H * 4 + H * 2 + E * 4
+
+
+def test_binding_refuses_short_buffers(mq):
+    w = np.zeros((4, 256), np.float32)
+    n = mq.mq_packed_size("Q4_K", 4, 256)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_pack("Q4_K", w, dst=np.empty(n - 1, np.uint8))
+    p = mq.mq_pack("Q4_K", w)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_unpack("Q4_K", p[: n - 16], 4, 256)
+    np.testing.assert_array_equal(mq.mq_unpack("Q4_K", p, 4, 256), w)
