@@ -206,16 +206,47 @@ def test_forward_tiny_layer_one_token_no_shared(torch_cuda, orc, decode_kernel):
     assert_close(y, ry)
 
 
-@pytest.mark.parametrize("T", [1, 3, 5, 9])
+SMALL_MIXED = LayerSpec(name="small_mixed", hidden=512, inter=256, n_experts=12, n_groups=4, topk_group=2,
+                        top_k=3, tokens=1, has_shared=True, mixed=True, router_std=1 / 22.6, bias_std=0.01)
+SMALL_MIXED_FMTS = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
+
+
+@pytest.mark.parametrize("T", [1, 3, 5, 9, 40, 63])
 def test_forward_small_mixed_layer_with_shared(torch_cuda, orc, T, decode_kernel):
-    spec = LayerSpec(name="small_mixed", hidden=512, inter=256, n_experts=12, n_groups=4, topk_group=2,
-                     top_k=3, tokens=T, has_shared=True, mixed=True, router_std=1 / 22.6, bias_std=0.01)
-    fm = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
-    layer = DeviceLayer(spec, T, fmts=fm)
+    spec = replace(SMALL_MIXED, tokens=T)
+    layer = DeviceLayer(spec, T, fmts=SMALL_MIXED_FMTS)
     x = tokens(spec, T)
     y, idx, w = layer.forward(x)
     ry, ridx, rw = layer.oracle_forward(orc, x)
     np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
+
+
+@pytest.mark.parametrize("T", [1, 6])
+def test_forward_routed_scale(torch_cuda, orc, T, decode_kernel):
+    """routed_scale != 1 (Sec. 3.2 weights scaled after normalisation): the
+    weights stay bit-exact and the output follows them."""
+    spec = replace(SMALL_MIXED, tokens=T, routed_scale=2.5)
+    layer = DeviceLayer(spec, 11 + T, fmts=SMALL_MIXED_FMTS)
+    x = tokens(spec, 11 + T)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    assert_close(y, ry)
+
+
+def test_forward_decode_beyond_cached_assignments(torch_cuda, orc, decode_kernel):
+    """2,400 routed assignments on the decode kernels, more than either keeps
+    in shared memory: the rest come from the permutation in global memory."""
+    spec = LayerSpec(name="many_assign", hidden=256, inter=256, n_experts=64, n_groups=8, topk_group=4,
+                     top_k=8, tokens=300, has_shared=True, mixed=True, router_std=1 / 16, bias_std=0.01)
+    layer = DeviceLayer(spec, 5)
+    x = tokens(spec, 5)
+    y, idx, w = layer.forward(x)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
     assert_close(y, ry)
 
 
