@@ -46,12 +46,16 @@ def _peaks():
 
 
 # DRAM traffic per launch of the decode FFN kernels, from the committed ncu
-# summary; reported only while the kernel sources are the ones captured.
+# summary; reported only for the captured workload and only while the kernel
+# sources are the ones captured.
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "ffn_kernel_v3_decode_t1.md")
+PROFILE_WORKLOAD = "v3_decode_t1"
 KERNEL_SOURCES = ("k_decode.cu", "mq_actprep.cuh", "mq_layout.h", "mq_internal.h")
 
 
-def _profiled_traffic(kernel: str):
+def _profiled_traffic(kernel: str, workload: str = PROFILE_WORKLOAD):
+    if workload != PROFILE_WORKLOAD:
+        return None
     import hashlib
     try:
         text = open(PROFILE_SUMMARY).read()
@@ -356,7 +360,7 @@ def run_native(args):
             avg_s = tot_ms / launches / 1e3
             achieved = per_launch_bytes / avg_s / 1e9
             roof = {"bound": "hbm", "kernel": name, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                    "frac": round(achieved / peak, 4), "traffic": _profiled_traffic(name), "peak_source": peak_src,
+                    "frac": round(achieved / peak, 4), "traffic": _profiled_traffic(name, spec.name), "peak_source": peak_src,
                     "algorithmic_bytes_per_launch": int(per_launch_bytes), "avg_launch_us": round(avg_s * 1e6, 2)}
         result = {
             "metric": METRIC, "value": round(job_throughput(world, T, K, dev_ms_max), 2), "unit": "tokens/s",

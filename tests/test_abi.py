@@ -146,3 +146,11 @@ def test_binding_refuses_short_buffers(mq):
     with pytest.raises(mq.MoeqError):
         mq.mq_unpack("Q4_K", p[: n - 16], 4, 256)
     np.testing.assert_array_equal(mq.mq_unpack("Q4_K", p, 4, 256), w)
+
+
+def test_bench_traffic_only_for_the_captured_workload():
+    import bench
+    t = bench._profiled_traffic("gateup_mma")
+    assert t is None or t > 0
+    assert bench._profiled_traffic("gateup_mma", "v3_decode_t1_k6") is None
+    assert bench._profiled_traffic("router_logits") is None

@@ -69,6 +69,7 @@ class _RouterOnly:
 
 
 @pytest.mark.parametrize("name,T", [("tiny", 4), ("tiny", 1), ("v3_decode_t1", 1), ("v3_decode_t1", 7),
+                                    ("v3_decode_t1_k6", 1), ("v3_decode_t1_k6", 5),
                                     ("v3_decode_t32_mixed", 32), ("v3_decode_t32_mixed", 256),
                                     ("v3_decode_t32_mixed", 257), ("v3_prefill_t2048_zipf", 2048)])
 def test_routing_bit_exact(torch_cuda, orc, name, T):
@@ -258,6 +259,20 @@ def test_forward_v3_decode_t1(torch_cuda, orc, decode_kernel):
     ry, ridx, rw = layer.oracle_forward(orc, x, idx_hint=idx)
     np.testing.assert_array_equal(idx, ridx)
     assert_close(y, ry)
+
+
+@pytest.mark.parametrize("T", [1, 5])
+def test_forward_v3_decode_k6(torch_cuda, orc, T, decode_kernel):
+    """The activation-adjusted layer (k = 6 of 192, Sec. 3.2) on the same kernels."""
+    spec = get_config("v3_decode_t1_k6")
+    layer = DeviceLayer(spec, 2)
+    x = tokens(spec, 2, T)
+    y, idx, w = layer.forward(x)
+    for t in sorted({0, T - 1}):
+        ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
+        np.testing.assert_array_equal(idx[t:t + 1], ridx)
+        np.testing.assert_array_equal(w[t:t + 1].view(np.uint32), rw.view(np.uint32))
+        assert_close(y[t:t + 1], ry)
 
 
 def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc, decode_kernel):

@@ -170,6 +170,9 @@ def test_paper_activation_adjustment_and_flops():
     of 192 experts (Sec. 3.2, Sec. 4.1); FLOPs_active = 2 sum k_i P_i."""
     from workloads import activation_adjusted_k, flops_active
     assert activation_adjusted_k(0.75, 8) == 6
+    from workloads import get_config
+    spec = get_config("v3_decode_t1_k6")
+    assert spec.top_k == activation_adjusted_k(spec.n_experts / spec.n_original_experts, 8)
     assert activation_adjusted_k(0.75, 256) == 192
     P = 3 * 7168 * 2048
     assert flops_active([8], [P]) == 2 * 8 * P

@@ -81,6 +81,9 @@ CONFIGS = {
                       quantize_from_fp32=True, n_original_experts=8),
     # 2: one V3-shaped layer at decode, 1 token
     "v3_decode_t1": _v3(name="v3_decode_t1", tokens=1),
+    # 2 with the paper's deployed activation adjustment: k = ceil(r k_orig) =
+    # ceil(0.75 * 8) = 6 experts per token of the 192 kept (Sec. 3.2)
+    "v3_decode_t1_k6": _v3(name="v3_decode_t1_k6", tokens=1, top_k=6),
     # 3: 32 decode tokens, per-tensor formats drawn 50/30/20 from Q2_K/Q3_K/Q4_K
     "v3_decode_t32_mixed": _v3(name="v3_decode_t32_mixed", tokens=32, mixed=True),
     # 4: prefill 2048 tokens, Zipf(1.1)-skewed expert counts, mixed formats
