@@ -43,6 +43,18 @@ class mq_expert_table(ctypes.Structure):
                 ("shared", ctypes.POINTER(mq_expert_weights))]
 
 
+class mq_plan_tensor(ctypes.Structure):
+    _fields_ = [("params", ctypes.c_int64), ("layer", ctypes.c_int32), ("kind", ctypes.c_int32),
+                ("sens", ctypes.c_double)]
+
+
+class mq_plan_cfg(ctypes.Structure):
+    _fields_ = [("n_levels", ctypes.c_int32), ("bits64", ctypes.POINTER(ctypes.c_int32)),
+                ("low", ctypes.c_int32), ("lowest", ctypes.c_int32), ("small_level", ctypes.c_int32),
+                ("medium_level", ctypes.c_int32), ("floor_level", ctypes.c_int32),
+                ("small_max", ctypes.c_int64), ("medium_max", ctypes.c_int64), ("mem_limit_bytes", ctypes.c_int64)]
+
+
 class mq_kernel_stat(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int32), ("total_ms", ctypes.c_double)]
 
@@ -68,6 +80,9 @@ def _load():
         "mq_set_path": (ctypes.c_int, [ctypes.c_int, i32]),
         "mq_profile_enable": (ctypes.c_int, [i32]),
         "mq_profile_collect": (ctypes.c_int, [ctypes.POINTER(mq_kernel_stat), i32]),
+        "mq_plan_precision": (ctypes.c_int, [ctypes.POINTER(mq_plan_cfg), ctypes.POINTER(mq_plan_tensor), i32, vp,
+                                             ctypes.POINTER(ctypes.c_int64)]),
+        "mq_binary_partition_order": (ctypes.c_int, [i32, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -78,7 +93,7 @@ def _load():
 _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
             "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
-            "mq_profile_collect")
+            "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order")
 
 
 def _ptr(a):
@@ -237,3 +252,32 @@ def mq_profile_collect(max_entries: int = 64):
     arr = (mq_kernel_stat * max_entries)()
     n = _lib.mq_profile_collect(arr, max_entries)
     return [(arr[i].name.decode(), int(arr[i].launches), float(arr[i].total_ms)) for i in range(n)]
+
+
+# ------------------------------------------------------------ planner ---
+MQ_TENSOR_OTHER, MQ_TENSOR_EXPERT_GATE, MQ_TENSOR_EXPERT_UP, MQ_TENSOR_EXPERT_DOWN = 0, 1, 2, 3
+
+
+def mq_plan_precision(tensors, bits64, low, lowest, small_level, medium_level, floor_level, small_max, medium_max,
+                      mem_limit_bytes):
+    """tensors: sequence of (params, layer, kind, sens).  Returns (levels as a
+    numpy int32 array, total bits in 1/64-bit units)."""
+    import numpy as np
+    n = len(tensors)
+    arr = (mq_plan_tensor * max(n, 1))()
+    for i, (p, ly, k, s) in enumerate(tensors):
+        arr[i] = mq_plan_tensor(int(p), int(ly), int(k), float(s))
+    b = (ctypes.c_int32 * len(bits64))(*[int(v) for v in bits64])
+    cfg = mq_plan_cfg(len(bits64), b, low, lowest, small_level, medium_level, floor_level, int(small_max),
+                      int(medium_max), int(mem_limit_bytes))
+    out = np.empty(max(n, 1), np.int32)
+    total = ctypes.c_int64(0)
+    _check("mq_plan_precision", _lib.mq_plan_precision(ctypes.byref(cfg), arr, n, out.ctypes.data, ctypes.byref(total)))
+    return out[:n], int(total.value)
+
+
+def mq_binary_partition_order(n: int):
+    import numpy as np
+    out = np.empty(max(n, 1), np.int32)
+    _check("mq_binary_partition_order", _lib.mq_binary_partition_order(n, out.ctypes.data))
+    return out[:n]
