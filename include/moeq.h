@@ -81,7 +81,7 @@ enum {
     MQ_ESHAPE = -4,     /* inconsistent layer shape (see moe_quant_forward) */
     MQ_EWORKSPACE = -5, /* workspace missing or smaller than moe_quant_workspace_size */
     MQ_ECUDA = -6,      /* CUDA launch or runtime error */
-    MQ_EDEVICE = -7,    /* a device-side check reported an error */
+    MQ_EDEVICE = -7,    /* a kernel gave up a bounded wait (see moe_quant_status) */
     MQ_ERANGE = -8,     /* size beyond a documented maximum */
 };
 
@@ -177,6 +177,24 @@ int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const v
                               const float* router_w, const float* bias,
                               const mq_expert_table* expert_table, const uint8_t* fmt_per_tensor,
                               float* out, int32_t* topk_idx, float* topk_w, void* cuda_stream);
+
+/* Result of the bounded waits of the last moe_quant_forward call made with
+ * this workspace and the same cfg / n_tokens.  The expert-FFN kernels give
+ * up a wait on a pipeline barrier after a time limit instead of hanging;
+ * they then set a bit in an error word of the workspace (cleared at the
+ * start of every forward call) and their outputs are not valid.  This call
+ * waits for the stream (cudaStreamSynchronize), reads the word and returns
+ * MQ_OK (0 bits), MQ_EDEVICE (some bit set; err_bits, or NULL, receives the
+ * bits), or the argument codes of moe_quant_forward (MQ_EWORKSPACE for a
+ * workspace that does not fit cfg / n_tokens) and MQ_ECUDA.  n_tokens = 0
+ * returns MQ_OK without touching the device.  Not for use while the stream
+ * is being captured. */
+int moe_quant_status(const mq_layer_cfg* cfg, int32_t n_tokens, const void* workspace, size_t ws_bytes,
+                     uint32_t* err_bits, void* cuda_stream);
+
+/* moe_quant_status for moe_quant_forward_noalloc: reads the error word of
+ * the library's fixed scratch (same cfg / n_tokens as that call). */
+int moe_quant_status_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, uint32_t* err_bits, void* cuda_stream);
 
 /* Routing and permutation only (steps 1-2 of the layer):
  *   topk_idx/topk_w device [n_tokens, top_k] (required),

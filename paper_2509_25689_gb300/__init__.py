@@ -76,6 +76,8 @@ def _load():
         "moe_quant_forward_noalloc": (ctypes.c_int, [cfgp, i32, vp, vp, vp, ctypes.POINTER(mq_expert_table), vp,
                                                      vp, vp, vp, vp]),
         "moe_quant_route": (ctypes.c_int, [cfgp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
+        "moe_quant_status": (ctypes.c_int, [cfgp, i32, vp, sz, ctypes.POINTER(ctypes.c_uint32), vp]),
+        "moe_quant_status_noalloc": (ctypes.c_int, [cfgp, i32, ctypes.POINTER(ctypes.c_uint32), vp]),
         "mq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "mq_set_path": (ctypes.c_int, [ctypes.c_int, i32]),
         "mq_profile_enable": (ctypes.c_int, [i32]),
@@ -93,7 +95,8 @@ def _load():
 _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
             "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
-            "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order")
+            "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order", "moe_quant_status",
+            "moe_quant_status_noalloc")
 
 
 def _ptr(a):
@@ -238,6 +241,27 @@ def moe_quant_route(cfg, n_tokens, x, router_w, bias, topk_idx, topk_w, offsets=
                               _ptr(topk_w), _ptr(offsets), _ptr(perm), _ptr(inv), _ptr(workspace), ws_bytes,
                               _stream(stream))
     return _check("moe_quant_route", rc)
+
+
+def moe_quant_status(cfg, n_tokens, workspace, ws_bytes=None, stream=None) -> int:
+    """Error bits of the last forward call with this workspace (0 = none);
+    raises MoeqError on bad arguments.  Waits for the stream."""
+    if ws_bytes is None:
+        ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    bits = ctypes.c_uint32(0)
+    rc = _lib.moe_quant_status(ctypes.byref(cfg), n_tokens, _ptr(workspace), ws_bytes, ctypes.byref(bits),
+                               _stream(stream))
+    if rc not in (MQ_OK, MQ_EDEVICE):
+        raise MoeqError("moe_quant_status", rc)
+    return int(bits.value)
+
+
+def moe_quant_status_noalloc(cfg, n_tokens, stream=None) -> int:
+    bits = ctypes.c_uint32(0)
+    rc = _lib.moe_quant_status_noalloc(ctypes.byref(cfg), n_tokens, ctypes.byref(bits), _stream(stream))
+    if rc not in (MQ_OK, MQ_EDEVICE):
+        raise MoeqError("moe_quant_status_noalloc", rc)
+    return int(bits.value)
 
 
 def mq_set_path(mode: int, prefill_threshold: int = 0):

@@ -321,6 +321,49 @@ extern "C" int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_toke
                              kNoAllocScratchBytes, stream);
 }
 
+namespace {
+
+// Reads the error word of the workspace laid out for (cfg, n_tokens) once the
+// stream's work is done.
+int read_status(const mq_layer_cfg* cfg, int32_t n_tokens, const void* ws, size_t ws_bytes, uint32_t* err_bits,
+                void* stream) {
+    const int rc = check_cfg(cfg);
+    if (rc != MQ_OK) return rc;
+    if (n_tokens < 0 || n_tokens > 65536) return MQ_ESHAPE;
+    const Dims d = dims_of(cfg, n_tokens);
+    const size_t need = workspace_plan(d, nullptr, nullptr);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u)) return MQ_EWORKSPACE;
+    if (err_bits) *err_bits = 0;
+    if (n_tokens == 0) return MQ_OK;   // a call without tokens launches nothing
+    Work w;
+    workspace_plan(d, const_cast<void*>(ws), &w);
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t v = 0;
+    if (cudaMemcpyAsync(&v, w.err, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess) return MQ_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MQ_ECUDA;
+    if (err_bits) *err_bits = v;
+    return v ? MQ_EDEVICE : MQ_OK;
+}
+
+}  // namespace
+
+extern "C" int moe_quant_status(const mq_layer_cfg* cfg, int32_t n_tokens, const void* workspace, size_t ws_bytes,
+                                uint32_t* err_bits, void* stream) {
+    return read_status(cfg, n_tokens, workspace, ws_bytes, err_bits, stream);
+}
+
+extern "C" int moe_quant_status_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, uint32_t* err_bits,
+                                        void* stream) {
+    const int rc = check_cfg(cfg);
+    if (rc != MQ_OK) return rc;
+    if (n_tokens < 0 || n_tokens > 65536) return MQ_ESHAPE;
+    if (workspace_plan(dims_of(cfg, n_tokens), nullptr, nullptr) > kNoAllocScratchBytes) return MQ_ERANGE;
+    void* scratch = nullptr;
+    const int sr = noalloc_scratch(&scratch);
+    if (sr != MQ_OK) return sr;
+    return read_status(cfg, n_tokens, scratch, kNoAllocScratchBytes, err_bits, stream);
+}
+
 extern "C" int mq_unpack_device(int fmt, const void* src, int64_t rows, int64_t cols, float* dst, void* stream) {
     if (!valid_format(fmt)) return MQ_EFORMAT;
     if (rows < 0 || cols < 0) return MQ_EINVAL;

@@ -157,3 +157,21 @@ def test_bench_traffic_only_for_the_captured_workload():
     assert t is None or t > 0
     assert bench._profiled_traffic("gateup_mma", "v3_decode_t1_k6") is None
     assert bench._profiled_traffic("router_logits") is None
+
+
+def test_status_argument_checks(mq):
+    cfg = mq.make_cfg(256, 128, 8, 1, 1, 2)
+    ws = mq.moe_quant_workspace_size(cfg, 4)
+    with pytest.raises(mq.MoeqError) as e:
+        mq.moe_quant_status(cfg, 4, None, ws)
+    assert e.value.status == mq.MQ_EWORKSPACE
+    with pytest.raises(mq.MoeqError):
+        mq.moe_quant_status(cfg, 4, 256, ws - 1)        # smaller than the forward call's layout
+    with pytest.raises(mq.MoeqError):
+        mq.moe_quant_status(cfg, 4, 128, ws)            # not 256-byte aligned
+    with pytest.raises(mq.MoeqError):
+        mq.moe_quant_status(mq.make_cfg(100, 128, 8, 1, 1, 2), 4, 256, ws)
+    assert mq.moe_quant_status(cfg, 0, 256, ws) == 0    # no tokens: nothing ran, no device access
+    with pytest.raises(mq.MoeqError) as e:
+        mq.moe_quant_status_noalloc(mq.make_cfg(7168, 2048, 192, 8, 4, 8, has_shared=True), 4096)
+    assert e.value.status == mq.MQ_ERANGE

@@ -286,6 +286,29 @@ def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc, decode_kernel):
         assert_close(y[t:t + 1], ry)
 
 
+def test_status_word_clean_after_forward_on_every_path(torch_cuda):
+    """The error word the kernels set when a bounded wait gives up stays 0 on
+    normal calls, on the decode (both kernels) and prefill paths."""
+    import torch
+    mq = mq_lib()
+    spec = replace(SMALL_MIXED, tokens=5)
+    layer = DeviceLayer(spec, 3, fmts=SMALL_MIXED_FMTS)
+    T = 5
+    x = torch.from_numpy(tokens(spec, 3).view(np.int16)).cuda()
+    out = torch.empty((T, spec.hidden), device="cuda")
+    wsb = mq.moe_quant_workspace_size(layer.cfg, T)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    for path in (1, 2, 3):
+        mq.mq_set_path(path)
+        try:
+            mq.moe_quant_forward(layer.cfg, T, x, layer.router_w, layer.bias, layer.table, layer.fmts, out,
+                                 workspace=ws, ws_bytes=wsb)
+        finally:
+            mq.mq_set_path(0)
+        assert mq.moe_quant_status(layer.cfg, T, ws, wsb) == 0
+        assert torch.isfinite(out).all()
+
+
 def test_forward_zero_tokens_is_noop(torch_cuda):
     import torch
     mq = mq_lib()

@@ -50,6 +50,7 @@ def test_noalloc_matches_workspace_forward_twice(torch_cuda):
         x = tokens(spec, seed, 5 + call)
         ref, ridx, rw = lay.forward(x)
         y, idx, w = _run_noalloc(lay, x)
+        assert mq_lib().moe_quant_status_noalloc(lay.cfg, x.shape[0]) == 0   # no wait gave up
         np.testing.assert_array_equal(idx, ridx)
         np.testing.assert_array_equal(w, rw)
         assert_close(y, ref)
