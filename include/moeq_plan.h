@@ -1,5 +1,6 @@
 /*
- * moeq_plan — tensor-level mixed-precision planner, C ABI (host only).
+ * moeq_plan — host-side compression planning, C ABI: the tensor-level
+ * mixed-precision planner and the expert-importance scores for pruning.
  *
  * Chooses a quantization level for every tensor of a model under a memory
  * limit, following arXiv 2509.25689 Sec. 3.3 ("Hardware-Constrained Budget
@@ -77,6 +78,22 @@ int mq_plan_precision(const mq_plan_cfg* cfg, const mq_plan_tensor* tensors, int
  * it starts 29, 15, 44, 8.  order_out: host int32 [n], a permutation of
  * 0..n-1.  n >= 0. */
 int mq_binary_partition_order(int32_t n, int32_t* order_out);
+
+/* Expert-importance scores for pruning (Sec. 3.1).  Over a routed
+ * calibration stream of n_tokens tokens (moe_quant_route's topk_idx /
+ * topk_w copied to the host: int32 / fp32 [n_tokens, top_k], ids in
+ * 0..n_experts-1, finite weights):
+ *   f_e = tokens selecting e / n_tokens, s_e = mean weight of e's
+ *   selections (0 if none), I_e = alpha f_e + (1 - alpha) s_e,
+ * counts and sums taken in token-major slot order in double precision.
+ * The ceil(retain * n_experts) experts of largest I_e (ties to the lower id)
+ * are kept: keep_out (host int32, room for n_experts) receives their ids in
+ * ascending order and *n_keep_out their number; scores_out (host double
+ * [n_experts], or NULL) receives I_e.  alpha in [0, 1], retain in (0, 1].
+ * Returns MQ_OK or MQ_EINVAL (nothing written). */
+int mq_expert_importance(const int32_t* topk_idx, const float* topk_w, int32_t n_tokens, int32_t top_k,
+                         int32_t n_experts, double alpha, double retain, double* scores_out, int32_t* keep_out,
+                         int32_t* n_keep_out);
 
 #ifdef __cplusplus
 }

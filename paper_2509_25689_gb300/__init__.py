@@ -85,6 +85,8 @@ def _load():
         "mq_plan_precision": (ctypes.c_int, [ctypes.POINTER(mq_plan_cfg), ctypes.POINTER(mq_plan_tensor), i32, vp,
                                              ctypes.POINTER(ctypes.c_int64)]),
         "mq_binary_partition_order": (ctypes.c_int, [i32, vp]),
+        "mq_expert_importance": (ctypes.c_int, [vp, vp, i32, i32, i32, ctypes.c_double, ctypes.c_double, vp, vp,
+                                                ctypes.POINTER(ctypes.c_int32)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -96,7 +98,7 @@ _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
             "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
             "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order", "moe_quant_status",
-            "moe_quant_status_noalloc")
+            "moe_quant_status_noalloc", "mq_expert_importance")
 
 
 def _ptr(a):
@@ -305,3 +307,21 @@ def mq_binary_partition_order(n: int):
     out = np.empty(max(n, 1), np.int32)
     _check("mq_binary_partition_order", _lib.mq_binary_partition_order(n, out.ctypes.data))
     return out[:n]
+
+
+def mq_expert_importance(topk_idx, topk_w, n_experts: int, alpha: float = 0.5, retain: float = 0.75):
+    """Host arrays [n_tokens, top_k] (numpy or CPU tensors).  Returns (kept
+    expert ids ascending, I_e scores)."""
+    import numpy as np
+    idx = np.ascontiguousarray(topk_idx.numpy() if hasattr(topk_idx, "numpy") else topk_idx, dtype=np.int32)
+    w = np.ascontiguousarray(topk_w.numpy() if hasattr(topk_w, "numpy") else topk_w, dtype=np.float32)
+    if idx.ndim != 2 or w.shape != idx.shape:
+        raise MoeqError("mq_expert_importance", MQ_EINVAL)
+    scores = np.empty(max(n_experts, 1), np.float64)
+    keep = np.empty(max(n_experts, 1), np.int32)
+    nk = ctypes.c_int32(0)
+    _check("mq_expert_importance",
+           _lib.mq_expert_importance(idx.ctypes.data, w.ctypes.data, idx.shape[0], idx.shape[1], n_experts,
+                                     float(alpha), float(retain), scores.ctypes.data, keep.ctypes.data,
+                                     ctypes.byref(nk)))
+    return keep[:nk.value], scores[:n_experts]
