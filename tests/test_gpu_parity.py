@@ -161,6 +161,28 @@ def test_forward_sizes_not_multiple_of_256(torch_cuda, orc, T, decode_kernel):
     assert_close(y, ry)
 
 
+def test_expert_pruning_scores_from_device_routing(torch_cuda, orc):
+    """Sec. 3.1 on the unpruned router (256 experts, 8 groups, top-8): a
+    synthetic calibration stream routed on the GPU, the importance scores and
+    the kept 192 experts from the library's host routine, against the oracle
+    routing the same tokens and scoring them itself."""
+    from oracle import prune as R
+    mq = mq_lib()
+    spec = LayerSpec(name="v3_unpruned_router", hidden=7168, inter=2048, n_experts=256, n_groups=8, topk_group=4,
+                     top_k=8, tokens=512, has_shared=True, router_std=1 / 7168 ** 0.5, bias_std=0.01)
+    lay = _RouterOnly(spec, 4)
+    x = tokens(spec, 4, 512)
+    idx, w, *_ = _route(torch_cuda, lay, x)
+    keep, scores = mq.mq_expert_importance(idx, w, 256, 0.5, 0.75)
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group, spec.top_k,
+                           spec.routed_scale, spec.has_shared)
+    ridx, rw, _, _ = orc.route(layer, x, lay.router_w_host, lay.bias_host)
+    rkeep, rscores = R.prune(ridx.tolist(), rw.tolist(), 256, 0.5, 0.75)
+    assert len(keep) == 192
+    assert list(keep) == rkeep
+    np.testing.assert_array_equal(scores, np.array(rscores))
+
+
 def test_routing_tie_break_on_device(torch_cuda, orc):
     """All-zero activations tie every expert; lowest ids must win."""
     spec = LayerSpec(name="ties", hidden=256, inter=128, n_experts=32, n_groups=4, topk_group=2, top_k=5,
