@@ -31,7 +31,11 @@ def test_hand_example_kept_sets():
 
 def test_keep_count_is_the_papers_ceiling():
     # Sec. 3.1 keeps ceil(r E): 192 of DeepSeek-V3's 256 routed experts at r = 0.75
-    assert R.keep_count(0.75, 256) == 192
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "paper_examples.json")) as f:
+        ex = json.load(f)["expert_retention"]
+    assert R.keep_count(ex["r"], ex["n_experts"]) == ex["kept"]
     assert R.keep_count(1.0, 256) == 256
     assert R.keep_count(0.001, 256) == 1
 

@@ -168,7 +168,12 @@ def test_permutation_invariants(orc):
 def test_paper_activation_adjustment_and_flops():
     """k_pruned = ceil(r k_orig): r = 0.75, k_orig = 8 gives the deployed 6
     of 192 experts (Sec. 3.2, Sec. 4.1); FLOPs_active = 2 sum k_i P_i."""
+    import json
+    import os
     from workloads import activation_adjusted_k, flops_active
+    with open(os.path.join(os.path.dirname(__file__), "golden", "paper_examples.json")) as f:
+        ex = json.load(f)["activation_adjustment"]
+    assert activation_adjusted_k(ex["r"], ex["k_orig"]) == ex["k_pruned"]
     assert activation_adjusted_k(0.75, 8) == 6
     from workloads import get_config
     spec = get_config("v3_decode_t1_k6")
