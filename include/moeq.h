@@ -143,6 +143,15 @@ size_t moe_quant_workspace_size(const mq_layer_cfg* cfg, int32_t n_tokens);
  *   workspace      device scratch of ws_bytes >= moe_quant_workspace_size
  * Routing follows a canonical fp32 order so expert ids are bit-exact with
  * the CPU reference; out is fp32 with fp32 accumulation.
+ * Range: any finite bf16 token is accepted.  The decode kernels scale every
+ * 32-element block of a token (and of the SwiGLU output) by its own power of
+ * two; the prefill grouped GEMM (n_tokens >= 64 by default) takes each token
+ * as fp16(x * 2^-e), e the exponent of the token's largest |x|, and its
+ * SwiGLU output as fp16(h * 2^-2e), undoing both in fp32.  A prefill SwiGLU
+ * output still beyond the fp16 range after that scaling (it needs
+ * |h| > 65504 * 2^2e, far outside trained models) is not passed on silently:
+ * the call's error word gets bit 16 and moe_quant_status returns
+ * MQ_EDEVICE.
  * Shape rules (MQ_ESHAPE): hidden and inter multiples of 128 (hidden <=
  * 32768, inter <= 16384), 1 <= n_experts <= 256, n_experts % n_groups == 0,
  * n_groups <= 64, 1 <= topk_group <= n_groups, 1 <= top_k <= 32 and
@@ -154,10 +163,10 @@ int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
                       void* workspace, size_t ws_bytes, void* cuda_stream);
 
 /* moe_quant_forward without a workspace argument, for callers that cannot
- * allocate device memory: plugins whose host owns every allocation, code
- * running while a stream is being captured (cudaMalloc is not allowed
- * there), or latency-bound loops that must not call cudaMalloc/cudaFree,
- * which can synchronize the device.  The paper has no counterpart; it is a
+ * allocate device memory: plugins and embedding runtimes whose host owns
+ * every allocation (they hand out no device buffers of their own), or
+ * latency-bound serving loops that must not call cudaMalloc/cudaFree, which
+ * can synchronize the whole device.  The paper has no counterpart; it is a
  * deployment convenience of this library.
  *   Arguments, layouts and results are those of moe_quant_forward.
  *   Scratch: a fixed 16 MiB device array inside this library, held on every
@@ -178,11 +187,14 @@ int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const v
                               const mq_expert_table* expert_table, const uint8_t* fmt_per_tensor,
                               float* out, int32_t* topk_idx, float* topk_w, void* cuda_stream);
 
-/* Result of the bounded waits of the last moe_quant_forward call made with
- * this workspace and the same cfg / n_tokens.  The expert-FFN kernels give
- * up a wait on a pipeline barrier after a time limit instead of hanging;
- * they then set a bit in an error word of the workspace (cleared at the
- * start of every forward call) and their outputs are not valid.  This call
+/* Result of the device-side checks of the last moe_quant_forward call made
+ * with this workspace and the same cfg / n_tokens.  The expert-FFN kernels
+ * give up a wait on a pipeline barrier after a time limit instead of
+ * hanging; they then set a bit in an error word of the workspace (cleared at
+ * the start of every forward call) and their outputs are not valid.  Bits:
+ * 1 / 2 a decode GEMV consumer / producer gave up a wait, 4 a prefill GEMM
+ * wait, 8 a tcgen05 GEMV wait, 16 a prefill SwiGLU output beyond the fp16
+ * range (see moe_quant_forward).  This call
  * waits for the stream (cudaStreamSynchronize), reads the word and returns
  * MQ_OK (0 bits), MQ_EDEVICE (some bit set; err_bits, or NULL, receives the
  * bits), or the argument codes of moe_quant_forward (MQ_EWORKSPACE for a
@@ -222,6 +234,17 @@ const char* mq_strerror(int status);
  * sets the initial value.  threshold <= 0 keeps the current one (default
  * 64).  Returns MQ_EINVAL for another mode. */
 int mq_set_path(int mode, int32_t prefill_threshold);
+
+/* Test hook for the bounded waits (no counterpart in the paper).  Arms a
+ * one-shot fault for the next decode call that runs the default (mma.sync)
+ * GEMV kernels: every limit on a pipeline wait becomes wait_ns (0 < wait_ns
+ * <= 1e9) and the gate/up kernel's producer posts nothing for its first
+ * stage, so the consumers' wait on that stage runs out.  The kernels then
+ * record the give-up in the call's error word and exit normally (no copy is
+ * left in flight); moe_quant_status reports MQ_EDEVICE, the call's outputs
+ * are not valid, and later calls are unaffected.  Process wide; returns
+ * MQ_EINVAL for wait_ns out of range. */
+int mq_test_fail_next_decode(uint64_t wait_ns);
 
 /* Kernel timing for measurement tools.  mq_profile_enable(n) makes the next
  * calls record a CUDA event pair around each kernel they launch (up to n

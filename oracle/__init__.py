@@ -16,6 +16,9 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SO = os.path.join(_HERE, f"liboracle_{platform.machine()}.so")
+# the same source built with -fopenmp: independent rows and tokens split over
+# threads, identical arithmetic per row/token (OMP_NUM_THREADS sets the count)
+_SO_OMP = os.path.join(_HERE, f"liboracle_omp_{platform.machine()}.so")
 
 Q2_K, Q3_K, Q4_K, Q8_0 = 1, 2, 3, 4
 FORMATS = {"Q2_K": Q2_K, "Q3_K": Q3_K, "Q4_K": Q4_K, "Q8_0": Q8_0}
@@ -31,26 +34,36 @@ class OracleLayer(ctypes.Structure):
 
 
 def build(force: bool = False) -> str:
-    """Compile oracle.c into liboracle.so (gcc, no fast-math, no contraction)."""
+    """Compile oracle.c into liboracle.so (gcc, no fast-math, no contraction),
+    and the OpenMP build of the same source."""
     src = os.path.join(_HERE, "oracle.c")
-    if not force and os.path.exists(_SO) and os.path.getmtime(_SO) >= max(
-            os.path.getmtime(src), os.path.getmtime(os.path.join(_HERE, "oracle.h"))):
-        return _SO
-    tmp = _SO + f".tmp{os.getpid()}"
-    subprocess.check_call(["gcc", "-O1", "-std=c11", "-ffp-contract=off", "-fno-fast-math",
-                           "-fPIC", "-shared", "-o", tmp, src, "-lm"])
-    os.replace(tmp, _SO)
+    newest = max(os.path.getmtime(src), os.path.getmtime(os.path.join(_HERE, "oracle.h")))
+    for so, extra in ((_SO, []), (_SO_OMP, ["-fopenmp"])):
+        if not force and os.path.exists(so) and os.path.getmtime(so) >= newest:
+            continue
+        tmp = so + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O1", "-std=c11", "-ffp-contract=off", "-fno-fast-math", *extra,
+                               "-fPIC", "-shared", "-o", tmp, src, "-lm"])
+        os.replace(tmp, so)
     return _SO
 
 
-_lib = None
+_libs = {}
+_omp = False
+
+
+def use_openmp(on: bool) -> None:
+    """Route the following calls to the OpenMP build (True) or the plain
+    single-threaded build (False, the default)."""
+    global _omp
+    _omp = bool(on)
 
 
 def lib():
-    global _lib
-    if _lib is None:
+    key = _omp
+    if key not in _libs:
         build()
-        L = ctypes.CDLL(_SO)
+        L = ctypes.CDLL(_SO_OMP if key else _SO)
         vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
         L.oracle_packed_size.restype = ctypes.c_size_t
         L.oracle_packed_size.argtypes = [ctypes.c_int, i64, i64]
@@ -69,8 +82,8 @@ def lib():
         L.oracle_moe_forward.restype = ctypes.c_int
         L.oracle_moe_forward.argtypes = [ctypes.POINTER(OracleLayer), i32, vp, vp, vp,
                                          vp, vp, vp, vp, vp, vp, vp]
-        _lib = L
-    return _lib
+        _libs[key] = L
+    return _libs[key]
 
 
 def _p(a: np.ndarray | None):

@@ -1,6 +1,9 @@
 /*
  * Oracle for the quantized MoE expert FFN — TEST INFRASTRUCTURE ONLY.
- * (Plain C, single thread, compiled with -O1 -ffp-contract=off.)
+ * (Plain C, compiled with -O1 -ffp-contract=off.  The default build is
+ * single-threaded; a second build with -fopenmp splits independent rows and
+ * tokens over threads through the `omp` pragmas below, which change no
+ * row's or token's arithmetic, so both builds give identical bits.)
  *
  * Only tests/, __graft_entry__.smoke() and the benchmark's CPU-baseline leg
  * may load this code.  It shares nothing with the CUDA library.
@@ -379,8 +382,10 @@ int oracle_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float
     int64_t nb = (cols + g.qk - 1) / g.qk, prow = round_up(rows, ROW_TILE);
     int64_t off[MAX_PLANES + 1];
     plane_offsets(&g, prow * nb, off);
-    uint8_t rec[MAX_PLANES][128];
+    /* rows are independent: the OpenMP build splits them over threads */
+#pragma omp parallel for schedule(static)
     for (int64_t r = 0; r < rows; r++) {
+        uint8_t rec[MAX_PLANES][128];
         for (int64_t b = 0; b < nb; b++) {
             /* gather the record of (row r, block b) from its units */
             for (int p = 0; p < g.nplanes; p++)
@@ -541,8 +546,12 @@ int oracle_route(const oracle_layer* L, int32_t T, const uint16_t* x,
                  float* w, float* z_out, float* s_out) {
     if (check_layer(L) || T < 0 || L->n_experts > 1024 || L->n_groups > 256) return -1;
     int E = L->n_experts, H = L->hidden;
+    /* tokens are independent: the OpenMP build splits them over threads */
+#pragma omp parallel
+    {
     float* s = (float*)malloc(sizeof(float) * E);
     float* u = (float*)malloc(sizeof(float) * E);
+#pragma omp for schedule(static)
     for (int t = 0; t < T; t++) {
         for (int e = 0; e < E; e++) {
             float z = oracle_router_logit(x + (int64_t)t * H, router_w + (int64_t)e * H, H);
@@ -554,6 +563,7 @@ int oracle_route(const oracle_layer* L, int32_t T, const uint16_t* x,
         select_token(L, s, u, idx + (int64_t)t * L->top_k, w + (int64_t)t * L->top_k);
     }
     free(s); free(u);
+    }
     return 0;
 }
 
@@ -587,6 +597,9 @@ static double silu(double v) { return v / (1.0 + exp(-v)); }
 static void expert_apply(int H, int I, const float* Wg, const float* Wu,
                          const float* Wd, const double* x, double wt,
                          double* hbuf, double* y) {
+    /* every output row is one dot product in a fixed order; the OpenMP build
+     * splits the rows over threads without changing any row's arithmetic */
+#pragma omp parallel for schedule(static)
     for (int i = 0; i < I; i++) {
         double g = 0.0, u = 0.0;
         const float* rg = Wg + (int64_t)i * H;
@@ -594,6 +607,7 @@ static void expert_apply(int H, int I, const float* Wg, const float* Wu,
         for (int c = 0; c < H; c++) { g += (double)rg[c] * x[c]; u += (double)ru[c] * x[c]; }
         hbuf[i] = silu(g) * u;
     }
+#pragma omp parallel for schedule(static)
     for (int r = 0; r < H; r++) {
         double o = 0.0;
         const float* rd = Wd + (int64_t)r * I;

@@ -80,6 +80,7 @@ def _load():
         "moe_quant_status_noalloc": (ctypes.c_int, [cfgp, i32, ctypes.POINTER(ctypes.c_uint32), vp]),
         "mq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "mq_set_path": (ctypes.c_int, [ctypes.c_int, i32]),
+        "mq_test_fail_next_decode": (ctypes.c_int, [ctypes.c_uint64]),
         "mq_profile_enable": (ctypes.c_int, [i32]),
         "mq_profile_collect": (ctypes.c_int, [ctypes.POINTER(mq_kernel_stat), i32]),
         "mq_plan_precision": (ctypes.c_int, [ctypes.POINTER(mq_plan_cfg), ctypes.POINTER(mq_plan_tensor), i32, vp,
@@ -98,7 +99,7 @@ _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
             "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
             "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order", "moe_quant_status",
-            "moe_quant_status_noalloc", "mq_expert_importance")
+            "moe_quant_status_noalloc", "mq_expert_importance", "mq_test_fail_next_decode")
 
 
 def _ptr(a):
@@ -264,6 +265,12 @@ def moe_quant_status_noalloc(cfg, n_tokens, stream=None) -> int:
     if rc not in (MQ_OK, MQ_EDEVICE):
         raise MoeqError("moe_quant_status_noalloc", rc)
     return int(bits.value)
+
+
+def mq_test_fail_next_decode(wait_ns: int):
+    """Test hook: the next decode call's pipeline waits give up after wait_ns
+    (the gate/up producer posts nothing for its first stage)."""
+    return _check("mq_test_fail_next_decode", _lib.mq_test_fail_next_decode(int(wait_ns)))
 
 
 def mq_set_path(mode: int, prefill_threshold: int = 0):

@@ -12,8 +12,9 @@ its per-tensor formats are its whole state.  A checkpoint directory holds
 Streams: "router_w" (fp32 [E, H]), "bias" (fp32 [E], optional), and
 "e{i}.gate|up|down" / "shared.gate|up|down" (packed bytes, sizes checked
 against mq_packed_size for the stream's format and shape).  Loading checks
-every size and checksum and raises ValueError on a mismatch, so a truncated
-or corrupted file never reaches the kernels.
+the configuration's bounds, the formats table (one row per expert, known
+codes), every size and checksum and raises ValueError on a mismatch, so a
+truncated, corrupted or inconsistent file never reaches the kernels.
 """
 from __future__ import annotations
 
@@ -28,6 +29,36 @@ from . import mq_packed_size
 VERSION = 1
 _ALIGN = 256
 _CFG_FIELDS = ("hidden", "inter", "n_experts", "n_groups", "topk_group", "top_k", "routed_scale", "has_shared")
+
+
+def _check_cfg(cfg: dict) -> None:
+    """The mq_layer_cfg bounds moe_quant_forward enforces, as ValueError."""
+    missing = [k for k in _CFG_FIELDS if k not in cfg]
+    if missing:
+        raise ValueError(f"cfg: missing fields {missing}")
+    try:
+        H, I, E, G, Gk, K, S = (int(cfg[k]) for k in _CFG_FIELDS if k != "routed_scale")
+        rs = float(cfg["routed_scale"])
+    except (TypeError, ValueError) as exc:
+        raise ValueError(f"cfg: non-numeric field ({exc})") from None
+    checks = [
+        (128 <= H <= 32768 and H % 128 == 0, "hidden must be a multiple of 128 in [128, 32768]"),
+        (128 <= I <= 16384 and I % 128 == 0, "inter must be a multiple of 128 in [128, 16384]"),
+        (1 <= E <= 256, "n_experts must be in [1, 256]"),
+        (1 <= G <= 64 and E % G == 0, "n_groups must be in [1, 64] and divide n_experts"),
+        (1 <= Gk <= G, "topk_group must be in [1, n_groups]"),
+        (1 <= K <= 32 and K <= Gk * (E // G), "top_k must be in [1, 32] and at most topk_group * n_experts / n_groups"),
+        (S in (0, 1), "has_shared must be 0 or 1"),
+        (np.isfinite(rs), "routed_scale must be finite"),
+    ]
+    for ok, msg in checks:
+        if not ok:
+            raise ValueError(f"cfg: {msg}")
+
+
+def _valid_format(f: int) -> bool:
+    """A format code the library knows (it sizes a tensor in it)."""
+    return mq_packed_size(int(f), 32, 256) > 0
 
 
 def _host(a) -> np.ndarray:
@@ -93,8 +124,16 @@ def load_layer(path: str, device=None) -> dict:
     if header.get("version") != VERSION:
         raise ValueError(f"unsupported checkpoint version {header.get('version')}")
     cfg = header["cfg"]
-    fm = np.asarray(header["formats"], np.uint8).reshape(-1, 3)
+    _check_cfg(cfg)
+    fm = np.asarray(header["formats"], np.int64)
     E = int(cfg["n_experts"])
+    n_rows = E + int(cfg["has_shared"])
+    if fm.ndim != 2 or fm.shape != (n_rows, 3):
+        raise ValueError(f"formats: shape {fm.shape}, the configuration needs ({n_rows}, 3)")
+    bad = sorted({int(f) for f in fm.reshape(-1) if not _valid_format(int(f))})
+    if bad:
+        raise ValueError(f"formats: unknown format codes {bad}")
+    fm = fm.astype(np.uint8)
     shp = _shapes(cfg)
     blob = np.fromfile(os.path.join(path, "layer.bin"), np.uint8)
     got = {}
@@ -120,7 +159,13 @@ def load_layer(path: str, device=None) -> dict:
     if rw.size != E * int(cfg["hidden"]):
         raise ValueError("router_w size does not match the configuration")
     out["router_w"] = conv(rw.reshape(E, int(cfg["hidden"])))
-    out["bias"] = conv(got["bias"].view(np.float32)) if "bias" in got else None
+    if "bias" in got:
+        b = got["bias"].view(np.float32)
+        if b.size != E:
+            raise ValueError(f"bias: {b.size} values, the configuration has {E} experts")
+        out["bias"] = conv(b)
+    else:
+        out["bias"] = None
 
     def trip(name, row):
         parts = []

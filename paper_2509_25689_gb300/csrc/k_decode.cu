@@ -77,13 +77,15 @@ __device__ __forceinline__ uint64_t global_ns() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
-// Bounded wait: gives up after ~1 s, records `code` in the error word.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err, uint32_t code) {
+// Bounded wait: gives up after `limit_ns` (1 s unless a test shortened it),
+// records `code` in the error word.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err, uint32_t code,
+                                          uint64_t limit_ns) {
     if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (;;) {
         if (mbar_try(bar, parity)) return true;
-        if (global_ns() - t0 > 1000000000ull) { atomicOr(err, code); return false; }
+        if (global_ns() - t0 > limit_ns) { atomicOr(err, code); return false; }
     }
 }
 __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -234,6 +236,8 @@ struct DecodeArgs {
     float* pdn;              // [A][H]
     uint32_t* next;          // [2] item counters
     uint32_t* err;
+    uint64_t wait_ns;        // limit of every bounded wait
+    int fail_first_stage;    // test hook: the gate/up producer posts nothing for its first stage
     float* out;
     Geo geo[4][kDecodeTok];  // stage geometry per (format, tokens), computed on the host
 };
@@ -708,9 +712,16 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             for (int pj = 0; pj < nst; ++pj) {
                 const int slot = p_q % kNST;
                 const uint32_t full = bar0 + 8 * slot, empty = bar0 + 8 * (kNST + slot);
-                if (p_q >= kNST && !mbar_wait(empty, ((p_q / kNST) & 1) ^ 1, A.err, kErrEmpty)) {
+                if (p_q >= kNST && !mbar_wait(empty, ((p_q / kNST) & 1) ^ 1, A.err, kErrEmpty, A.wait_ns)) {
                     failed = true;
                     break;
+                }
+                if (!kDown && A.fail_first_stage && p_q == 0) {
+                    // test hook: nothing arrives on this slot's full barrier and
+                    // no copy targets it, so the consumers' wait runs out
+                    ++p_q;
+                    if (item < 0) break;
+                    continue;
                 }
                 if (item < 0) {   // sentinel: consumers stop here
                     if (lane == 0) { hdr[slot].item = -1; s_posted[slot] = p_q; mbar_arrive(full); }
@@ -785,7 +796,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         int n_done = 0;   // items finished by this CTA (selects the reduction buffer and the owner warps)
         for (int q = 0;; ++q) {
             const int slot = q % kNST;
-            if (!mbar_wait(bar0 + 8 * slot, (q / kNST) & 1, A.err, kErrFull)) {
+            if (!mbar_wait(bar0 + 8 * slot, (q / kNST) & 1, A.err, kErrFull, A.wait_ns)) {
                 if (lane == 0) s_fail = 1;
                 break;
             }
@@ -903,7 +914,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     // has been consumed, so nothing is in flight.
     __syncthreads();
     if (warp == kProducerWarp && s_fail && lane < kNST && s_posted[lane] >= 0)
-        mbar_wait(bar0 + 8 * lane, (s_posted[lane] / kNST) & 1, A.err, kErrFull);
+        mbar_wait(bar0 + 8 * lane, (s_posted[lane] / kNST) & 1, A.err, kErrFull, A.wait_ns);
 }
 
 // out[t] = sum of the token's routed expert outputs in slot order, then the
@@ -921,7 +932,14 @@ __global__ void combine_kernel(Dims d, const float* __restrict__ pdn, float* __r
     }
 }
 
-int g_num_sms = 0;
+void decode_setup() {
+    cudaFuncSetAttribute(ffn_kernel<false, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<true, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<false, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<true, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+}
+
+void combine_setup() { prefer_max_shared(combine_kernel); }
 
 }  // namespace
 
@@ -933,16 +951,8 @@ size_t decode_counter_bytes(const Dims& d) {
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int smem = kRingBytes;
-    if (g_num_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_num_sms <= 0) g_num_sms = 148;
-        cudaFuncSetAttribute(ffn_kernel<false, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        cudaFuncSetAttribute(ffn_kernel<true, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        cudaFuncSetAttribute(ffn_kernel<false, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        cudaFuncSetAttribute(ffn_kernel<true, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    }
+    const int g_num_sms = device_setup(kSetupDecode, decode_setup);
+    if (g_num_sms <= 0) return cudaErrorInvalidDevice;
     DecodeArgs A;
     A.d = d;
     A.nsbx = (d.H + 255) / 256;
@@ -953,6 +963,10 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.pdn = w.pdn;
     A.next = w.counters;
     A.err = w.err;
+    A.wait_ns = 1000000000ull;
+    A.fail_first_stage = 0;
+    uint64_t test_ns = 0;
+    if (take_wait_test(&test_ns)) { A.wait_ns = test_ns; A.fail_first_stage = 1; }
     A.out = out;
     auto fill_geo = [&](bool down) {
         for (int f = 1; f <= 4; ++f)
@@ -976,8 +990,7 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
 }
 
 cudaError_t launch_combine(const Dims& d, const float* pdn, float* out, cudaStream_t s) {
-    static const bool carve = (prefer_max_shared(combine_kernel), true);
-    (void)carve;
+    if (device_setup(kSetupCombine, combine_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("combine", s);
     // one CTA row per token (up to 65535; the kernel strides over the rest),
     // so large batches stream the partial outputs at full bandwidth

@@ -18,7 +18,11 @@
 // (rows x 16) bytes apart along K.
 // Epilogue (tcgen05.ld, lane = weight row): gate/up -> h = silu(g) * u * w
 // stored as fp16 per assignment; down -> one fp32 partial output row block
-// per assignment, summed in slot order by the combine kernel.
+// per assignment, summed in slot order by the combine kernel.  Range: token
+// t enters as fp16(x * 2^-e_t), e_t = the exponent of its largest |x| (so
+// any finite bf16 token fits), and h as fp16(h * 2^-2 e_t); the epilogues
+// undo both scalings in fp32.  An h that would still overflow fp16 sets an
+// error bit (MQ_EDEVICE from moe_quant_status) instead of passing an inf on.
 // Every mbarrier wait is bounded (about 1 s) and reports to the error word;
 // tensor memory is released on every exit path.
 #include <cuda_fp16.h>
@@ -44,12 +48,14 @@ constexpr int kABytes = kMT * kKC * 2;         // one weight chunk, 16 KB
 constexpr int kBBytes = kNT * kKC * 2;         // one activation chunk, 32 KB
 constexpr int kSlotBytes = 2 * kABytes + kBBytes;
 constexpr uint32_t kErrMma = 4u;
+constexpr uint32_t kErrRange = 16u;            // an fp16 SwiGLU output would overflow (see the epilogue)
 
 struct PrefillArgs {
     Dims d;
     const int32_t* offsets; const int32_t* perm; const int32_t* active; const float* wts;
-    const __half* x16;       // [T][H] tokens in fp16
-    __half* h16;             // [A][I] SwiGLU outputs (routing weight folded in)
+    const __half* x16;       // [T][H] tokens in fp16, token t scaled by 2^-xe[t]
+    const int32_t* xe;       // [T] the tokens' exponents
+    __half* h16;             // [A][I] SwiGLU outputs (routing weight folded in), scaled by 2^-2 xe[t]
     float* pdn;              // [A][H]
     uint32_t* next;          // unit counters (gate/up, down), zeroed per call
     uint32_t* err;
@@ -350,7 +356,7 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
     pdl_launch();
     extern __shared__ __align__(1024) uint8_t smem[];
     __shared__ PSlots sl;
-    __shared__ int32_t s_row[kNT], s_asg[kNT];
+    __shared__ int32_t s_row[kNT], s_asg[kNT], s_ex[kNT];
     __shared__ float s_w[kNT];
     __shared__ __align__(8) uint64_t bars[kPSlots];   // the MMAs of the slot's chunk are done
     __shared__ __align__(8) uint64_t fbar[kPSlots];   // the slot's chunk is in shared memory (every worker)
@@ -460,15 +466,16 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
         const bool shared = p < d.has_shared;
         // the unit's activation rows, assignments and weights
         for (int n = tid; n < kNT; n += kPWorkers) {
-            int a = -1, row = 0;
+            int a = -1, row = 0, ex = 0;
             float w = 0.0f;
             if (n < N) {
                 const int q = n0 + n;
                 if (shared) { a = d.T * d.K + q; row = q; w = 1.0f; }
                 else { a = A.perm[sl.first[p] + q]; row = a / d.K; w = A.wts[a]; }
+                ex = A.xe[row];   // row is the token here
                 if (kDown) row = a;
             }
-            s_row[n] = row; s_asg[n] = a; s_w[n] = w;
+            s_row[n] = row; s_asg[n] = a; s_w[n] = w; s_ex[n] = ex;
         }
         const int f0 = sl.fmt[p][0], f1 = sl.fmt[p][1];
         const TensorLayout L0 = tensor_layout(f0, kDown ? d.H : d.I, K);
@@ -628,18 +635,26 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
                              : "=r"(u8[0]), "=r"(u8[1]), "=r"(u8[2]), "=r"(u8[3]), "=r"(u8[4]), "=r"(u8[5]),
                                "=r"(u8[6]), "=r"(u8[7]) : "r"(ta + kNT));
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            // tokens enter scaled by 2^-e (e = s_ex): gate and up sums are
+            // multiplied back before SwiGLU, h leaves scaled by 2^-2e (it
+            // grows like the square of the token), the down sums are
+            // multiplied back by 2^2e
+            bool over = false;
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int nn = n + j;
                 if (nn >= N) break;
-                const int a = s_asg[nn];
+                const int a = s_asg[nn], ex = s_ex[nn];
                 if (kDown) {
-                    A.pdn[(size_t)a * d.H + row] = __uint_as_float(g8[j]);
+                    A.pdn[(size_t)a * d.H + row] = ldexpf(__uint_as_float(g8[j]), 2 * ex);
                 } else {
-                    const float gv = __uint_as_float(g8[j]), uv = __uint_as_float(u8[j]);
-                    A.h16[(size_t)a * d.I + row] = __float2half_rn(silu(gv) * uv * s_w[nn]);
+                    const float gv = ldexpf(__uint_as_float(g8[j]), ex), uv = ldexpf(__uint_as_float(u8[j]), ex);
+                    const float hs = ldexpf(silu(gv) * uv * s_w[nn], -2 * ex);
+                    over |= !(fabsf(hs) <= 65504.0f);
+                    A.h16[(size_t)a * d.I + row] = __float2half_rn(hs);
                 }
             }
+            if (over) atomicOr(A.err, kErrRange);
         }
         // the accumulators are read: the next unit's MMAs (posted after this
         // point by every worker) may overwrite them
@@ -668,25 +683,23 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
     }
 }
 
-int g_psms = 0;
+void prefill_setup() {
+    const int smem = kPSlots * kSlotBytes;
+    cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
 
 }  // namespace
 
 cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int smem = kPSlots * kSlotBytes;
-    if (g_psms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_psms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_psms <= 0) g_psms = 148;
-        cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    }
+    const int g_psms = device_setup(kSetupPrefill, prefill_setup);
+    if (g_psms <= 0) return cudaErrorInvalidDevice;
     PrefillArgs A;
     A.d = d;
     A.offsets = w.offsets; A.perm = w.perm; A.active = w.active; A.wts = w.wts;
-    A.x16 = w.x16; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
+    A.x16 = w.x16; A.xe = w.xe; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
     A.next = w.counters;
     prof_begin("gateup_tc", s);
     cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(prefill_threads(false)), smem, s, tab, A);

@@ -29,6 +29,12 @@ constexpr unsigned kFull = 0xffffffffu;
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
+// Power-of-two exponent of a token's fp16 copy for the prefill GEMM: the
+// token is stored as x * 2^-e with its largest magnitude in [1, 2), so any
+// finite bf16 input fits the fp16 range (entries below 2^-24 of the largest
+// become fp16 subnormals or zero, an error far below the fp32 accumulation's).
+__device__ __forceinline__ int token_exp(float amax) { return amax > 0.0f ? ilogbf(amax) : 0; }
+
 // ---------------------------------------------------------------------------
 // logits: grid (E, ceil(T / kTok)), one warp per 1024-element segment
 // ---------------------------------------------------------------------------
@@ -38,9 +44,10 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
                                                              const float* __restrict__ W, int H, int T,
                                                              int E, float* __restrict__ z,
                                                              __half* __restrict__ xq, float* __restrict__ xs,
-                                                             __half* __restrict__ x16,
+                                                             __half* __restrict__ x16, int32_t* __restrict__ xe,
                                                              uint32_t* __restrict__ zero_words, int n_zero) {
     __shared__ float part[32][kTok];
+    __shared__ float pmax[32][kTok];   // per segment: largest |x| of each token (prefill copy only)
     const int e = blockIdx.x, t0 = blockIdx.y * kTok;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
@@ -58,9 +65,9 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     // per-call words that must start at zero (work counters, error word)
     if (blockIdx.x == 0 && blockIdx.y == 0)
         for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
-    float acc[kTok];
+    float acc[kTok], amx[kTok];
 #pragma unroll
-    for (int j = 0; j < kTok; ++j) acc[j] = 0.0f;
+    for (int j = 0; j < kTok; ++j) acc[j] = amx[j] = 0.0f;
 #pragma unroll
     for (int j = 0; j < kTok; ++j) {
         const int t = t0 + j;
@@ -74,6 +81,9 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
                 acc[j] = __fmaf_rn(bf16_hi(xv.x), wv[c].y, acc[j]);
                 acc[j] = __fmaf_rn(bf16_lo(xv.y), wv[c].z, acc[j]);
                 acc[j] = __fmaf_rn(bf16_hi(xv.y), wv[c].w, acc[j]);
+                if (x16 != nullptr)
+                    amx[j] = fmaxf(amx[j], fmaxf(fmaxf(fabsf(bf16_lo(xv.x)), fabsf(bf16_hi(xv.x))),
+                                                 fmaxf(fabsf(bf16_lo(xv.y)), fabsf(bf16_hi(xv.y)))));
             }
         }
     }
@@ -81,10 +91,11 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     for (int j = 0; j < kTok; ++j) {
 #pragma unroll
         for (int off = 16; off >= 1; off >>= 1) acc[j] = __fadd_rn(acc[j], __shfl_xor_sync(kFull, acc[j], off));
+        if (x16 != nullptr) amx[j] = warp_max_abs(amx[j]);
     }
     if (lane == 0) {
 #pragma unroll
-        for (int j = 0; j < kTok; ++j) part[seg][j] = acc[j];
+        for (int j = 0; j < kTok; ++j) { part[seg][j] = acc[j]; pmax[seg][j] = amx[j]; }
     }
     __syncthreads();
     if (threadIdx.x < kTok) {
@@ -95,13 +106,18 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
             z[(size_t)t * E + e] = r;
         }
     }
-    // fp16 copy of the tokens for the prefill GEMM, spread over the CTAs
+    // fp16 copy of the tokens for the prefill GEMM (each token scaled by its
+    // power of two), spread over the CTAs
     if (x16 != nullptr) {
         for (int j = 0; j < kTok; ++j) {
             const int t = t0 + j;
             if (t >= T) break;
+            float m = pmax[0][j];
+            for (int s = 1; s < nseg; ++s) m = fmaxf(m, pmax[s][j]);
+            const int ex = token_exp(m);
+            if (e == 0 && threadIdx.x == 0) xe[t] = ex;
             for (int k = e * blockDim.x + threadIdx.x; k < H; k += E * blockDim.x)
-                x16[(size_t)t * H + k] = __float2half_rn(bf16_lo(x[(size_t)t * H + k]));
+                x16[(size_t)t * H + k] = __float2half_rn(ldexpf(bf16_lo(x[(size_t)t * H + k]), -ex));
         }
     }
     // The CTAs also prepare the tokens' activations for the expert-FFN
@@ -138,9 +154,10 @@ constexpr int kTokT = 4;
 __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t* __restrict__ x,
                                                                   const float* __restrict__ W, int H, int T,
                                                                   int E, float* __restrict__ z,
-                                                                  __half* __restrict__ x16,
+                                                                  __half* __restrict__ x16, int32_t* __restrict__ xe,
                                                                   uint32_t* __restrict__ zero_words, int n_zero) {
     __shared__ float part[8][kEB][kTokT];   // per segment (warp): each expert's sums of the CTA's tokens
+    __shared__ float pmax[8][kTokT];        // per segment: largest |x| of each token (prefill copy)
     const int e0 = blockIdx.x * kEB, t0 = blockIdx.y * kTokT;
     const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
@@ -163,16 +180,39 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
             if (c < nc && t0 + j < T)
                 v = __ldg(reinterpret_cast<const uint2*>(x + (size_t)(t0 + j) * H + (c0 + c) * 128 + 4 * lane));
             xf[j][c] = make_float4(bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y));
-            if (x16 != nullptr && blockIdx.x == 0 && c < nc && t0 + j < T) {
-                // fp16 copy of the tokens for the prefill GEMM
-                const __half2 h0 = __floats2half2_rn(xf[j][c].x, xf[j][c].y);
-                const __half2 h1 = __floats2half2_rn(xf[j][c].z, xf[j][c].w);
+        }
+    if (x16 != nullptr && blockIdx.x == 0) {
+        // fp16 copy of the tokens for the prefill GEMM, each token scaled by
+        // its power of two (the CTA holds its tokens' whole rows)
+#pragma unroll
+        for (int j = 0; j < kTokT; ++j) {
+            float m = 0.0f;
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                m = fmaxf(m, fmaxf(fmaxf(fabsf(xf[j][c].x), fabsf(xf[j][c].y)), fmaxf(fabsf(xf[j][c].z), fabsf(xf[j][c].w))));
+            m = warp_max_abs(m);
+            if (lane == 0) pmax[seg][j] = m;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kTokT; ++j) {
+            if (t0 + j >= T) break;
+            float m = pmax[0][j];
+            for (int s2 = 1; s2 < nseg; ++s2) m = fmaxf(m, pmax[s2][j]);
+            const int ex = token_exp(m);
+            if (threadIdx.x == 0) xe[t0 + j] = ex;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                if (c >= nc) break;
+                const __half2 h0 = __floats2half2_rn(ldexpf(xf[j][c].x, -ex), ldexpf(xf[j][c].y, -ex));
+                const __half2 h1 = __floats2half2_rn(ldexpf(xf[j][c].z, -ex), ldexpf(xf[j][c].w, -ex));
                 uint2 hv;
                 hv.x = *reinterpret_cast<const uint32_t*>(&h0);
                 hv.y = *reinterpret_cast<const uint32_t*>(&h1);
                 *reinterpret_cast<uint2*>(x16 + (size_t)(t0 + j) * H + (c0 + c) * 128 + 4 * lane) = hv;
             }
         }
+    }
     // expert el's weights in wv, expert el + 1's loading into wn while el is
     // reduced; the per-warp sums of all 16 experts wait in shared memory and
     // the segments are added once at the end
@@ -469,24 +509,30 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
     }
 }
 
+void route_setup() {
+    prefer_max_shared(router_logits_kernel);
+    prefer_max_shared(router_logits_tile_kernel);
+    prefer_max_shared(topk_kernel);
+    prefer_max_shared(permute_kernel);
+}
+
 }  // namespace
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 __half* x16, uint32_t* zero_words, int n_zero, cudaStream_t s) {
+                                 __half* x16, int32_t* xe, uint32_t* zero_words, int n_zero, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
-    static const bool carve = (prefer_max_shared(router_logits_kernel), prefer_max_shared(router_logits_tile_kernel), true);
-    (void)carve;
+    if (device_setup(kSetupRoute, route_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("router_logits", s);
     cudaError_t e;
     if (xq == nullptr && d.T >= 16 && nseg <= 8) {
         // larger batches without activation preparation: tokens reused across 16 experts
         dim3 grid((d.E + kEB - 1) / kEB, (d.T + kTokT - 1) / kTokT);
-        e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16,
+        e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16, xe,
                        zero_words, n_zero);
     } else {
         dim3 grid(d.E, (d.T + kTok - 1) / kTok);
-        e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq, xs, x16,
+        e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe,
                        zero_words, n_zero);
     }
     prof_end(s);
@@ -496,8 +542,7 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                         cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
-    static const bool carve = (prefer_max_shared(topk_kernel), true);
-    (void)carve;
+    if (device_setup(kSetupRoute, route_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("router_topk", s);
     const cudaError_t e = launch_pdl(topk_kernel, dim3((d.T + kTopkWarps - 1) / kTopkWarps), dim3(kTopkWarps * 32),
                                      0, s, z, bias, d, idx, wts);
@@ -507,8 +552,7 @@ cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_
 
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, Plan* plan, cudaStream_t s) {
-    static const bool carve = (prefer_max_shared(permute_kernel), true);
-    (void)carve;
+    if (device_setup(kSetupRoute, route_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("permute", s);
     const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, const_cast<int32_t*>(idx), d,
                                      offsets, perm, inv, active, plan, (const float*)nullptr, (const float*)nullptr,
@@ -520,8 +564,7 @@ cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, 
 cudaError_t launch_route_permute(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts,
                                  int32_t* offsets, int32_t* perm, int32_t* inv, int32_t* active, Plan* plan,
                                  cudaStream_t s) {
-    static const bool carve = (prefer_max_shared(permute_kernel), true);
-    (void)carve;
+    if (device_setup(kSetupRoute, route_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("route_permute", s);
     const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), 0, s, idx, d, offsets, perm, inv,
                                      active, plan, z, bias, wts);

@@ -628,20 +628,14 @@ __global__ void __launch_bounds__(kTThreads, 1) tgemv_kernel(const __grid_consta
     }
 }
 
-int g_tsms = 0;
-
 }  // namespace
 
 bool decode_tc_fits(const Dims& d) { return d.H % kRowsT == 0 && d.I % kRowsT == 0; }
 
 cudaError_t launch_decode_tc(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
-    if (g_tsms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_tsms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_tsms <= 0) g_tsms = 148;
-    }
+    const int g_tsms = device_setup(kSetupTgemv, nullptr);
+    if (g_tsms <= 0) return cudaErrorInvalidDevice;
     TArgs A;
     A.d = d;
     A.nsbx = (d.H + 255) / 256;

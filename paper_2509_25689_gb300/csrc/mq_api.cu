@@ -90,6 +90,7 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_hs = take(A * nsbi * kStatFloats * 4);
     const size_t o_pdn = take(A * d.H * 4);
     const size_t o_plan = take(sizeof(Plan));
+    const size_t o_xe = take((size_t)d.T * 4);
     const size_t cnt_bytes = decode_counter_bytes(d);
     const size_t o_cnt = take(cnt_bytes + 4);   // work counters, then the error word (zeroed per call)
     const size_t o_err = o_cnt + cnt_bytes;
@@ -111,12 +112,47 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
         w->counter_bytes = cnt_bytes;
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
+        w->xe = reinterpret_cast<int32_t*>(b + o_xe);
         w->x16 = w->xq;   // the prefill path uses these bytes instead of the decode preparation
         w->h16 = w->hq;
         w->zero_words = w->counters;
         w->n_zero = (int)((cnt_bytes + 4) / 4);
     }
     return at;
+}
+
+namespace {
+constexpr int kMaxSetupDevices = 64;
+std::mutex g_setup_mu;
+int g_setup_sms[kMaxSetupDevices][kSetupSlots] = {};
+}  // namespace
+
+int device_setup(int slot, void (*init)()) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxSetupDevices || slot < 0 || slot >= kSetupSlots)
+        return 0;
+    std::lock_guard<std::mutex> lk(g_setup_mu);
+    int& sms = g_setup_sms[dev][slot];
+    if (sms == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 0;
+        if (init) init();
+        sms = n;
+    }
+    return sms;
+}
+
+namespace {
+std::mutex g_wait_test_mu;
+uint64_t g_wait_test_ns = 0;   // armed when non-zero
+}  // namespace
+
+bool take_wait_test(uint64_t* wait_ns) {
+    std::lock_guard<std::mutex> lk(g_wait_test_mu);
+    if (g_wait_test_ns == 0) return false;
+    *wait_ns = g_wait_test_ns;
+    g_wait_test_ns = 0;
+    return true;
 }
 
 void prof_begin(const char* name, cudaStream_t s) {
@@ -190,7 +226,7 @@ int run_route(const Dims& d, const void* x, const float* router_w, const float* 
               cudaStream_t s, int mode) {
     const bool fwd = mode != 0;
     if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, mode == 1 ? w.xq : nullptr, w.xs,
-                             mode == 2 ? w.x16 : nullptr, fwd ? w.zero_words : nullptr, fwd ? w.n_zero : 0,
+                             mode == 2 ? w.x16 : nullptr, w.xe, fwd ? w.zero_words : nullptr, fwd ? w.n_zero : 0,
                              s) != cudaSuccess)
         return MQ_ECUDA;
     Plan* plan = mode == 1 ? w.plan : nullptr;
@@ -362,6 +398,13 @@ extern "C" int moe_quant_status_noalloc(const mq_layer_cfg* cfg, int32_t n_token
     const int sr = noalloc_scratch(&scratch);
     if (sr != MQ_OK) return sr;
     return read_status(cfg, n_tokens, scratch, kNoAllocScratchBytes, err_bits, stream);
+}
+
+extern "C" int mq_test_fail_next_decode(uint64_t wait_ns) {
+    if (wait_ns == 0 || wait_ns > 1000000000ull) return MQ_EINVAL;
+    std::lock_guard<std::mutex> lk(g_wait_test_mu);
+    g_wait_test_ns = wait_ns;
+    return MQ_OK;
 }
 
 extern "C" int mq_unpack_device(int fmt, const void* src, int64_t rows, int64_t cols, float* dst, void* stream) {

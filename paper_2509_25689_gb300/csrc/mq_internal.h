@@ -61,13 +61,28 @@ struct Work {
     uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
     size_t counter_bytes;
     uint32_t* err;     // device error word (bounded waits that ran out)
-    __half* x16;       // [T][H] tokens in fp16 for the prefill GEMM (shares xq's bytes)
+    __half* x16;       // [T][H] tokens in fp16 for the prefill GEMM (shares xq's bytes),
+                       // each token scaled by 2^-xe[t]
+    int32_t* xe;       // [T] per-token power-of-two exponents of x16 (prefill path)
     __half* h16;       // [A][I] fp16 SwiGLU outputs for the prefill GEMM (shares hq's bytes)
     uint32_t* zero_words; // counters + error word, cleared by the first kernel of a call
     int n_zero;
 };
 
 size_t workspace_plan(const Dims& d, void* base, Work* w);
+
+// Per-device one-time set-up.  Function attributes (shared-memory limits,
+// carveout preference) apply to one device, so a translation unit's set-up
+// runs once for every device it is used on: device_setup(slot, init) runs
+// init() the first time `slot` is used with the current device (under a
+// process-wide mutex) and returns that device's SM count (0 if the device
+// query failed).  Slots: one per translation unit or kernel group.
+enum SetupSlot : int { kSetupDecode = 0, kSetupPrefill, kSetupTgemv, kSetupRoute, kSetupCombine, kSetupSlots };
+int device_setup(int slot, void (*init)());
+
+// Test hook of the bounded waits (mq_test_fail_next_decode): true once after
+// it was armed, with the shortened wait limit in *wait_ns.
+bool take_wait_test(uint64_t* wait_ns);
 
 // launch helpers; each returns cudaGetLastError() of its launch
 // Programmatic dependent launch: every kernel of the layer is launched with
@@ -104,7 +119,7 @@ void prefer_max_shared(void (*kernel)(KArgs...)) {
 #endif
 
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 __half* x16, uint32_t* zero_words, int n_zero,
+                                 __half* x16, int32_t* xe, uint32_t* zero_words, int n_zero,
                                  cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,

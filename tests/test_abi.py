@@ -175,3 +175,10 @@ def test_status_argument_checks(mq):
     with pytest.raises(mq.MoeqError) as e:
         mq.moe_quant_status_noalloc(mq.make_cfg(7168, 2048, 192, 8, 4, 8, has_shared=True), 4096)
     assert e.value.status == mq.MQ_ERANGE
+
+
+def test_wait_test_hook_argument_checks(mq):
+    for bad in (0, 2_000_000_000):
+        with pytest.raises(mq.MoeqError) as e:
+            mq.mq_test_fail_next_decode(bad)
+        assert e.value.status == mq.MQ_EINVAL

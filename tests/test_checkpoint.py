@@ -82,3 +82,35 @@ def test_save_checks_sizes_against_the_formats(mq, tmp_path):
         save_layer(str(tmp_path), cfg, fm, bad, sh, rw, b)
     with pytest.raises(ValueError):
         save_layer(str(tmp_path), cfg, fm, ex, None, rw, b)   # has_shared but no shared expert
+
+
+@pytest.mark.parametrize("edit,match", [
+    (lambda h: h["formats"].pop(), "formats: shape"),                       # one row short
+    (lambda h: h["formats"][1].__setitem__(2, 9), "unknown format"),          # bad code
+    (lambda h: h["cfg"].__setitem__("n_groups", 3), "n_groups"),              # does not divide E
+    (lambda h: h["cfg"].__setitem__("top_k", 64), "top_k"),
+    (lambda h: h["cfg"].__setitem__("hidden", 200), "hidden"),
+    (lambda h: h["cfg"].pop("inter"), "missing"),
+])
+def test_inconsistent_headers_are_refused(mq, tmp_path, edit, match):
+    from paper_2509_25689_gb300.checkpoint import load_layer, save_layer
+    cfg, fm, ex, sh, rw, b = _layer(mq, np.random.default_rng(4))
+    save_layer(str(tmp_path), cfg, fm, ex, sh, rw, b)
+    hdr = json.load(open(tmp_path / "layer.json"))
+    edit(hdr)
+    json.dump(hdr, open(tmp_path / "layer.json", "w"))
+    with pytest.raises(ValueError, match=match):
+        load_layer(str(tmp_path))
+
+
+def test_bias_of_the_wrong_length_is_refused(mq, tmp_path):
+    from paper_2509_25689_gb300.checkpoint import load_layer, save_layer
+    cfg, fm, ex, sh, rw, b = _layer(mq, np.random.default_rng(5))
+    save_layer(str(tmp_path), cfg, fm, ex, sh, rw, b)
+    hdr = json.load(open(tmp_path / "layer.json"))
+    streams = {s["name"]: s for s in hdr["streams"]}
+    # the header's bias entry points at the router's bytes (checksum intact)
+    streams["bias"].update({k: streams["router_w"][k] for k in ("offset", "bytes", "sha256")})
+    json.dump(hdr, open(tmp_path / "layer.json", "w"))
+    with pytest.raises(ValueError, match="bias"):
+        load_layer(str(tmp_path))

@@ -297,15 +297,23 @@ def test_forward_v3_decode_k6(torch_cuda, orc, T, decode_kernel):
         assert_close(y[t:t + 1], ry)
 
 
-def test_forward_v3_decode_t32_mixed_sampled(torch_cuda, orc, decode_kernel):
+def test_forward_v3_decode_t32_mixed_full(torch_cuda, orc, decode_kernel):
+    """Config 3 in full: all 32 tokens of the mixed-format V3 layer against one
+    oracle call (the oracle's OpenMP build, identical bits to the plain one)."""
     spec = get_config("v3_decode_t32_mixed")
     layer = DeviceLayer(spec, 0)
     x = tokens(spec, 0)
     y, idx, w = layer.forward(x)
-    for t in (0, 13, 31):
-        ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
-        np.testing.assert_array_equal(idx[t:t + 1], ridx)
-        assert_close(y[t:t + 1], ry)
+    orc.use_openmp(True)
+    try:
+        ry, ridx, rw = layer.oracle_forward(orc, x, idx_hint=idx)
+    finally:
+        orc.use_openmp(False)
+    np.testing.assert_array_equal(idx, ridx)
+    np.testing.assert_array_equal(w.view(np.uint32), rw.view(np.uint32))
+    assert_close(y, ry)
+    for t in range(spec.tokens):   # and every token against its own scale
+        assert_close(y[t:t + 1], ry[t:t + 1])
 
 
 def test_status_word_clean_after_forward_on_every_path(torch_cuda):
@@ -329,6 +337,42 @@ def test_status_word_clean_after_forward_on_every_path(torch_cuda):
             mq.mq_set_path(0)
         assert mq.moe_quant_status(layer.cfg, T, ws, wsb) == 0
         assert torch.isfinite(out).all()
+
+
+def test_wait_give_up_reports_status_and_context_stays_usable(torch_cuda, orc):
+    """The bounded-wait give-up path, made to run out on purpose: a test hook
+    shortens every pipeline wait of the next decode call to 1 ms and has the
+    gate/up producer post nothing for its first stage.  The consumers' wait
+    on that stage ends, the kernels record it in the error word and exit
+    (no copy left in flight), moe_quant_status returns MQ_EDEVICE with the
+    full-barrier bit, and the next call runs normally and matches the oracle."""
+    import torch
+    mq = mq_lib()
+    spec = replace(SMALL_MIXED, tokens=3)
+    layer = DeviceLayer(spec, 4, fmts=SMALL_MIXED_FMTS)
+    T = 3
+    x_bits = tokens(spec, 4)
+    x = torch.from_numpy(x_bits.view(np.int16)).cuda()
+    out = torch.empty((T, spec.hidden), device="cuda")
+    wsb = mq.moe_quant_workspace_size(layer.cfg, T)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    mq.mq_set_path(1)
+    try:
+        mq.mq_test_fail_next_decode(1_000_000)
+        mq.moe_quant_forward(layer.cfg, T, x, layer.router_w, layer.bias, layer.table, layer.fmts, out,
+                             workspace=ws, ws_bytes=wsb)
+        bits = mq.moe_quant_status(layer.cfg, T, ws, wsb)
+        assert bits & 1, bits          # a consumer gave up its wait on a full barrier
+        assert bits & ~3 == 0, bits    # only the pipeline-wait bits
+        # the hook is one-shot: the next call is clean and correct
+        mq.moe_quant_forward(layer.cfg, T, x, layer.router_w, layer.bias, layer.table, layer.fmts, out,
+                             workspace=ws, ws_bytes=wsb)
+        assert mq.moe_quant_status(layer.cfg, T, ws, wsb) == 0
+    finally:
+        mq.mq_set_path(0)
+    y = out.cpu().numpy()
+    ry, _, _ = layer.oracle_forward(orc, x_bits)
+    assert_close(y, ry)
 
 
 def test_forward_zero_tokens_is_noop(torch_cuda):

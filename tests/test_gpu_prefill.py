@@ -80,16 +80,53 @@ def test_prefill_v3_layer_sampled(torch_cuda, orc, prefill_path):
         assert_close(y[t:t + 1], ry)
 
 
-def test_prefill_v3_zipf_t2048_sampled(torch_cuda, orc):
+def _stratified_tokens(idx: np.ndarray, n_experts: int, tile: int = 256, cap: int = 96) -> list:
+    """Tokens that exercise the grouped GEMM's corner cases: three on each of
+    the hottest expert's second and third token tiles, and the last token of
+    every expert's last (partial) tile, thinned evenly to `cap`; padded with
+    evenly spaced tokens to at least 64."""
+    T = idx.shape[0]
+    per_e = [np.nonzero((idx == e).any(axis=1))[0] for e in range(n_experts)]   # ascending = unit order
+    hot = int(np.argmax([len(p) for p in per_e]))
+    hot_pick = []
+    for j in (1, 2):
+        tl = per_e[hot][tile * j: tile * (j + 1)]
+        if len(tl):
+            hot_pick += [int(tl[0]), int(tl[len(tl) // 2]), int(tl[-1])]
+    last = sorted({int(p[-1]) for p in per_e if len(p)} - set(hot_pick))
+    room = max(0, cap - len(hot_pick))
+    if len(last) > room:
+        last = [last[i] for i in np.linspace(0, len(last) - 1, room).astype(int)]
+    pick = set(hot_pick) | set(last)
+    for v in np.linspace(0, T - 1, 64).astype(int):
+        if len(pick) >= 64:
+            break
+        pick.add(int(v))
+    return sorted(pick)
+
+
+def test_prefill_v3_zipf_t2048_stratified(torch_cuda, orc):
     """The Zipf-skewed V3 prefill workload (T = 2048, mixed formats) through
-    the automatic path choice; a few tokens against the oracle."""
+    the automatic path choice, against one oracle call on a stratified sample
+    of at least 64 tokens: tokens on the hottest expert's second and third
+    256-token tiles, on every expert's last partial tile, and so on every
+    format in the layer."""
     spec = get_config("v3_prefill_t2048_zipf")
     layer = DeviceLayer(spec, 0)
     x = tokens(spec, 0)
     y, idx, w = layer.forward(x)
     counts = np.bincount(idx.reshape(-1), minlength=spec.n_experts)
     assert counts.max() >= 4 * counts[counts > 0].mean()   # skewed towards a few experts
-    for t in (0, 1337, 2047):
-        ry, ridx, rw = layer.oracle_forward(orc, x[t:t + 1], idx_hint=idx[t])
-        np.testing.assert_array_equal(idx[t:t + 1], ridx)
-        assert_close(y[t:t + 1], ry)
+    pick = _stratified_tokens(idx, spec.n_experts)
+    assert len(pick) >= 64
+    used = set(int(e) for e in idx[pick].reshape(-1))
+    assert {int(f) for e in used for f in layer.fmts[e]} == {1, 2, 3}   # every routed format
+    orc.use_openmp(True)
+    try:
+        ry, ridx, rw = layer.oracle_forward(orc, x[pick], idx_hint=idx[pick])
+    finally:
+        orc.use_openmp(False)
+    np.testing.assert_array_equal(idx[pick], ridx)
+    np.testing.assert_array_equal(w[pick].view(np.uint32), rw.view(np.uint32))
+    for i, t in enumerate(pick):
+        assert_close(y[t:t + 1], ry[i:i + 1])

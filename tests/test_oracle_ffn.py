@@ -109,3 +109,37 @@ def test_zero_tokens(orc):
                                  None, [np.zeros(1, np.uint8)] * 8, [np.zeros(1, np.uint8)] * 8,
                                  [np.zeros(1, np.uint8)] * 8, np.full((8, 3), 3, np.uint8))
     assert y.shape == (0, 256)
+
+
+def test_openmp_build_gives_identical_bits(orc):
+    """The OpenMP build splits rows and tokens over threads without changing
+    any row's arithmetic: every output bit equals the single-threaded build's."""
+    import os
+    spec = get_config("tiny")
+    x = draw_tokens(3, 9, spec.hidden)
+    rw, b = draw_router(spec, 1)
+    fmts = draw_formats(spec, 1)
+    ws = draw_fp32_weights(spec, 1)
+    gate = [orc.pack("Q4_K", g) for g, _, _ in ws]
+    up = [orc.pack("Q4_K", u) for _, u, _ in ws]
+    down = [orc.pack("Q4_K", d) for _, _, d in ws]
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
+                           spec.top_k)
+    y1, idx1, w1 = orc.moe_forward(layer, x, rw, b, gate, up, down, fmts)
+    u1 = orc.unpack("Q4_K", gate[0], spec.inter, spec.hidden)
+    old = os.environ.get("OMP_NUM_THREADS")
+    os.environ["OMP_NUM_THREADS"] = "4"
+    try:
+        orc.use_openmp(True)
+        y2, idx2, w2 = orc.moe_forward(layer, x, rw, b, gate, up, down, fmts)
+        u2 = orc.unpack("Q4_K", gate[0], spec.inter, spec.hidden)
+    finally:
+        orc.use_openmp(False)
+        if old is None:
+            os.environ.pop("OMP_NUM_THREADS", None)
+        else:
+            os.environ["OMP_NUM_THREADS"] = old
+    np.testing.assert_array_equal(idx1, idx2)
+    np.testing.assert_array_equal(w1.view(np.uint32), w2.view(np.uint32))
+    np.testing.assert_array_equal(y1.view(np.uint32), y2.view(np.uint32))
+    np.testing.assert_array_equal(u1.view(np.uint32), u2.view(np.uint32))

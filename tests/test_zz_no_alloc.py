@@ -1,10 +1,12 @@
 """moe_quant_forward_noalloc: the forward pass for callers that cannot
-allocate device memory (a plugin whose host owns all allocations, code under
-stream capture, loops that must not call cudaMalloc).  Its scratch is a fixed
-16 MiB device array inside the library, so the test checks that its output
-matches the workspace-based moe_quant_forward on two calls in a row (the
-second call sees the first call's leftovers in the shared array) and that
-requests larger than the array are refused before anything is enqueued.
+allocate device memory (a plugin whose host owns all allocations, serving
+loops that must not call cudaMalloc/cudaFree because those can synchronize
+the device).  Its scratch is a fixed 16 MiB device array inside the library,
+so the test checks that its output is bit-identical to the workspace-based
+moe_quant_forward (both run the same deterministic kernels; only the scratch
+differs) on two calls in a row (the second call sees the first call's
+leftovers in the shared array) and that requests larger than the array are
+refused before anything is enqueued.
 
 This file is collected last on purpose, and it must pass both on its own in a
 fresh process (the first call on the device does the address lookup) and
@@ -15,7 +17,7 @@ import numpy as np
 import pytest
 
 from workloads.configs import LayerSpec
-from tests.gpu_helpers import DeviceLayer, assert_close, mq_lib, tokens
+from tests.gpu_helpers import DeviceLayer, mq_lib, tokens
 
 pytestmark = pytest.mark.gpu
 
@@ -53,7 +55,8 @@ def test_noalloc_matches_workspace_forward_twice(torch_cuda):
         assert mq_lib().moe_quant_status_noalloc(lay.cfg, x.shape[0]) == 0   # no wait gave up
         np.testing.assert_array_equal(idx, ridx)
         np.testing.assert_array_equal(w, rw)
-        assert_close(y, ref)
+        assert np.isfinite(y).all()
+        np.testing.assert_array_equal(y.view(np.uint32), ref.view(np.uint32))
 
 
 def test_noalloc_refuses_requests_beyond_its_scratch(torch_cuda):
