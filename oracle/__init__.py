@@ -77,6 +77,8 @@ def lib():
         L.oracle_router_logit.argtypes = [vp, vp, i32]
         L.oracle_route.restype = ctypes.c_int
         L.oracle_route.argtypes = [ctypes.POINTER(OracleLayer), i32, vp, vp, vp, vp, vp, vp, vp]
+        L.oracle_select.restype = ctypes.c_int
+        L.oracle_select.argtypes = [ctypes.POINTER(OracleLayer), i32, vp, vp, vp, vp]
         L.oracle_permute.restype = ctypes.c_int
         L.oracle_permute.argtypes = [i32, i32, i32, vp, vp, vp, vp]
         L.oracle_moe_forward.restype = ctypes.c_int
@@ -150,6 +152,21 @@ def route(layer: OracleLayer, x_bits: np.ndarray, router_w: np.ndarray,
                           _p(idx), _p(w), _p(z), _p(s)):
         raise ValueError("oracle_route failed")
     return idx, w, z, s
+
+
+def select(layer: OracleLayer, s: np.ndarray, bias: np.ndarray | None):
+    """The selection step alone on precomputed sigmoid scores s [T, E]:
+    returns idx [T,k] int32, w [T,k] f32 (identical to route's for the same
+    scores and bias)."""
+    s = np.ascontiguousarray(s, dtype=np.float32)
+    T = s.shape[0]
+    K = layer.top_k
+    idx = np.zeros((T, K), np.int32)
+    w = np.zeros((T, K), np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    if lib().oracle_select(ctypes.byref(layer), T, _p(s), _p(b), _p(idx), _p(w)):
+        raise ValueError("oracle_select failed")
+    return idx, w
 
 
 def permute(idx: np.ndarray, n_experts: int):

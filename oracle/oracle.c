@@ -567,6 +567,24 @@ int oracle_route(const oracle_layer* L, int32_t T, const uint16_t* x,
     return 0;
 }
 
+int oracle_select(const oracle_layer* L, int32_t T, const float* s, const float* bias,
+                  int32_t* idx, float* w) {
+    if (check_layer(L) || T < 0 || L->n_experts > 1024 || L->n_groups > 256 || !s) return -1;
+    int E = L->n_experts;
+#pragma omp parallel
+    {
+    float* u = (float*)malloc(sizeof(float) * E);
+#pragma omp for schedule(static)
+    for (int t = 0; t < T; t++) {
+        const float* st = s + (int64_t)t * E;
+        for (int e = 0; e < E; e++) u[e] = st[e] + (bias ? bias[e] : 0.0f);
+        select_token(L, st, u, idx + (int64_t)t * L->top_k, w + (int64_t)t * L->top_k);
+    }
+    free(u);
+    }
+    return 0;
+}
+
 int oracle_permute(int32_t T, int32_t k, int32_t E, const int32_t* idx,
                    int32_t* offsets, int32_t* perm, int32_t* inv) {
     int64_t n = (int64_t)T * k;

@@ -63,6 +63,13 @@ int oracle_route(const oracle_layer* L, int32_t T, const uint16_t* x,
                  const float* router_w, const float* bias, int32_t* idx,
                  float* w, float* z_out, float* s_out);
 
+/* The selection step of oracle_route alone, on precomputed scores: s [T, E]
+   (sigmoid scores, e.g. s_out of oracle_route) plus the selection bias ->
+   idx/w [T, k].  Lets a caller re-select under other biases without
+   recomputing the logits (the logits do not depend on the bias). */
+int oracle_select(const oracle_layer* L, int32_t T, const float* s, const float* bias,
+                  int32_t* idx, float* w);
+
 /* Stable counting sort of (token, slot) entries by expert.
    offsets [E+1], perm [T*k] (entry ids), inv [T*k] (position of entry). */
 int oracle_permute(int32_t T, int32_t k, int32_t E, const int32_t* idx,

@@ -181,3 +181,19 @@ def test_paper_activation_adjustment_and_flops():
     assert activation_adjusted_k(0.75, 256) == 192
     P = 3 * 7168 * 2048
     assert flops_active([8], [P]) == 2 * 8 * P
+
+
+def test_select_on_precomputed_scores_equals_route(orc):
+    """oracle.select re-runs only the selection step: on route's own scores it
+    returns route's ids and weights bit for bit, for any bias."""
+    from workloads.synth import draw_router, draw_tokens
+    from workloads import get_config
+    spec = get_config("v3_decode_t1")
+    x = draw_tokens(9, 24, spec.hidden)
+    rw, b = draw_router(spec, 2)
+    layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group, spec.top_k)
+    for bias in (b, None, b * 40):
+        idx, w, z, s = orc.route(layer, x, rw, bias)
+        idx2, w2 = orc.select(layer, s, bias)
+        np.testing.assert_array_equal(idx, idx2)
+        np.testing.assert_array_equal(w.view(np.uint32), w2.view(np.uint32))

@@ -68,22 +68,21 @@ def zipf_ranks(spec: LayerSpec, seed: int) -> np.ndarray:
     return rng_for(seed + 5).permutation(spec.n_experts).astype(np.int64)
 
 
-def zipf_bias_shape(spec: LayerSpec, seed: int) -> np.ndarray:
-    """-s * ln(rank + 1): the bias direction that skews expert counts towards
-    a Zipf(s) law; its scale gamma is fitted once (tests/golden/zipf_gamma.json)."""
-    return (-float(spec.zipf_s) * np.log(zipf_ranks(spec, seed) + 1.0)).astype(np.float32)
-
-
-def zipf_gamma() -> float:
+def zipf_bias() -> np.ndarray:
+    """Per-expert selection bias of the Zipf-skewed prefill workload, fitted
+    once through oracle routing (tests/golden/fit_zipf_bias.py) so that the
+    routed counts follow the water-filled Zipf(s) target; stored bit-exact."""
     import json
     import os
     path = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "tests", "golden",
-                        "zipf_gamma.json")
+                        "zipf_bias.json")
     with open(path) as f:
-        return float(json.load(f)["gamma"])
+        return np.array([float.fromhex(v) for v in json.load(f)["bias_f32_hex"]], np.float32)
 
 
-def draw_router(spec: LayerSpec, seed: int, gamma: float | None = None):
+def draw_router(spec: LayerSpec, seed: int, base_only: bool = False):
+    """Router weights and selection bias.  Zipf-skewed workloads (zipf_s set)
+    take the fitted bias instead of the N(0, bias_std) draw unless base_only."""
     r = rng_for(seed + 1)
     w = (r.standard_normal((spec.n_experts, spec.hidden), dtype=np.float32)
          * np.float32(spec.router_std)).astype(np.float32)
@@ -91,9 +90,8 @@ def draw_router(spec: LayerSpec, seed: int, gamma: float | None = None):
         b = (r.standard_normal(spec.n_experts, dtype=np.float32) * np.float32(spec.bias_std)).astype(np.float32)
     else:
         b = np.zeros(spec.n_experts, np.float32)
-    if spec.zipf_s is not None:
-        g = zipf_gamma() if gamma is None else gamma
-        b = (b + np.float32(g) * zipf_bias_shape(spec, seed)).astype(np.float32)
+    if spec.zipf_s is not None and not base_only:
+        b = zipf_bias()
     return w, b
 
 
