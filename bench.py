@@ -66,7 +66,7 @@ def _profiled_traffic(kernel: str, workload: str = PROFILE_WORKLOAD):
         fields = dict(line.split(": ", 1) for line in text.splitlines() if ": " in line and " " not in line.split(": ")[0])
         if fields.get("kernel_sources_sha256_16", "").strip() != h.hexdigest()[:16]:
             return None
-        key = {"gateup_mma": "dram_bytes_per_launch_gateup", "down_mma": "dram_bytes_per_launch_down"}.get(kernel)
+        key = {"ffn_mma": "dram_bytes_per_launch_ffn"}.get(kernel)
         return int(fields[key]) if key in fields else None
     except Exception:
         return None
@@ -138,7 +138,8 @@ def step_bytes(spec, fmts, idx_steps):
         b_dn = sum(dn(e) for e in touched) + (dn(sh) if sh is not None else 0) + (T * K + T) * I * 4 + T * H * 4
         b_rt = E * H * 4 + T * H * 2 + T * E * 4
         quant = sum(gu(e) + dn(e) for e in touched) + ((gu(sh) + dn(sh)) if sh is not None else 0)
-        out.append({"gateup_mma": b_gu, "down_mma": b_dn, "router_logits": b_rt, "quantized": quant,
+        out.append({"ffn_mma": b_gu + b_dn, "gateup_mma": b_gu, "down_mma": b_dn, "router_logits": b_rt,
+                    "quantized": quant,
                     "total": b_gu + b_dn + b_rt, "gateup_tc": b_gu, "down_tc": b_dn,
                     "gateup_tgemv": b_gu, "down_tgemv": b_dn})
     return out
@@ -164,19 +165,55 @@ def _tensor_peak():
         return 1900.0, "fallback"
 
 
-def cpu_baseline(host_layer, x_steps, budget_s=15.0, max_tokens=8):
-    """The oracle (plain single-threaded C) on a bounded sample of tokens."""
+def cpu_baseline(host_layer, x_full, budget_s=12.0, sample_tokens=8, openmp=False):
+    """The oracle as it stands (plain C, fp64 FFN) timed on the host cores on
+    a bounded sample of the workload, scaled to the whole workload.
+
+    The oracle unpacks every expert a call touches once and then applies it
+    to that expert's tokens, so its cost per call is (distinct experts) x
+    unpack + (assignments) x apply.  A sample of at most `sample_tokens` of
+    the workload's tokens is timed end to end, the unpack of the sample's
+    experts is timed on its own, and the two per-unit costs are scaled to the
+    full batch's own counts (its distinct experts from an untimed oracle
+    routing of every token, its assignments T * k + T).  For one-token
+    workloads the sample is the workload.  openmp: the oracle's OpenMP build
+    on all host cores (identical results)."""
     import oracle
     oracle.build()
-    done, t_used = 0, 0.0
-    for i in range(min(max_tokens, len(x_steps))):
-        t_used += host_layer.timed_forward(oracle, x_steps[i])
-        done += x_steps[i].shape[0]
-        if t_used > budget_s:
-            break
-    return {"value": done / t_used, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-            "sample": f"{done} token(s) of a V3 layer of the same recipe (fresh token each), full layer "
-                      f"per token: routing + 8 routed experts + shared expert, fp64 FFN; {t_used:.1f} s"}
+    oracle.use_openmp(openmp)
+    try:
+        spec = host_layer.spec
+        T = x_full.shape[0]
+        n_s = min(T, sample_tokens)
+        t_fwd, t_unpack, d_s, a_s, done = 0.0, 0.0, 0, 0, 0
+        for i in range(0, T, n_s):
+            xs = x_full[i:i + n_s]
+            tf, tu, ds = host_layer.timed_parts(oracle, xs)
+            t_fwd += tf
+            t_unpack += tu
+            d_s += ds
+            a_s += xs.shape[0] * spec.top_k + (xs.shape[0] if spec.has_shared else 0)
+            done += xs.shape[0]
+            if t_fwd + t_unpack > budget_s or n_s == T:
+                break
+        if done == T:
+            value = T / t_fwd
+            how = f"all {T} token(s) of the workload, {t_fwd:.1f} s"
+        else:
+            d_full = host_layer.distinct_experts(oracle, x_full)
+            a_full = T * spec.top_k + (T if spec.has_shared else 0)
+            per_expert = t_unpack / d_s
+            per_assign = max(t_fwd - t_unpack, 0.0) / a_s
+            t_full = d_full * per_expert + a_full * per_assign
+            value = T / t_full
+            how = (f"{done} of the workload's {T} tokens timed ({t_fwd:.1f} s, {d_s} expert unpacks in "
+                   f"{t_unpack:.1f} s); scaled to its {d_full} distinct experts and {a_full} assignments")
+        cores = os.cpu_count() if openmp else 1
+        return {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                "build": "OpenMP, all host cores" if openmp else "single thread",
+                "sample": f"{spec.name}: {how}"}
+    finally:
+        oracle.use_openmp(False)
 
 
 class HostOracleLayer:
@@ -190,11 +227,22 @@ class HostOracleLayer:
         self.router_w, self.bias = draw_router(spec, seed)
         self.cache = {}
 
-    def timed_forward(self, orc, x_bits):
-        from workloads.synth import draw_packed_layer_host
+    def _layer(self, orc):
         spec = self.spec
-        layer = orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
-                               spec.top_k, spec.routed_scale, spec.has_shared)
+        return orc.make_layer(spec.hidden, spec.inter, spec.n_experts, spec.n_groups, spec.topk_group,
+                              spec.top_k, spec.routed_scale, spec.has_shared)
+
+    def distinct_experts(self, orc, x_bits):
+        """Experts one oracle call on x_bits unpacks (routed ones plus the shared one)."""
+        idx, _, _, _ = orc.route(self._layer(orc), x_bits, self.router_w, self.bias)
+        return len(set(int(e) for e in idx.reshape(-1))) + (1 if self.spec.has_shared else 0)
+
+    def timed_parts(self, orc, x_bits):
+        """(time of one oracle call on x_bits, time of unpacking its experts
+        alone, number of those experts)."""
+        from workloads.synth import draw_packed_layer_host, tensor_shapes
+        spec = self.spec
+        layer = self._layer(orc)
         idx, _, _, _ = orc.route(layer, x_bits, self.router_w, self.bias)
         n = spec.n_experts + (1 if spec.has_shared else 0)
         used = set(int(e) for e in idx.reshape(-1)) | set(range(spec.n_experts, n))
@@ -207,7 +255,17 @@ class HostOracleLayer:
         d = [self.cache[e][2] if e in used else dummy for e in range(n)]
         t0 = time.perf_counter()
         orc.moe_forward(layer, x_bits, self.router_w, self.bias, g, u, d, self.fmts)
-        return time.perf_counter() - t0
+        t_fwd = time.perf_counter() - t0
+        shapes = tensor_shapes(spec)
+        t0 = time.perf_counter()
+        for e in used:
+            for j in range(3):
+                orc.unpack(int(self.fmts[e, j]), self.cache[e][j], *shapes[j])
+        t_unpack = time.perf_counter() - t0
+        return t_fwd, t_unpack, len(used)
+
+    def timed_forward(self, orc, x_bits):
+        return self.timed_parts(orc, x_bits)[0]
 
 
 class BenchLayer:
@@ -256,20 +314,16 @@ def job_throughput(world: int, tokens_per_step: int, steps: int, ms_max: float) 
     return world * tokens_per_step * steps / (ms_max / 1e3)
 
 
-def run_native(args):
+def measure_layer(spec, K, W, rank=0, world=1, local=0):
+    """One layer workload: K timed steps after W warm-up steps (L2 flushed
+    before each), per-kernel times, end-to-end through host buffers.  Returns
+    (result dict for rank 0 or None, the timed steps' token batches, the
+    timed steps' expert ids)."""
     import torch
     import torch.distributed as dist
-    from workloads import get_config
     from workloads.synth import draw_tokens
 
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
-    spec = get_config(args.config)
-    T, K, W = spec.tokens, args.steps, args.warmup
+    T = spec.tokens
     layer = BenchLayer(spec, seed=rank)
     steps = W + K
     # a fresh token batch per step (decode); prefill cycles through a pool of
@@ -381,9 +435,62 @@ def run_native(args):
             "e2e": {"value": round(job_throughput(world, T, K, e2e_ms_max), 2), "unit": "tokens/s",
                     "h2d_bytes_per_step": int(T * spec.hidden * 2), "d2h_bytes_per_step": int(T * spec.hidden * 4)},
         }
-        if world == 1 and not args.no_cpu_baseline:
-            xs = [x_host[xi(W + i)][:1] for i in range(min(K, 8))]
-            result["cpu_baseline"] = cpu_baseline(HostOracleLayer(spec, seed=0), xs)
+    del layer, x_dev, flush
+    torch.cuda.empty_cache()
+    return result, x_host[xi(W)], idx_host
+
+
+def zipf_histogram(spec, idx_host):
+    """Routed count histogram of a Zipf-skewed workload against its
+    water-filled Zipf target (per expert), as reported beside the line."""
+    from workloads.synth import zipf_ranks, zipf_target_counts
+    T, E, K = spec.tokens, spec.n_experts, spec.top_k
+    steps = idx_host.size // (T * K)
+    counts = np.bincount(idx_host.reshape(-1), minlength=E) / max(steps, 1)
+    target = zipf_target_counts(E, T * K, float(spec.zipf_s), T)[zipf_ranks(spec, 0)]
+    return {"zipf_s": spec.zipf_s, "l1_distance_to_target": round(float(np.abs(counts - target).sum() / (T * K)), 4),
+            "experts_touched": int((counts > 0).sum()), "top_count": float(counts.max()),
+            "top_count_target": float(target.max())}
+
+
+SUB_RECORDS = (("v3_decode_t32_mixed", 50, 5), ("v3_prefill_t2048_zipf", 10, 3))
+
+
+def run_native(args):
+    import torch
+    import torch.distributed as dist
+    from workloads import get_config
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    spec = get_config(args.config)
+    result, x_first, idx_host = measure_layer(spec, args.steps, args.warmup, rank, world, local)
+    if result is not None and spec.zipf_s is not None:
+        result["routing_histogram"] = zipf_histogram(spec, idx_host)
+    if result is not None and world == 1 and not args.no_cpu_baseline:
+        host = HostOracleLayer(spec, seed=0)
+        result["cpu_baseline"] = cpu_baseline(host, x_first, openmp=True)
+        result["cpu_baseline_1thread"] = cpu_baseline(host, x_first, openmp=False)
+    if world == 1 and not args.no_sub_records and args.config == WORKLOAD:
+        # the other workloads of the suite, each with its own roofline, e2e
+        # and oracle baseline (not timed into the headline)
+        subs = []
+        for name, k, w in SUB_RECORDS:
+            sp = get_config(name)
+            r, xf, ih = measure_layer(sp, k, w, rank, world, local)
+            if sp.zipf_s is not None:
+                r["routing_histogram"] = zipf_histogram(sp, ih)
+            if not args.no_cpu_baseline:
+                r["cpu_baseline"] = cpu_baseline(HostOracleLayer(sp, seed=0), xf, openmp=True)
+            subs.append(r)
+        for tokens in (1, 8):
+            subs.append(measure_stack(get_config("v3_stack20"), tokens, 64, 5, rank, world, local,
+                                      cpu=not args.no_cpu_baseline))
+        result["sub_records"] = subs
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
@@ -391,29 +498,18 @@ def run_native(args):
         print(json.dumps(result))
 
 
-def run_stack(args):
+def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
     """A stack of independent V3 layers (each with its own 192 mixed-format
     experts + shared expert, all resident in HBM); one step = one batch of
     fresh tokens through every layer, the layer calls captured once in a CUDA
     graph and replayed.  Weights per step (several GB) far exceed the L2, so no
-    flush is needed between steps."""
+    flush is needed between steps.  Returns the result dict (rank 0) or None."""
     import torch
-    from workloads import get_config
     from workloads.synth import draw_tokens
-    from workloads.configs import packed_bytes
     from dataclasses import replace
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    torch.cuda.set_device(local)
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    base = get_config(args.config)
-    T = args.tokens if args.tokens else base.tokens
     spec = replace(base, tokens=T)
-    L, K, W = spec.n_layers, args.steps, args.warmup
+    L = spec.n_layers
     layers = [BenchLayer(spec, seed=1000 * rank + l) for l in range(L)]
     resident = sum(int(t.numel()) for lay in layers for trip in lay.tensors for t in trip)
     n_pool = max(1, min(W + K, (64 << 20) // (L * T * spec.hidden * 2)))
@@ -491,6 +587,7 @@ def run_stack(args):
             touched += sb["quantized"]
     peak, peak_src = _peaks()
     gbs = touched / (dev_ms / 1e3) / 1e9
+    result = None
     if rank == 0:
         result = {
             "metric": METRIC, "value": round(job_throughput(world, T, K, dev_ms_max), 2), "unit": "tokens/s",
@@ -523,12 +620,31 @@ def run_stack(args):
                                   "traffic": None, "peak_source": peak_src,
                                   "algorithmic_bytes_per_launch": int(per_launch),
                                   "avg_launch_us": round(avg_s * 1e6, 2)}
-        if world == 1 and not args.no_cpu_baseline:
+        if world == 1 and cpu:
             host = HostOracleLayer(spec, seed=0)
-            cb = cpu_baseline(host, [x_host[0, 0][:1]], budget_s=15.0, max_tokens=1)
-            cb["value"] = cb["value"] / L      # one token through the whole stack
-            cb["sample"] = "one token through one layer of the stack, timed, divided by the layer count: " + cb["sample"]
+            cb = cpu_baseline(host, x_host[0, 0], openmp=True)
+            cb["value"] = cb["value"] / L      # a token goes through every layer
+            cb["sample"] = f"one layer of the stack, divided by its {L} layers: " + cb["sample"]
             result["cpu_baseline"] = cb
+    del layers, x_dev, xbuf, graph
+    torch.cuda.empty_cache()
+    return result
+
+
+def run_stack(args):
+    import torch
+    from workloads import get_config
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    base = get_config(args.config)
+    result = measure_stack(base, args.tokens if args.tokens else base.tokens, args.steps, args.warmup, rank, world,
+                           local, cpu=not args.no_cpu_baseline)
+    if result is not None:
         print(json.dumps(result))
     if world > 1:
         import torch.distributed as dist
@@ -537,40 +653,49 @@ def run_stack(args):
 
 
 def run_reference(args):
-    """Reference arm: the oracle as it stands, on the host cores, rank 0."""
+    """Reference arm: the oracle as it stands (its OpenMP build, identical
+    results to the plain one) on the host cores, rank 0 only.  Every step is
+    a fresh batch of the workload; the oracle is timed on a bounded sample of
+    it and scaled to the whole batch (cpu_baseline), the run capped at about
+    150 s of oracle time."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    import oracle
     from workloads import get_config
     from workloads.synth import draw_tokens
-    oracle.build()
     spec = get_config(args.config)
+    T = args.tokens if (args.tokens and spec.n_layers > 1) else spec.tokens
+    if T != spec.tokens:
+        from dataclasses import replace
+        spec = replace(spec, tokens=T)
     host = HostOracleLayer(spec, seed=0)
-    budget_s, done_steps, t_used = 150.0, 0, 0.0
-    # each step is a bounded sample of the workload's tokens (the oracle
-    # handles tokens independently, so tokens/s carries over)
-    n_s = min(spec.tokens, 8)
+    budget_s, t_est, t_real, done_steps = 150.0, 0.0, 0.0, 0
+    last = None
     for i in range(min(args.warmup, 1)):
-        host.timed_forward(oracle, draw_tokens(1000 + i, n_s, spec.hidden))
+        cpu_baseline(host, draw_tokens(1000 + i, T, spec.hidden), budget_s=4.0, openmp=True)
     for i in range(args.steps):
-        t_used += host.timed_forward(oracle, draw_tokens(1000 + args.warmup + i, n_s, spec.hidden))
+        w0 = time.perf_counter()
+        last = cpu_baseline(host, draw_tokens(1000 + args.warmup + i, T, spec.hidden), budget_s=6.0, openmp=True)
+        t_real += time.perf_counter() - w0
+        t_est += T / last["value"]
         done_steps += 1
-        if t_used > budget_s:
+        if t_real > budget_s:
             break
-    value = done_steps * n_s / t_used
+    value = done_steps * T / t_est
     if spec.n_layers > 1:
         value /= spec.n_layers      # a token of the stack goes through every layer
+    cb = dict(last)
+    cb["value"] = round(value, 4)
+    cb["sample"] = f"{done_steps} step(s); last: " + cb["sample"]
     line = {"metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": 1, "steps": done_steps,
-            "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t_used / done_steps * 1e3, 2),
+            "requested_steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(t_est / done_steps * 1e3 * (spec.n_layers if spec.n_layers > 1 else 1), 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": f"{spec.name} (oracle: plain single-threaded C, fp64 FFN"
-                                   + (f"; one layer timed per token, value divided by the {spec.n_layers} layers)"
-                                      if spec.n_layers > 1 else ")")},
-            "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": f"{done_steps} step(s) of {n_s} of the workload's {spec.tokens} token(s) "
-                                       f"each (time budget {budget_s} s)"},
+            "config": {"workload": f"{spec.name} (oracle: plain C, fp64 FFN, OpenMP build on {os.cpu_count()} "
+                                   f"host cores" + (f"; one layer timed, value divided by the {spec.n_layers} "
+                                                    f"layers)" if spec.n_layers > 1 else ")")},
+            "cpu_baseline": cb,
             "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 
@@ -583,6 +708,8 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--config", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sub-records", action="store_true",
+                    help="only the headline workload (no per-config sub-records)")
     ap.add_argument("--tokens", type=int, default=0, help="tokens per layer call for the layer-stack workload")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -192,7 +192,8 @@ int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const v
  * give up a wait on a pipeline barrier after a time limit instead of
  * hanging; they then set a bit in an error word of the workspace (cleared at
  * the start of every forward call) and their outputs are not valid.  Bits:
- * 1 / 2 a decode GEMV consumer / producer gave up a wait, 4 a prefill GEMM
+ * 1 / 2 a decode GEMV consumer / producer gave up a wait, 32 a decode down
+ * item gave up waiting for its expert's SwiGLU output, 4 a prefill GEMM
  * wait, 8 a tcgen05 GEMV wait, 16 a prefill SwiGLU output beyond the fp16
  * range (see moe_quant_forward).  This call
  * waits for the stream (cudaStreamSynchronize), reads the word and returns

@@ -1,4 +1,4 @@
-// Expert FFN kernels for decode-sized batches (arXiv 2509.25689 Fig. 1: a
+// Expert FFN kernel for decode-sized batches (arXiv 2509.25689 Fig. 1: a
 // shared expert plus router-weighted routed SwiGLU experts; each expert
 // tensor stored in its own k-quant style block format, Sec. 3.3).
 //
@@ -13,19 +13,29 @@
 //     per lane so nothing is masked in the loop;
 //   D (16 rows x 8 cols) = per-(row, sub-block) partial dot products, so the
 //     sub-block scales and mins are applied once per tile in fp32.
-// Work is cut into items (gate/up: 32 rows x all superblocks of gate and of
-// up; down: two 32-row blocks x all superblocks; of one expert x up to 4
-// tokens), claimed by the persistent CTAs (one per SM) from a per-call
-// counter.  The packed layout keeps any superblock range of a 32-row tile
-// contiguous in every plane, so a dedicated producer warp streams each item
-// through a shared-memory ring (3 x 64 KB for gate/up, 4 x 48 KB for down)
-// with 1D bulk (TMA) copies that complete on mbarriers; 8 consumer warps (all
-// 32 rows x every 8th superblock of a stage each, the columns rotated from
-// stage to stage) run the tensor-core math.  At the end of an item the CTA
-// reduces its warps' sums in a fixed
-// order (SwiGLU and the prepared h for gate/up, one partial output row block
-// per assignment for down), so results are deterministic.  Every wait on an
-// mbarrier is bounded (about 1 s) and reports to an error word.
+// One persistent kernel runs the whole expert FFN of a call.  Work is cut
+// into items claimed from one per-call counter in this order: the shared
+// expert's gate/up items (they need no routing result and start while the
+// routing kernel runs), the routed experts' gate/up items, the shared
+// expert's down items, the routed experts' down items.  A gate/up item is 32
+// rows x all superblocks of gate and of up, a down item two 32-row blocks x
+// all superblocks, of one expert x up to 4 tokens.  The SwiGLU output h of an
+// expert slot is published per 32-row block (the item's finisher writes it,
+// fences, and increments the slot's counter); a down item's producer streams
+// its weights at once and copies h only when the slot's counter says every
+// block is in, so down items of the first experts overlap the last gate/up
+// items and no CTA idles at a kernel boundary.  Every gate/up item is claimed
+// before any down item, so each awaited block is held by a CTA that finishes
+// it without waiting on anything.
+// The packed layout keeps any superblock range of a 32-row tile contiguous in
+// every plane, so a dedicated producer warp streams each item through a
+// shared-memory ring with 1D bulk (TMA) copies that complete on mbarriers; the
+// consumer warps (all 32 rows x every kCols-th superblock of a stage each,
+// the columns rotated from stage to stage) run the tensor-core math.  At the
+// end of an item the CTA reduces its warps' sums in a fixed order (SwiGLU and
+// the prepared h for gate/up, one partial output row block per assignment
+// for down), so results are deterministic.  Every wait (mbarriers, the h
+// counters) is bounded (about 1 s) and reports to an error word.
 #include <cuda_fp16.h>
 
 #include "mq_actprep.cuh"
@@ -128,33 +138,47 @@ __device__ __forceinline__ uint32_t lds8(uint32_t a) {
 }
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
-constexpr int kConsumers = 8;                       // consumer warps
+#ifndef MQ_DECODE_CONSUMERS
+#define MQ_DECODE_CONSUMERS 8
+#endif
+#ifndef MQ_DECODE_SLOTS
+#define MQ_DECODE_SLOTS 4
+#endif
+constexpr int kConsumers = MQ_DECODE_CONSUMERS;     // consumer warps
 constexpr int kNT = kConsumers >= 16 ? 1 : 2;       // 16-row MMA tiles per warp (of the stage's two)
 constexpr int kCols = kConsumers * kNT / 2;         // superblock columns the warps are spread over
-constexpr int kRedBufs = kConsumers >= 16 ? 1 : 2;  // item-end reduction buffers (smem budget)
 constexpr int kThreads = (kConsumers + 1) * 32;     // + one producer warp
 constexpr int kProducerWarp = kConsumers;
-// Ring: 3 slots of 64 KB (gate/up: Q8_0 stages of the shared expert are
-// 61 KB) or 4 of 48 KB (down: Q3_K stages are 37 KB, more of them in flight)
-constexpr int kNSTmax = 4;
-__host__ __device__ constexpr int ring_slots(bool down) { return down ? 4 : 3; }
-__host__ __device__ constexpr int slot_bytes(bool down) { return down ? 48 * 1024 : 64 * 1024; }
+// Ring of kNST slots (4 x 48 KB: Q3_K down stages are 37 KB, Q2_K gate/up
+// stages of 14 superblocks 47 KB, Q8_0 stages of 5 superblocks 44 KB)
+constexpr int kNST = MQ_DECODE_SLOTS;
 constexpr int kRingBytes = 192 * 1024;
-static_assert(ring_slots(false) * slot_bytes(false) == kRingBytes && ring_slots(true) * slot_bytes(true) == kRingBytes,
-              "ring size");
+constexpr int kSlotBytes = kRingBytes / kNST;
 constexpr int kStageSb = 16;                        // superblocks per stage (Q8_0: 8), fewer if over budget
-constexpr int kMaxCachedAssign = 2048;              // routed assignments cached in smem
-constexpr uint32_t kErrFull = 1u, kErrEmpty = 2u;
+constexpr int kMaxCachedAssign = 1024;              // routed assignments cached in smem
+#ifndef MQ_PREROUTE_DEPTH
+#define MQ_PREROUTE_DEPTH 3
+#endif
+constexpr int kPreRouteDepth = MQ_PREROUTE_DEPTH;   // stages in flight before the routing result is in
+static_assert(kPreRouteDepth >= 1 && kPreRouteDepth <= kNST, "pre-routing depth");
+constexpr uint32_t kErrFull = 1u, kErrEmpty = 2u, kErrReady = 32u;
 // named barrier 1: the consumer warps only
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers * 32) : "memory"); }
-
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 
 // stage header written by the producer (one per ring slot); the stage's
-// byte layout is geo[fmt - 1][ntok - 1]
+// byte layout is geo[down][fmt - 1][ntok - 1]
 struct __align__(16) Hdr {
     int32_t item, j, nst, s0;
-    int32_t ks, fmt, tensor, ntok;
-    int32_t rb, e, shared, pad;
+    int32_t ks, fmt, tensor, ntok;   // tensor: 0 gate, 1 up, 2 down rows rb, 3 down rows rb + 1
+    int32_t rb, e, shared, slot;
     int32_t asg[kDecodeTok];
 };
 
@@ -185,45 +209,43 @@ __host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok, int stage_by
     return ks;
 }
 
-// per-CTA cache of the routing result (slot -> expert, first entry, tokens)
+// per-CTA cache of the routing result: slot -> expert, first entry, tokens,
+// and the items before each slot (gate/up and down)
 struct SlotCache {
     int32_t e[kMaxExperts + 1], first[kMaxExperts + 1], ntot[kMaxExperts + 1];
-    int32_t pre[kMaxExperts + 2];
-    const uint8_t* ptr[kMaxExperts + 1];   // the streamed tensor(s) of the slot's expert (gate or down)
-    const uint8_t* ptr_up[kMaxExperts + 1];
-    uint8_t fmt[kMaxExperts + 1][2];
+    int32_t pre_gu[kMaxExperts + 2], pre_dn[kMaxExperts + 2];
 };
 
-// Stage geometry of one (format, tokens per item) pair, computed once per CTA
-// so the producer does no layout arithmetic per stage.
+// Stage geometry of one (kind, format, tokens per item), computed once per
+// launch on the host so the producer does no layout arithmetic per stage.
 struct Geo {
-    int64_t pl[4];       // plane starts in the tensor
-    int64_t rbstr[4];    // bytes per 32-row block in each plane
-    int per, nst, npl;   // superblocks per stage, stages per tensor, planes
-    int woff[4], cstr[4];// plane regions in the stage, bytes per superblock
-    int tok0, tstride, tx, ts;
+    int32_t pl[4];       // plane starts in the tensor
+    int32_t rbstr[4];    // bytes per 32-row block in each plane
+    int32_t woff[4], cstr[4];  // plane regions in the stage, bytes per superblock
+    int32_t tok0, tstride, tx, ts;   // token pieces: first byte, bytes per token, fragments, statistics
+    int16_t per, nst, npl, pad;      // superblocks per stage, stages per tensor, planes
 };
+static_assert(sizeof(Geo) == 88, "geometry record");
 
-// Stage geometry of (format, tokens per item) for the gate/up (down = false)
-// or down kernel; the host computes it once per launch.
 __host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int fmt, int ntok) {
     const int nsb = down ? (d.I + 255) / 256 : (d.H + 255) / 256;
     const TensorLayout L = tensor_layout(fmt, down ? d.H : d.I, down ? d.I : d.H);
     const PlaneBytes pb = plane_bytes(fmt);
     const int bmul = fmt == kQ80 ? 8 : 1;
-    G.per = stage_sb(fmt, ntok, slot_bytes(down));
-    G.nst = (nsb + G.per - 1) / G.per;
-    G.npl = pb.n;
+    G.per = (int16_t)stage_sb(fmt, ntok, kSlotBytes);
+    G.nst = (int16_t)((nsb + G.per - 1) / G.per);
+    G.npl = (int16_t)pb.n;
     int at = 0;
     for (int pl = 0; pl < 4; ++pl) {
         G.woff[pl] = at;
         G.cstr[pl] = pl < pb.n ? 32 * bmul * pb.b[pl] : 0;
-        G.pl[pl] = L.plane[pl];
-        G.rbstr[pl] = pl < pb.n ? L.blocks_per_row * 32 * pb.b[pl] : 0;
+        G.pl[pl] = (int32_t)L.plane[pl];
+        G.rbstr[pl] = pl < pb.n ? (int32_t)(L.blocks_per_row * 32 * pb.b[pl]) : 0;
         if (pl < pb.n) at += (32 * bmul * G.per * pb.b[pl] + 127) & ~127;
     }
     const TokLay tl = tok_lay(fmt, G.per);
     G.tok0 = at; G.tstride = tl.stride; G.tx = tl.x; G.ts = tl.s;
+    G.pad = 0;
 }
 
 struct DecodeArgs {
@@ -231,35 +253,44 @@ struct DecodeArgs {
     int nsbx, nsbi;          // superblocks along hidden / inter
     const __half* xq; const float* xs;   // prepared tokens
     __half* hq; float* hs;               // prepared SwiGLU outputs (per assignment)
-    const int32_t* offsets; const int32_t* perm; const int32_t* active; const float* wts;
+    const int32_t* perm; const float* wts;
     const Plan* plan;
     float* pdn;              // [A][H]
-    uint32_t* next;          // [2] item counters
+    uint32_t* next;          // item counter
+    uint32_t* hready;        // [kMaxExperts + 1] per slot: published h blocks (tokens x 32-row blocks)
+    const uint32_t* logits_done;   // logits CTAs done (their prepared tokens are written)
+    const uint32_t* route_ready;   // non-zero once the routing result is written
+    uint32_t n_logit_ctas;
     uint32_t* err;
     uint64_t wait_ns;        // limit of every bounded wait
-    int fail_first_stage;    // test hook: the gate/up producer posts nothing for its first stage
-    float* out;
-    Geo geo[4][kDecodeTok];  // stage geometry per (format, tokens), computed on the host
+    int fail_first_stage;    // test hook: the producer posts nothing for its first stage
+    Geo geo[2][4][kDecodeTok];   // [down][format][tokens], computed on the host
 };
 
 struct ItemDesc {            // decoded item (producer side)
-    int e, rb, tg, ntok, shared, nst0, nst;
+    int e, rb, tg, ntok, shared, nst0, nst, down, slot;
     int vec[kDecodeTok], asg[kDecodeTok];
 };
 
-template <bool kDown>
+// Item id -> slot, rows, tokens.  Ids [0, n_gu) are gate/up items, [n_gu,
+// n_gu + n_dn) down items; both in slot order (the shared expert first).
 __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache& sc, const int32_t* s_perm,
-                                            const Geo (*geo)[kDecodeTok], int n_slots, int id, int& cursor,
-                                            ItemDesc& it, int& slot) {
-    while (cursor + 1 < n_slots && sc.pre[cursor + 1] <= id) ++cursor;
+                                            int n_slots, int n_gu, int id, int& cur_gu, int& cur_dn,
+                                            ItemDesc& it) {
+    const bool down = id >= n_gu;
+    const int32_t* pre = down ? sc.pre_dn : sc.pre_gu;
+    const int lid = down ? id - n_gu : id;
+    int& cursor = down ? cur_dn : cur_gu;   // ids grow, so each walk only moves forward
+    while (cursor + 1 < n_slots && pre[cursor + 1] <= lid) ++cursor;
     const int p = cursor;
-    slot = p;
-    const int local = id - sc.pre[p];
+    it.slot = p;
+    it.down = down ? 1 : 0;
+    const int local = lid - pre[p];
     const Dims& d = A.d;
     // gate/up items: one 32-row block of gate and up; down items: two 32-row blocks
-    const int nrb = kDown ? d.H / 64 : d.I / 32;
+    const int nrb = down ? d.H / 64 : d.I / 32;
     it.tg = local / nrb;
-    it.rb = (local - it.tg * nrb) * (kDown ? 2 : 1);
+    it.rb = (local - it.tg * nrb) * (down ? 2 : 1);
     it.e = sc.e[p];
     it.shared = p < d.has_shared;
     it.ntok = min(kDecodeTok, sc.ntot[p] - it.tg * kDecodeTok);
@@ -276,10 +307,10 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
             }
         }
         it.asg[j] = a;
-        it.vec[j] = kDown ? a : t;
+        it.vec[j] = down ? a : t;
     }
-    it.nst0 = geo[sc.fmt[p][0] - 1][it.ntok - 1].nst;
-    it.nst = kDown ? 2 * it.nst0 : it.nst0 + geo[sc.fmt[p][1] - 1][it.ntok - 1].nst;
+    it.nst0 = 0;
+    it.nst = 0;
 }
 
 // ---- consumer math: one warp = the 32 rows of the stage (two 16-row MMA
@@ -364,11 +395,13 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
                                  (sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk, XA[gm][m], XB[gm][m]);
             }
         } else {
-            // Q3_K: the high bit of pair m (bit m of its half of the hmask word)
-            // goes right above the pair's 2-bit code, so one operand carries the
-            // 3-bit code (low2 + 4 hbit) at the code's positional power.  Bit 10
-            // of an fp16 still has the subnormal ulp (2^-24), so position 10
-            // (m = 4) stays linear.
+            // Q3_K: code = low2 + 4 hbit.  The low two bits go through the same
+            // MMAs as Q2_K; the high bits get MMAs of their own into the same
+            // accumulators: the high bit of pair m sits at bit m (and 16 + m)
+            // of its half of the hmask word (the second sub-block of a word one
+            // byte up, shifted down once), so one AND makes an fp16 pair
+            // hbit * 2^(m-24), and the activation operand is scaled by
+            // 4 * 2^(pos(m) - m) (exact powers of two) to weigh it 4 x.
             uint32_t ha[2][NR], hb[2][NR];
 #pragma unroll
             for (int gm = 0; gm < 2; ++gm)
@@ -376,21 +409,34 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
                 for (int i = 0; i < NR; ++i) { ha[gm][i] = gm ? hv[i].y : hv[i].x; hb[gm][i] = ha[gm][i] >> 8; }
 #pragma unroll
             for (int m = 0; m < 8; ++m) {
-                const int pos = m <= 4 ? 2 * m : 2 * (m - 5);
-                const uint32_t mk = 0x00030003u << pos, mh = 0x00040004u << pos;
+                const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
                 const bool sh = m > 4;
-                // hbit m from bit m to bit pos + 2
-                auto hsh = [&](uint32_t w) { return (m <= 4 ? (w << (m + 2)) : (w >> (8 - m))) & mh; };
 #pragma unroll
                 for (int gm = 0; gm < 2; ++gm)
 #pragma unroll
                     for (int tl = 0; tl < NT; ++tl)
-                        mma16816(T.DD[tl][gm][m & 1],
-                                 ((sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk) | hsh(ha[gm][2 * tl]),
-                                 ((sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk) | hsh(ha[gm][2 * tl + 1]),
-                                 ((sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk) | hsh(hb[gm][2 * tl]),
-                                 ((sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk) | hsh(hb[gm][2 * tl + 1]),
-                                 XA[gm][m], XB[gm][m]);
+                        mma16816(T.DD[tl][gm][m & 1], (sh ? sa[gm][2 * tl] : qa[gm][2 * tl]) & mk,
+                                 (sh ? sa[gm][2 * tl + 1] : qa[gm][2 * tl + 1]) & mk,
+                                 (sh ? sbb[gm][2 * tl] : qb[gm][2 * tl]) & mk,
+                                 (sh ? sbb[gm][2 * tl + 1] : qb[gm][2 * tl + 1]) & mk, XA[gm][m], XB[gm][m]);
+            }
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const uint32_t mh = 0x00010001u << m;
+                // 4 * 2^(pos(m) - m): 2^(m+2) for m <= 4, 2^(m-8) above (fp16 bits)
+                const int e = m <= 4 ? m + 2 : m - 8;
+                const uint32_t sc16 = (uint32_t)(15 + e) << 10;
+                const __half2 scl = __halves2half2(__ushort_as_half((unsigned short)sc16), __ushort_as_half((unsigned short)sc16));
+#pragma unroll
+                for (int gm = 0; gm < 2; ++gm) {
+                    const __half2 xa = __hmul2(*reinterpret_cast<const __half2*>(&XA[gm][m]), scl);
+                    const __half2 xb2 = __hmul2(*reinterpret_cast<const __half2*>(&XB[gm][m]), scl);
+                    const uint32_t ua = *reinterpret_cast<const uint32_t*>(&xa), ub = *reinterpret_cast<const uint32_t*>(&xb2);
+#pragma unroll
+                    for (int tl = 0; tl < NT; ++tl)
+                        mma16816(T.DD[tl][gm][(m + 1) & 1], ha[gm][2 * tl] & mh, ha[gm][2 * tl + 1] & mh,
+                                 hb[gm][2 * tl] & mh, hb[gm][2 * tl + 1] & mh, ua, ub);
+                }
             }
         }
     } else if (FMT == kQ4K) {
@@ -457,11 +503,16 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
     auto rec_of = [&](int i) { return rbase + 16 * (i >> 1) + 8 * (i & 1); };
 
     if (FMT == kQ2K || FMT == kQ3K) {
-        // slot-ordered scale word of each row: bytes b = 2*group + col
+        // slot-ordered scale fields of each row: slot 4t + b (b = 2 * group + col)
+        // holds the lane's sub-block of D[group][col].  Fields are turned into
+        // fp16 pairs (b0, b2) / (b1, b3) whose values are field * 2^-24 (masked
+        // bits in the mantissa of an fp16 subnormal), then widened to fp32; the
+        // 2^24 is folded into d (d * 2^24 <= 2^40, exact).
         const float cf0 = ldsf(sb + 4 * (kStatC + t)), cf1 = ldsf(sb + 4 * (kStatC + 4 + t));
         const uint4 Su = lds128(sb + 4 * (kStatS16 + 4 * t));
         const float S[4] = {__uint_as_float(Su.x), __uint_as_float(Su.y), __uint_as_float(Su.z),
                             __uint_as_float(Su.w)};
+        auto h2pair = [](uint32_t bits) { return __half22float2(*reinterpret_cast<const __half2*>(&bits)); };
 #pragma unroll
         for (int i = 0; i < NR; ++i) {
             const int tl = i >> 1, hl = i & 1;
@@ -472,25 +523,41 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
                 for (int cc = 0; cc < 2; ++cc)
                     D[gm][cc] = T.DD[tl][gm][0][2 * hl + cc] + T.DD[tl][gm][1][2 * hl + cc];
             const int rec = rec_of(i);
-            const float d = h2f(lds16(st + w0 + rec * 2));
+            const float d = h2f(lds16(st + w0 + rec * 2)) * 16777216.0f;
             if (FMT == kQ2K) {
-                const float dm = h2f(lds16(st + w1 + rec * 2));
+                // byte b = sc | m << 4; bytes 1 and 3 moved down to bytes 0 and 2
+                const float dm = h2f(lds16(st + w1 + rec * 2)) * 1048576.0f;   // m sits 4 bits up: 2^-20
                 const uint32_t f = lds32(st + w2 + rec * 16 + 4 * t);
-                const uint32_t sc4 = f & 0x0F0F0F0Fu, m4 = (f >> 4) & 0x0F0F0F0Fu;
-                const float a0 = fmaf(u8f(sc4, 1), D[0][1], u8f(sc4, 0) * D[0][0]);
-                const float a1 = fmaf(u8f(sc4, 3), D[1][1], u8f(sc4, 2) * D[1][0]);
-                const float am = fmaf(u8f(m4, 3), S[3], fmaf(u8f(m4, 2), S[2], fmaf(u8f(m4, 1), S[1], u8f(m4, 0) * S[0])));
+                const uint32_t fo = __byte_perm(f, 0u, 0x7371u);
+                const float2 s02 = h2pair(f & 0x000F000Fu), s13 = h2pair(fo & 0x000F000Fu);
+                const float2 m02 = h2pair(f & 0x00F000F0u), m13 = h2pair(fo & 0x00F000F0u);
+                const float a0 = fmaf(s13.x, D[0][1], s02.x * D[0][0]);
+                const float a1 = fmaf(s13.y, D[1][1], s02.y * D[1][0]);
+                const float am = fmaf(m13.y, S[3], fmaf(m02.y, S[2], fmaf(m13.x, S[1], m02.x * S[0])));
                 acc[i] += fmaf(d, fmaf(cf1, a1, cf0 * a0), -dm * am);
             } else {
+                // 6-bit scale s (stored s + 32): low nibble of slot u at bits 4u..4u+3
+                // of bytes 0-7, high two bits at bits 2u..2u+1 of bytes 8-11
                 const uint32_t sp = st + w1 + rec * 12;
-                const uint32_t f = lds16(sp + 2 * t) | (lds8(sp + 8 + t) << 16);
-                float a = 0.0f;
-#pragma unroll
-                for (int b = 0; b < 4; ++b) {
-                    const float sv = (float)((int)(((f >> (4 * b)) & 15u) | (((f >> (16 + 2 * b)) & 3u) << 4)) - 32);
-                    const float P = fmaf(D[b >> 1][b & 1], (b >> 1) ? cf1 : cf0, -4.0f * S[b]);
-                    a = fmaf(sv, P, a);
-                }
+                const uint32_t lo = lds16(sp + 2 * t), hi = lds8(sp + 8 + t);
+                const uint32_t u = __byte_perm(lo, 0u, 0x7170u);   // halves: n0 | n1 << 4, n2 | n3 << 4
+                const uint32_t v = __byte_perm(hi, 0u, 0x7070u);   // both halves: h0 | h1 << 2 | h2 << 4 | h3 << 6
+                // (n0 + 16 h0, n2 + 16 h2) and (n1 + 16 h1, n3 + 16 h3), exact in fp16
+                // subnormals (the 2-bit fields weighed up to bit 4 by the multipliers),
+                // then minus 32
+                const __half2 c32 = __halves2half2(__ushort_as_half((unsigned short)32), __ushort_as_half((unsigned short)32));
+                const uint32_t uA = u & 0x000F000Fu, uB = (u >> 4) & 0x000F000Fu;
+                const __half2 lA = *reinterpret_cast<const __half2*>(&uA);
+                const __half2 lB = *reinterpret_cast<const __half2*>(&uB);
+                const uint32_t hA = v & 0x00300003u, hB = v & 0x00C0000Cu;
+                const __half2 mA = __halves2half2(__float2half(16.0f), __float2half(1.0f));
+                const __half2 mB = __halves2half2(__float2half(4.0f), __float2half(0.25f));
+                const __half2 sA = __hsub2(__hfma2(*reinterpret_cast<const __half2*>(&hA), mA, lA), c32);
+                const __half2 sB = __hsub2(__hfma2(*reinterpret_cast<const __half2*>(&hB), mB, lB), c32);
+                const float2 vA = __half22float2(sA), vB = __half22float2(sB);   // slots (0, 2), (1, 3)
+                const float P0 = fmaf(D[0][0], cf0, -4.0f * S[0]), P1 = fmaf(D[0][1], cf0, -4.0f * S[1]);
+                const float P2 = fmaf(D[1][0], cf1, -4.0f * S[2]), P3 = fmaf(D[1][1], cf1, -4.0f * S[3]);
+                const float a = fmaf(vB.y, P3, fmaf(vA.y, P2, fmaf(vB.x, P1, vA.x * P0)));
                 acc[i] = fmaf(d, a, acc[i]);
             }
         }
@@ -546,30 +613,31 @@ __device__ __forceinline__ void tile_cols(const Geo& h, uint32_t st, int col, in
     }
 }
 
+
 // MT: most tokens an item of this launch carries (1 when the call has one token)
-template <bool kDown, int MT>
+template <int MT>
 __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant__ ExpertTab tab,
                                                           const __grid_constant__ DecodeArgs A) {
     extern __shared__ __align__(128) uint8_t smem[];
+    constexpr int kRedBufs = MT == 1 ? 2 : 1;          // item-end reduction buffers (smem budget)
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
-    constexpr int kNST = ring_slots(kDown), kStageBytes = slot_bytes(kDown);
-    __shared__ __align__(8) uint64_t bars[2 * kNSTmax];
-    __shared__ Hdr hdr[kNSTmax];
-    __shared__ float red[kRedBufs][kConsumers][2][kDecodeTok][32];
-    __shared__ int s_posted[kNSTmax];   // last stage index posted to each ring slot
+    __shared__ __align__(8) uint64_t bars[2 * kNST];
+    __shared__ Hdr hdr[kNST];
+    __shared__ float red[kRedBufs][kConsumers][2][MT][32];
+    __shared__ int s_posted[kNST];   // last stage index posted to each ring slot
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
     __shared__ int s_touch;
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
-    __shared__ Geo geo[4][kDecodeTok];
+    __shared__ Geo geo[2][4][kDecodeTok];
     const Dims& d = A.d;
     // ---- set-up that does not depend on the routing result runs before the
     // wait for the previous kernel (overlapping its tail)
     {
         // stage geometry (host-computed) into shared memory, one word per thread
         static_assert(sizeof(geo) % 4 == 0, "geometry table");
-        const uint32_t* src = reinterpret_cast<const uint32_t*>(&A.geo[0][0]);
-        uint32_t* dst = reinterpret_cast<uint32_t*>(&geo[0][0]);
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(&A.geo[0][0][0]);
+        uint32_t* dst = reinterpret_cast<uint32_t*>(&geo[0][0][0]);
         for (int i = threadIdx.x; i < (int)(sizeof(geo) / 4); i += kThreads) dst[i] = src[i];
     }
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
@@ -578,8 +646,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     if (threadIdx.x == 0) s_fail = 0;
     {
         // Touch the expert table (a kernel parameter) once on this SM, so the
-        // per-slot pointer lookups made after the routing result arrives (one
-        // distinct expert per lane) hit the constant cache.
+        // per-item pointer lookups made after the routing result arrives hit
+        // the constant cache.
         uintptr_t v = 0;
         for (int i = threadIdx.x; i < 3 * (d.E + 1); i += kThreads) v |= reinterpret_cast<uintptr_t>(tab.p[i / 3][i % 3]);
         for (int i = threadIdx.x; i < d.E + 1; i += kThreads) v |= (uintptr_t)tab.fmt[i][0] << 8;
@@ -598,19 +666,12 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     // the wait for the routing kernel.  (The tokens' prepared activations come
     // from the logits kernel, which completed before the routing kernel let
     // this grid launch.)
-    const int n_sh_items = (!kDown && d.has_shared) ? (d.I / 32) * ((d.T + kDecodeTok - 1) / kDecodeTok) : 0;
+    const int n_sh_items = d.has_shared ? (d.I / 32) * ((d.T + kDecodeTok - 1) / kDecodeTok) : 0;
     if (threadIdx.x == 0 && n_sh_items > 0) {
-        sc.pre[0] = 0; sc.pre[1] = n_sh_items;
+        sc.pre_gu[0] = 0; sc.pre_gu[1] = n_sh_items;
         sc.e[0] = d.E; sc.first[0] = 0; sc.ntot[0] = d.T;
-        sc.ptr[0] = tab.p[d.E][0]; sc.ptr_up[0] = tab.p[d.E][1];
-        sc.fmt[0][0] = tab.fmt[d.E][0]; sc.fmt[0][1] = tab.fmt[d.E][1];
     }
     __syncthreads();
-    // The down kernel lets its successor (the combine) launch right away; the
-    // gate/up kernel only once it holds the routing result (below), so that
-    // the down kernel, launched after that, may read the routing result
-    // before its own wait.
-    if (kDown) pdl_launch();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
 
@@ -621,53 +682,80 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // most one copy: lanes 0..3 a weight plane, lanes 4.. one piece of one
         // token (family fragments or statistics).  A stage then only advances
         // the source by the stage's first superblock.
-        const VecSrc vs = kDown ? VecSrc{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi}
-                                : VecSrc{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
-        int p_cursor = 0, p_q = 0;
+        const VecSrc vx{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
+        const VecSrc vh{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi};
+        int cur_gu = 0, cur_dn = 0, p_q = 0;
         // weights are read once per call: evict-first in L2, so they do not
-        // displace the activations, h and partial outputs the kernels share
+        // displace the activations, h and partial outputs the kernel shares
         const uint64_t wpol = evict_first_policy();
-        const int p_nsb = vs.nsb;
         ItemDesc P;
-        int pslot = 0;
+        int fmt0 = 1, fmt1 = 1;
         // the routing result: slot table (one level of independent loads; the
         // plan holds each slot's expert, first entry and token count) and the
         // cached permutation
-        int n_slots = n_sh_items > 0 ? 1 : 0, n_items = n_sh_items;
+        int n_slots = n_sh_items > 0 ? 1 : 0, n_gu = n_sh_items, n_items = n_sh_items;
         bool routed = false;
-        // gate/up: the routing kernel is the predecessor, wait for it.  down:
-        // the routing result is two kernels back (complete before the gate/up
-        // kernel let this grid launch); only h, from the gate/up kernel, needs
-        // the wait, taken before the first copy of h (deps below).
-        bool deps = !kDown;
-        auto wait_routing = [&]() {
-            if (!kDown) pdl_wait();
-            // read through L2 (ld.global.cg): the down kernel reads before its
-            // wait, and an SM's L1 may still hold lines of an earlier call
-            n_slots = __ldcg(&A.plan->n_slots);
-            // one pass per 32 slots (one for a decode call): the pass's loads
-            // go out together, then the stores
-            for (int i = lane; i <= n_slots; i += 32) {
-                const int pre = __ldcg(kDown ? &A.plan->pre_dn[i] : &A.plan->pre_gu[i]);
-                int e = 0, first = 0, ntot = 0;
-                if (i < n_slots) {
-                    e = __ldcg(&A.plan->slot_e[i]);
-                    first = __ldcg(&A.plan->slot_first[i]);
-                    ntot = __ldcg(&A.plan->slot_ntot[i]);
+        // bounded acquire-spin on a word another kernel publishes with release
+        auto wait_word = [&](const uint32_t* wp, uint32_t target) {
+            if (lane == 0 && ld_acquire(wp) < target) {
+                const uint64_t t0 = global_ns();
+                // polled with a back-off: every CTA's producer polls the same word
+                while (ld_acquire(wp) < target) {
+                    if (global_ns() - t0 > A.wait_ns) { atomicOr(A.err, kErrReady); s_fail = 1; break; }
+                    __nanosleep(256);
                 }
-                sc.pre[i] = pre;
+            }
+            __syncwarp();
+            (void)ld_acquire(wp);   // every lane acquires before its own reads and copies
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+        };
+        bool tokens_in = false;   // the logits kernel's prepared tokens are written
+        auto wait_routing = [&]() {
+            // the routing result: published by the last CTA of the logits kernel
+            wait_word(A.route_ready, 1u);
+            tokens_in = true;   // published after every logits CTA counted itself
+            // read through L2 (ld.global.cg): an SM's L1 may still hold lines
+            // of an earlier call
+            // The slot count and the first 32 slots' entries (every slot of a
+            // call with at most 31 active experts) and the first 128 routed
+            // entries of the permutation go out as one batch of independent
+            // loads (one round trip); later passes only for larger calls.
+            const int n_routed = min(d.T * d.K, kMaxCachedAssign);
+            const int ns0 = __ldcg(&A.plan->n_slots);
+            int pg0 = __ldcg(&A.plan->pre_gu[lane]), pd0 = __ldcg(&A.plan->pre_dn[lane]);
+            int e0 = __ldcg(&A.plan->slot_e[lane]), f0 = __ldcg(&A.plan->slot_first[lane]);
+            int nt0 = __ldcg(&A.plan->slot_ntot[lane]);
+            int pv0[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = 32 * u + lane;
+                pv0[u] = i < n_routed ? __ldcg(A.perm + i) : 0;
+            }
+            n_slots = ns0;
+            for (int i = lane; i <= n_slots; i += 32) {
+                int pg = pg0, pd = pd0, e = e0, first = f0, ntot = nt0;
+                if (i >= 32) {
+                    pg = __ldcg(&A.plan->pre_gu[i]); pd = __ldcg(&A.plan->pre_dn[i]);
+                    if (i < n_slots) {
+                        e = __ldcg(&A.plan->slot_e[i]);
+                        first = __ldcg(&A.plan->slot_first[i]);
+                        ntot = __ldcg(&A.plan->slot_ntot[i]);
+                    }
+                }
+                sc.pre_gu[i] = pg;
+                sc.pre_dn[i] = pd;
                 if (i < n_slots) {
                     sc.e[i] = e;
                     sc.first[i] = first;
                     sc.ntot[i] = ntot;
-                    sc.ptr[i] = tab.p[e][kDown ? 2 : 0];
-                    sc.ptr_up[i] = tab.p[e][1];
-                    sc.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
-                    sc.fmt[i][1] = tab.fmt[e][1];
                 }
             }
-            const int n_routed = min(d.T * d.K, kMaxCachedAssign);
-            for (int i0 = 0; i0 < n_routed; i0 += 128) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = 32 * u + lane;
+                if (i < n_routed) s_perm[i] = pv0[u];
+            }
+            for (int i0 = 128; i0 < n_routed; i0 += 128) {
                 int v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
@@ -681,29 +769,37 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 }
             }
             __syncwarp();
-            n_items = sc.pre[n_slots];
+            n_gu = sc.pre_gu[n_slots];
+            n_items = n_gu + sc.pre_dn[n_slots];
             routed = true;
-            if (!kDown) pdl_launch();
+            pdl_launch();
         };
         if (n_sh_items == 0) wait_routing();
-        // items are handed out by a global counter (zeroed per call), in slot
-        // order: the shared expert's (Q8_0, the heaviest) first, so the CTAs
-        // even out on the lighter routed items that follow
+        // items are handed out by one counter (zeroed per call) in the order
+        // above: the shared expert's gate/up items (Q8_0, the heaviest) first,
+        // so the CTAs even out on the lighter routed items that follow
         auto claim = [&]() -> int {
             int v = 0;
-            if (lane == 0) v = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+            if (lane == 0) v = (int)atomicAdd(A.next, 1u);
             return __shfl_sync(kFull, v, 0);
         };
         int id_next = claim();
-        for (int k = 0;; ++k) {
+        for (;;) {
             const int id = id_next;
             if (!routed && id >= n_sh_items) wait_routing();
             const int item = id < n_items ? id : -1;
             // claim the following item now; the atomic's latency hides behind this item's stages
             if (item >= 0) id_next = claim();
-            if (item >= 0) decode_item<kDown>(A, sc, s_perm, geo, n_slots, item, p_cursor, P, pslot);
+            if (item >= 0) {
+                decode_item(A, sc, s_perm, n_slots, n_gu, item, cur_gu, cur_dn, P);
+                fmt0 = tab.fmt[P.e][P.down ? 2 : 0];
+                fmt1 = tab.fmt[P.e][P.down ? 2 : 1];
+                P.nst0 = geo[P.down][fmt0 - 1][P.ntok - 1].nst;
+                P.nst = P.down ? 2 * P.nst0 : P.nst0 + geo[0][fmt1 - 1][P.ntok - 1].nst;
+            }
             const int nst = item >= 0 ? P.nst : 1;
             bool failed = false;
+            bool h_in = !(item >= 0 && P.down);   // a down item copies h once its slot's blocks are in
             // this lane's copy for the current phase (one tensor of the item)
             const uint8_t* c_src = nullptr;
             uint32_t c_stride = 0, c_dst = 0;
@@ -716,7 +812,19 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     failed = true;
                     break;
                 }
-                if (!kDown && A.fail_first_stage && p_q == 0) {
+                if (!routed && p_q >= kPreRouteDepth) {
+                    // Before the routing result is in, keep at most
+                    // kPreRouteDepth stages in flight: the routing's own memory
+                    // round trips (logits, the published result, the first
+                    // routed weights) are on the step's critical path, and
+                    // full queues would stretch each of them.
+                    const int sq = p_q - kPreRouteDepth;
+                    if (!mbar_wait(bar0 + 8 * (kNST + sq % kNST), (sq / kNST) & 1, A.err, kErrEmpty, A.wait_ns)) {
+                        failed = true;
+                        break;
+                    }
+                }
+                if (A.fail_first_stage && p_q == 0) {
                     // test hook: nothing arrives on this slot's full barrier and
                     // no copy targets it, so the consumers' wait runs out
                     ++p_q;
@@ -730,11 +838,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 }
                 if (pj == 0 || pj == P.nst0) {
                     // phases: gate then up (gate/up items); rows rb then rb + 1 (down items, tensor 2 / 3)
-                    tensor = kDown ? (pj == 0 ? 2 : 3) : (pj == 0 ? 0 : 1);
+                    tensor = P.down ? (pj == 0 ? 2 : 3) : (pj == 0 ? 0 : 1);
                     phase_j = pj;
-                    fmt = sc.fmt[pslot][tensor == 1 ? 1 : 0];
-                    G = &geo[fmt - 1][P.ntok - 1];
-                    const uint8_t* tbase = tensor == 1 ? sc.ptr_up[pslot] : sc.ptr[pslot];
+                    fmt = tensor == 1 ? fmt1 : fmt0;
+                    G = &geo[P.down][fmt - 1][P.ntok - 1];
+                    const uint8_t* tbase = tab.p[P.e][tensor >= 2 ? 2 : tensor];
                     c_src = nullptr; c_stride = 0; c_dst = 0;
                     if (lane < G->npl) {
                         c_src = tbase + G->pl[lane] + (int64_t)(P.rb + (tensor == 3 ? 1 : 0)) * G->rbstr[lane];
@@ -742,6 +850,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         c_dst = G->woff[lane];
                     }
                     if (lane >= 4 && lane < 4 + 2 * P.ntok) {
+                        const VecSrc& vs = P.down ? vh : vx;
                         const int tk = (lane - 4) / 2, piece = (lane - 4) - 2 * tk;
                         int v = P.vec[0];
 #pragma unroll
@@ -755,8 +864,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     }
                 }
                 const int per = G->per;
-                const int s0 = (pj - phase_j) * per, ks = min(per, p_nsb - s0);
-                const uint32_t stage = ring + slot * kStageBytes;
+                const int s0 = (pj - phase_j) * per, ks = min(per, (P.down ? A.nsbi : A.nsbx) - s0);
+                const uint32_t stage = ring + slot * kSlotBytes;
                 const uint32_t bytes = c_src ? (uint32_t)ks * c_stride : 0u;
                 uint32_t total = bytes;
 #pragma unroll
@@ -765,16 +874,40 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     int4* H = reinterpret_cast<int4*>(&hdr[slot]);
                     H[0] = make_int4(item, pj, P.nst, s0);
                     H[1] = make_int4(ks, fmt, tensor, P.ntok);
-                    H[2] = make_int4(P.rb, P.e, P.shared, 0);
+                    H[2] = make_int4(P.rb, P.e, P.shared, P.slot);
                     H[3] = make_int4(P.asg[0], P.asg[1], P.asg[2], P.asg[3]);
                     s_posted[slot] = p_q;
                     mbar_arrive_tx(full, total);
                 }
                 __syncwarp();
-                // weight planes (lanes 0..3) first; the down kernel's first copy
-                // of h waits for the gate/up kernel, while its weights stream
+                // weight planes (lanes 0..3) first; a down item's weights stream
+                // while the last blocks of its slot's h may still be computed
                 if (bytes && lane < 4) bulk_copy_hint(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full, wpol);
-                if (!deps) { pdl_wait(); deps = true; }
+                if (!h_in) {
+                    // h of the slot: every gate/up item of the slot publishes its
+                    // tokens' 32-row blocks (release add on the slot's counter)
+                    const uint32_t target = (uint32_t)((d.I / 32) * sc.ntot[P.slot]);
+                    const uint32_t* cnt = A.hready + P.slot;
+                    if (lane == 0 && ld_acquire(cnt) < target) {
+                        const uint64_t t0 = global_ns();
+                        while (ld_acquire(cnt) < target) {
+                            if (global_ns() - t0 > A.wait_ns) { atomicOr(A.err, kErrReady); s_fail = 1; break; }
+                            __nanosleep(100);
+                        }
+                    }
+                    __syncwarp();
+                    // every lane that copies h acquires the counter itself, then
+                    // orders its bulk (async proxy) reads after that acquire
+                    if (lane >= 4) (void)ld_acquire(cnt);
+                    asm volatile("fence.proxy.async.global;" ::: "memory");
+                    h_in = true;
+                }
+                if (!tokens_in && !P.down) {
+                    // the shared expert's items run before routing: wait for the
+                    // prepared tokens once
+                    wait_word(A.logits_done, A.n_logit_ctas);
+                    tokens_in = true;
+                }
                 if (bytes && lane >= 4) bulk_copy(stage + c_dst, c_src + (size_t)s0 * c_stride, bytes, full);
                 ++p_q;
             }
@@ -787,7 +920,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // superblocks col, col + kCols, ... (Q8_0: both halves of the code
         // pairs of each)
         const int rt0 = kNT == 2 ? 0 : (warp & 1), col = kNT == 2 ? warp : (warp >> 1);
-        float acc[2][MT][4];   // [0] gate (or down), [1] up; rows g + 8 i
+        float acc[2][MT][4];   // [0] gate (or rows rb), [1] up (or rows rb + 1); rows g + 8 i
         float cur[MT][4];      // the tensor being streamed
 #pragma unroll
         for (int tk = 0; tk < MT; ++tk)
@@ -802,16 +935,17 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             const Hdr& H = hdr[slot];
             if (H.item < 0) break;
-            const uint32_t stage = ring + slot * kStageBytes;
+            const uint32_t stage = ring + slot * kSlotBytes;
             const int fmt = H.fmt, ks = H.ks, ntok = H.ntok;
-            const Geo& GS = geo[fmt - 1][ntok - 1];
+            const bool dn = H.tensor >= 2;
+            const Geo& GS = geo[dn ? 1 : 0][fmt - 1][ntok - 1];
             // superblock jj of the stage goes to warp column (jj + s) % kCols, s the
             // stage's first superblock counted over the whole item, so every warp
             // gets the same share of an item even where a stage's count is not a
             // multiple of kCols
-            const int s_item = H.s0 + ((H.tensor & 1) ? (kDown ? A.nsbi : A.nsbx) : 0);
+            const int s_item = H.s0 + ((H.tensor & 1) ? (dn ? A.nsbi : A.nsbx) : 0);
             const int wcol = (col - s_item % kCols + kCols) % kCols;
-            if ((H.tensor == 1 || H.tensor == 3) && H.s0 == 0) {
+            if ((H.tensor & 1) && H.s0 == 0) {
                 // first stage of the second phase: the first phase's sums are complete
 #pragma unroll
                 for (int tk = 0; tk < MT; ++tk)
@@ -839,10 +973,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             // fields needed after the slot is released to the producer
             const bool item_end = H.j == H.nst - 1;
-            int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0;
+            int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0, e_slot = 0;
             int e_asg[kDecodeTok];
             if (item_end) {
-                e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e;
+                e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e; e_slot = H.slot;
 #pragma unroll
                 for (int tk = 0; tk < kDecodeTok; ++tk) e_asg[tk] = H.asg[tk];
             }
@@ -886,13 +1020,14 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     v0 += red[buf][c2][0][tk][lane];
                     v1 += red[buf][c2][1][tk][lane];
                 }
-                if (kDown) {
+                if (dn) {
                     A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
                     A.pdn[(size_t)a * d.H + 32 * (e_rb + 1) + lane] = v1;
                 } else {
                     // SwiGLU (routing weight folded in), then prepare h for the down projection
-                    if (!e_shared) pdl_wait();   // routing weights come from the routing kernel
-                    const float w = e_shared ? 1.0f : A.wts[a];
+                    // routing weights: written by the logits kernel's routing CTA and
+                    // acquired by this CTA's producer before it posted the item
+                    const float w = e_shared ? 1.0f : __ldcg(A.wts + a);
                     const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
                     const int fam = families_of(tab.fmt[e_e][2]);
                     __half* hq = A.hq + (size_t)a * 4 * A.nsbi * 256;
@@ -901,6 +1036,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     const int n_rb = d.I / 32;
                     if (e_rb == n_rb - 1)
                         for (int jb = n_rb; jb < 8 * A.nsbi; ++jb) prep_block32(0.0f, jb, fam, hq, hs, A.nsbi);
+                    // publish the block: every lane's writes, then one release add
+                    // on the slot's counter (down items of the slot wait for it)
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0) red_release_add(A.hready + e_slot, 1u);
                 }
             }
             // with two buffers the next item end writes the other one and its
@@ -933,10 +1073,8 @@ __global__ void combine_kernel(Dims d, const float* __restrict__ pdn, float* __r
 }
 
 void decode_setup() {
-    cudaFuncSetAttribute(ffn_kernel<false, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
-    cudaFuncSetAttribute(ffn_kernel<true, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
-    cudaFuncSetAttribute(ffn_kernel<false, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
-    cudaFuncSetAttribute(ffn_kernel<true, kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
 }
 
 void combine_setup() { prefer_max_shared(combine_kernel); }
@@ -945,45 +1083,40 @@ void combine_setup() { prefer_max_shared(combine_kernel); }
 
 size_t decode_counter_bytes(const Dims& d) {
     (void)d;
-    return 2 * 4;   // gate/up and down item counters
+    return 4 + 4 * (kMaxExperts + 1);   // the item counter, then one h counter per expert slot
 }
 
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int smem = kRingBytes;
-    const int g_num_sms = device_setup(kSetupDecode, decode_setup);
-    if (g_num_sms <= 0) return cudaErrorInvalidDevice;
+    const int num_sms = device_setup(kSetupDecode, decode_setup);
+    if (num_sms <= 0) return cudaErrorInvalidDevice;
     DecodeArgs A;
     A.d = d;
     A.nsbx = (d.H + 255) / 256;
     A.nsbi = (d.I + 255) / 256;
     A.xq = w.xq; A.xs = w.xs; A.hq = w.hq; A.hs = w.hs;
-    A.offsets = w.offsets; A.perm = w.perm; A.active = w.active; A.wts = w.wts;
+    A.perm = w.perm; A.wts = w.wts;
     A.plan = w.plan;
     A.pdn = w.pdn;
     A.next = w.counters;
+    A.hready = w.counters + 1;
+    A.logits_done = w.logits_done;
+    A.route_ready = w.route_ready;
+    A.n_logit_ctas = (uint32_t)(d.E * ((d.T + 7) / 8));   // the logits kernel's grid (experts x 8-token groups)
     A.err = w.err;
     A.wait_ns = 1000000000ull;
     A.fail_first_stage = 0;
     uint64_t test_ns = 0;
     if (take_wait_test(&test_ns)) { A.wait_ns = test_ns; A.fail_first_stage = 1; }
-    A.out = out;
-    auto fill_geo = [&](bool down) {
+    for (int dn = 0; dn < 2; ++dn)
         for (int f = 1; f <= 4; ++f)
-            for (int n = 1; n <= kDecodeTok; ++n) make_geo(A.geo[f - 1][n - 1], d, down, f, n);
-    };
-    fill_geo(false);
+            for (int n = 1; n <= kDecodeTok; ++n) make_geo(A.geo[dn][f - 1][n - 1], d, dn == 1, f, n);
     // one token: every item carries one, and the accumulators shrink to one token's
     const bool one = d.T == 1;
-    prof_begin("gateup_mma", s);
-    cudaError_t err = one ? launch_pdl(ffn_kernel<false, 1>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A)
-                          : launch_pdl(ffn_kernel<false, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
-    prof_end(s);
-    if (err != cudaSuccess) return err;
-    fill_geo(true);
-    prof_begin("down_mma", s);
-    err = one ? launch_pdl(ffn_kernel<true, 1>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A)
-              : launch_pdl(ffn_kernel<true, kDecodeTok>, dim3(g_num_sms), dim3(kThreads), smem, s, tab, A);
+    prof_begin("ffn_mma", s);
+    cudaError_t err = one ? launch_pdl(ffn_kernel<1>, dim3(num_sms), dim3(kThreads), smem, s, tab, A)
+                          : launch_pdl(ffn_kernel<kDecodeTok>, dim3(num_sms), dim3(kThreads), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);

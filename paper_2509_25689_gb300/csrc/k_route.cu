@@ -36,111 +36,6 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ int token_exp(float amax) { return amax > 0.0f ? ilogbf(amax) : 0; }
 
 // ---------------------------------------------------------------------------
-// logits: grid (E, ceil(T / kTok)), one warp per 1024-element segment
-// ---------------------------------------------------------------------------
-constexpr int kTok = 8;
-
-__global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
-                                                             const float* __restrict__ W, int H, int T,
-                                                             int E, float* __restrict__ z,
-                                                             __half* __restrict__ xq, float* __restrict__ xs,
-                                                             __half* __restrict__ x16, int32_t* __restrict__ xe,
-                                                             uint32_t* __restrict__ zero_words, int n_zero) {
-    __shared__ float part[32][kTok];
-    __shared__ float pmax[32][kTok];   // per segment: largest |x| of each token (prefill copy only)
-    const int e = blockIdx.x, t0 = blockIdx.y * kTok;
-    const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
-    const int c0 = seg * 8, nc = min(8, nchunk - c0);
-    const float* wrow = W + (size_t)e * H;
-    // The router weights are an input no kernel of this library writes, so
-    // their loads go out before the wait for the previous kernel (which may
-    // be the previous layer's combine, writing this call's x).
-    float4 wv[8];
-#pragma unroll
-    for (int c = 0; c < 8; ++c)
-        if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(wrow + (c0 + c) * 128 + 4 * lane));
-    pdl_wait();
-    pdl_launch();
-    // per-call words that must start at zero (work counters, error word)
-    if (blockIdx.x == 0 && blockIdx.y == 0)
-        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
-    float acc[kTok], amx[kTok];
-#pragma unroll
-    for (int j = 0; j < kTok; ++j) acc[j] = amx[j] = 0.0f;
-#pragma unroll
-    for (int j = 0; j < kTok; ++j) {
-        const int t = t0 + j;
-        if (t >= T) break;
-        const uint16_t* xr = x + (size_t)t * H;
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            if (c < nc) {
-                const uint2 xv = __ldg(reinterpret_cast<const uint2*>(xr + (c0 + c) * 128 + 4 * lane));
-                acc[j] = __fmaf_rn(bf16_lo(xv.x), wv[c].x, acc[j]);
-                acc[j] = __fmaf_rn(bf16_hi(xv.x), wv[c].y, acc[j]);
-                acc[j] = __fmaf_rn(bf16_lo(xv.y), wv[c].z, acc[j]);
-                acc[j] = __fmaf_rn(bf16_hi(xv.y), wv[c].w, acc[j]);
-                if (x16 != nullptr)
-                    amx[j] = fmaxf(amx[j], fmaxf(fmaxf(fabsf(bf16_lo(xv.x)), fabsf(bf16_hi(xv.x))),
-                                                 fmaxf(fabsf(bf16_lo(xv.y)), fabsf(bf16_hi(xv.y)))));
-            }
-        }
-    }
-#pragma unroll
-    for (int j = 0; j < kTok; ++j) {
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) acc[j] = __fadd_rn(acc[j], __shfl_xor_sync(kFull, acc[j], off));
-        if (x16 != nullptr) amx[j] = warp_max_abs(amx[j]);
-    }
-    if (lane == 0) {
-#pragma unroll
-        for (int j = 0; j < kTok; ++j) { part[seg][j] = acc[j]; pmax[seg][j] = amx[j]; }
-    }
-    __syncthreads();
-    if (threadIdx.x < kTok) {
-        const int t = t0 + threadIdx.x;
-        if (t < T) {
-            float r = part[0][threadIdx.x];
-            for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
-            z[(size_t)t * E + e] = r;
-        }
-    }
-    // fp16 copy of the tokens for the prefill GEMM (each token scaled by its
-    // power of two), spread over the CTAs
-    if (x16 != nullptr) {
-        for (int j = 0; j < kTok; ++j) {
-            const int t = t0 + j;
-            if (t >= T) break;
-            float m = pmax[0][j];
-            for (int s = 1; s < nseg; ++s) m = fmaxf(m, pmax[s][j]);
-            const int ex = token_exp(m);
-            if (e == 0 && threadIdx.x == 0) xe[t] = ex;
-            for (int k = e * blockDim.x + threadIdx.x; k < H; k += E * blockDim.x)
-                x16[(size_t)t * H + k] = __float2half_rn(ldexpf(bf16_lo(x[(size_t)t * H + k]), -ex));
-        }
-    }
-    // The CTAs also prepare the tokens' activations for the expert-FFN
-    // kernels, spread over all of them: warp `seg` of the CTA of expert e
-    // takes the 32-element blocks 32*seg + e, 32*seg + e + E, ... of its
-    // segment (blocks past the hidden size, up to the 256 padding, are zero).
-    if (xq != nullptr) {
-        const int nsb = (H + 255) / 256;
-        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)nsb * kStatFloats;
-        for (int j = 0; j < kTok; ++j) {
-            const int t = t0 + j;
-            if (t >= T) break;
-            for (int jb = 32 * seg + e; jb < 32 * seg + 32 && jb < 8 * nsb; jb += E) {
-                const int k = 32 * jb + lane;
-                const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
-                prep_block32(v, jb, (1 << kF2) | (1 << kF4) | (1 << kF8), xq + (size_t)t * qstride,
-                             xs + (size_t)t * sstride, nsb);
-            }
-        }
-    }
-}
-
-// ---------------------------------------------------------------------------
 // logits for larger batches (no activation preparation): grid
 // (ceil(E / kEB), ceil(T / kTokT)); a CTA keeps its 4 tokens' segments in
 // registers as fp32 and runs through 16 experts, so the tokens are read and
@@ -154,8 +49,7 @@ constexpr int kTokT = 4;
 __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t* __restrict__ x,
                                                                   const float* __restrict__ W, int H, int T,
                                                                   int E, float* __restrict__ z,
-                                                                  __half* __restrict__ x16, int32_t* __restrict__ xe,
-                                                                  uint32_t* __restrict__ zero_words, int n_zero) {
+                                                                  __half* __restrict__ x16, int32_t* __restrict__ xe) {
     __shared__ float part[8][kEB][kTokT];   // per segment (warp): each expert's sums of the CTA's tokens
     __shared__ float pmax[8][kTokT];        // per segment: largest |x| of each token (prefill copy)
     const int e0 = blockIdx.x * kEB, t0 = blockIdx.y * kTokT;
@@ -169,8 +63,6 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
         if (c < nc && e0 < E) wv[c] = __ldg(reinterpret_cast<const float4*>(W + (size_t)e0 * H + (c0 + c) * 128 + 4 * lane));
     pdl_wait();
     pdl_launch();
-    if (blockIdx.x == 0 && blockIdx.y == 0)
-        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_words[i] = 0u;
     float4 xf[kTokT][8];   // the tokens' segment elements 4 lane + 0..3 of each chunk, as fp32
 #pragma unroll
     for (int j = 0; j < kTokT; ++j)
@@ -263,6 +155,17 @@ __global__ void __launch_bounds__(256) router_logits_tile_kernel(const uint16_t*
     }
 }
 
+// Per-call words that must start at zero (work counters, the h and routing
+// flags, the error word), cleared by the first kernel of a forward call.  It
+// lets its successor launch at once (that kernel waits for this one before
+// touching the words) and itself waits for the previous kernel on the
+// stream, so the previous call no longer uses them.
+__global__ void zero_kernel(uint32_t* __restrict__ words, int n) {
+    pdl_launch();
+    pdl_wait();
+    for (int i = threadIdx.x; i < n; i += blockDim.x) words[i] = 0u;
+}
+
 constexpr int kTopkWarps = 4;
 
 __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __restrict__ z,
@@ -284,43 +187,50 @@ __global__ void __launch_bounds__(kTopkWarps * 32) topk_kernel(const float* __re
 // ---------------------------------------------------------------------------
 constexpr int kPermThreads = 512;
 constexpr int kPermWarps = kPermThreads / 32;
+// barrier 2 over the kPermThreads routing threads (the CTA may have more)
+__device__ __forceinline__ void perm_sync() { asm volatile("bar.sync 2, %0;" ::"n"(kPermThreads) : "memory"); }
 
-// With `z` given, the same CTA first routes every token (one warp per token,
+// Shared memory of the routing + permutation step (one CTA).
+struct PermSmem {
+    int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
+    int32_t s_off[kMaxExperts + 1];
+    int32_t s_act[kMaxExperts + 1];
+    float g_sh[kPermWarps][kMaxGroups];
+    float s_bias[kMaxExperts];
+};
+
+// Routing and permutation by the first kPermThreads threads of one CTA (the
+// caller has staged the selection bias in S.s_bias and synchronised).  With
+// `z` given, the CTA first routes every token (one warp per token,
 // decode-sized batches) and then permutes.  Offsets and the active list are
 // kept in shared memory as well, so nothing written here is read back from
-// global memory.
-__global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restrict__ idx, Dims d,
-                                                               int32_t* __restrict__ offsets,
-                                                               int32_t* __restrict__ perm,
-                                                               int32_t* __restrict__ inv,
-                                                               int32_t* __restrict__ active,
-                                                               Plan* __restrict__ plan,
-                                                               const float* __restrict__ z,
-                                                               const float* __restrict__ bias,
-                                                               float* __restrict__ wts) {
+// global memory.  offsets, inv and active may be NULL (not written).  Threads
+// leave by returning; block-wide steps use a named barrier over the
+// kPermThreads threads, so the CTA may hold more.  route_warp: the warp that
+// routes a single token (the others return at once on that path).
+__device__ void route_permute_cta(PermSmem& S, int32_t* __restrict__ idx, const Dims& d,
+                                  int32_t* __restrict__ offsets, int32_t* __restrict__ perm,
+                                  int32_t* __restrict__ inv, int32_t* __restrict__ active,
+                                  Plan* __restrict__ plan, const float* __restrict__ z,
+                                  float* __restrict__ wts, int route_warp = 0) {
     const int n = d.T * d.K, E = d.E;
-    __shared__ int32_t cnt[kPermWarps][kMaxExperts];   // per-warp segment counts, then cursors
-    __shared__ int32_t s_off[kMaxExperts + 1];
-    __shared__ int32_t s_act[kMaxExperts + 1];
-    __shared__ float g_sh[kPermWarps][kMaxGroups];
-    __shared__ float s_bias[kMaxExperts];
+    auto& cnt = S.cnt;
+    auto& s_off = S.s_off;
+    auto& s_act = S.s_act;
+    auto& g_sh = S.g_sh;
+    const float* s_bias = S.s_bias;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // the selection bias is an input no kernel of this library writes: staged
-    // before the wait for the logits kernel
-    if (z != nullptr)
-        for (int i = threadIdx.x; i < E; i += kPermThreads) s_bias[i] = bias ? bias[i] : 0.0f;
-    __syncthreads();
-    pdl_wait();
-    pdl_launch();
+    if (warp >= kPermWarps) return;
     if (z != nullptr && d.T == 1 && d.K <= 32 && E <= 256) {
         // One token: the selection holds K distinct experts, one entry each, so
         // the counting sort reduces to ranking them.  One warp does all of it
         // in registers (no block barriers, nothing read back from global memory).
-        if (warp != 0) return;
+        if (warp != route_warp) return;
         const int K = d.K;
         int sel = 0;
-        sel::route_token(z, s_bias, d.E, d.G, d.Gk, K, d.routed_scale, 0, reinterpret_cast<float*>(cnt[0]), g_sh[0],
-                         idx, wts, &sel);
+        // scratch: rows 0 and 1 of the counting table (free on this path)
+        sel::route_token_compact(z, s_bias, d.E, d.G, d.Gk, K, d.routed_scale, 0, reinterpret_cast<float*>(cnt[0]),
+                                 g_sh[route_warp], idx, wts, &sel);
         // the selection as a 256-bit set; an expert's rank (and offsets[e]) is
         // the number of selected ids below it
         uint32_t mask[8];
@@ -337,17 +247,19 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         const int rank = below(sel);
         if (lane < K) {
             perm[rank] = lane;   // entry a = t * K + j = j
-            inv[lane] = rank;
-            active[1 + rank] = sel;
+            if (inv) inv[lane] = rank;
+            if (active) active[1 + rank] = sel;
         }
-        if (lane == 0) active[0] = K;
+        if (lane == 0 && active) active[0] = K;
         // offsets[e] = selected experts with a lower id; offsets[E] = K
+        if (offsets) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const int e = lane * 8 + q;
-            if (e < E) offsets[e] = below(e);
+            for (int q = 0; q < 8; ++q) {
+                const int e = lane * 8 + q;
+                if (e < E) offsets[e] = below(e);
+            }
+            if (lane == 0) offsets[E] = K;
         }
-        if (lane == 0) offsets[E] = K;
         if (plan == nullptr) return;
         // work plan: slot p (shared expert first) holds one token
         const int n_slots = K + d.has_shared;
@@ -375,14 +287,14 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         for (int t = warp; t < d.T; t += kPermWarps)
             sel::route_token(z, s_bias, d.E, d.G, d.Gk, d.K, d.routed_scale, t, reinterpret_cast<float*>(cnt[warp]),
                         g_sh[warp], idx, wts);
-        __syncthreads();
+        perm_sync();
     }
     for (int i = threadIdx.x; i < kPermWarps * kMaxExperts; i += kPermThreads) (&cnt[0][0])[i] = 0;
-    __syncthreads();
+    perm_sync();
     const int seg = (n + kPermWarps - 1) / kPermWarps;
     const int a0 = warp * seg, a1 = min(n, a0 + seg);
     for (int a = a0 + lane; a < a1; a += 32) atomicAdd(&cnt[warp][idx[a]], 1);
-    __syncthreads();
+    perm_sync();
     // per-expert totals and per-warp starting cursors (warp order = entry order)
     if (threadIdx.x < E) {
         const int e = threadIdx.x;
@@ -391,7 +303,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         for (int wv = 0; wv < kPermWarps; ++wv) { const int c = cnt[wv][e]; cnt[wv][e] = run; run += c; }
         s_off[e] = run;
     }
-    __syncthreads();
+    perm_sync();
     if (warp == 0) {
         // exclusive scan of totals over experts (E <= 256: 8 per lane)
         int local[8], sum = 0;
@@ -412,17 +324,17 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             const int e = lane * 8 + q;
-            if (e < E) { offsets[e] = run; s_off[e] = run; }
+            if (e < E) { if (offsets) offsets[e] = run; s_off[e] = run; }
             run += local[q];
         }
-        if (lane == 31) { offsets[E] = run; s_off[E] = run; }
+        if (lane == 31) { if (offsets) offsets[E] = run; s_off[E] = run; }
     }
-    __syncthreads();
+    perm_sync();
     for (int i = threadIdx.x; i < kPermWarps * E; i += kPermThreads) {
         const int wv = i / E, e = i - wv * E;
         cnt[wv][e] += s_off[e];
     }
-    __syncthreads();
+    perm_sync();
     // stable scatter: each warp walks its segment in order, 32 entries a step
     for (int base = a0; base < a1; base += 32) {
         const int a = base + lane;
@@ -433,7 +345,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         if (ok) {
             const int pos = cnt[warp][e] + rank;
             perm[pos] = a;
-            inv[a] = pos;
+            if (inv) inv[a] = pos;
         }
         __syncwarp();
         if (ok && rank == 0) cnt[warp][e] += __popc(peers);
@@ -458,11 +370,11 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
         int pos = incl - c;
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (flags & (1 << q)) { active[1 + pos] = lane * 8 + q; s_act[1 + pos] = lane * 8 + q; ++pos; }
-        if (lane == 31) { active[0] = incl; s_act[0] = incl; }
+            if (flags & (1 << q)) { if (active) active[1 + pos] = lane * 8 + q; s_act[1 + pos] = lane * 8 + q; ++pos; }
+        if (lane == 31) { if (active) active[0] = incl; s_act[0] = incl; }
     }
     if (plan == nullptr) return;
-    __syncthreads();
+    perm_sync();
     // decode work plan: items per expert slot (shared expert first)
     if (warp == 0) {
         const int n_slots = s_act[0] + d.has_shared;
@@ -509,6 +421,156 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
     }
 }
 
+// Standalone routing + permutation kernel (one CTA of kPermThreads).
+__global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restrict__ idx, Dims d,
+                                                               int32_t* __restrict__ offsets,
+                                                               int32_t* __restrict__ perm,
+                                                               int32_t* __restrict__ inv,
+                                                               int32_t* __restrict__ active,
+                                                               Plan* __restrict__ plan,
+                                                               const float* __restrict__ z,
+                                                               const float* __restrict__ bias,
+                                                               float* __restrict__ wts) {
+    __shared__ PermSmem S;
+    // the selection bias is an input no kernel of this library writes: staged
+    // before the wait for the logits kernel
+    if (z != nullptr)
+        for (int i = threadIdx.x; i < d.E; i += kPermThreads) S.s_bias[i] = bias ? bias[i] : 0.0f;
+    __syncthreads();
+    pdl_wait();
+    pdl_launch();
+    route_permute_cta(S, idx, d, offsets, perm, inv, active, plan, z, wts);
+}
+
+// ---------------------------------------------------------------------------
+// logits: grid (E, ceil(T / kTok)), one warp per 1024-element segment
+// ---------------------------------------------------------------------------
+constexpr int kTok = 8;
+
+__global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
+                                                             const float* __restrict__ W, int H, int T,
+                                                             int E, float* __restrict__ z,
+                                                             __half* __restrict__ xq, float* __restrict__ xs,
+                                                             __half* __restrict__ x16, int32_t* __restrict__ xe,
+                                                             const FusedRoute fr) {
+    __shared__ float part[32][kTok];
+    __shared__ float pmax[32][kTok];   // per segment: largest |x| of each token (prefill copy only)
+    __shared__ int s_last;
+    const int e = blockIdx.x, t0 = blockIdx.y * kTok;
+    const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
+    const int c0 = seg * 8, nc = min(8, nchunk - c0);
+    const float* wrow = W + (size_t)e * H;
+    // The router weights are an input no kernel of this library writes, so
+    // their loads go out before the wait for the previous kernel (which may
+    // be the previous layer's combine, writing this call's x).
+    float4 wv[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        if (c < nc) wv[c] = __ldg(reinterpret_cast<const float4*>(wrow + (c0 + c) * 128 + 4 * lane));
+    // fused routing: every CTA stages the selection bias (an input as well)
+    // now, so the CTA that ends up routing has it without another round trip
+    extern __shared__ __align__(16) uint8_t dyn_smem[];
+    PermSmem& S = *reinterpret_cast<PermSmem*>(dyn_smem);
+    if (fr.on) {
+        for (int i = threadIdx.x; i < E; i += blockDim.x) S.s_bias[i] = fr.bias ? __ldg(fr.bias + i) : 0.0f;
+        __syncthreads();
+    }
+    pdl_wait();
+    pdl_launch();
+    float acc[kTok], amx[kTok];
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) acc[j] = amx[j] = 0.0f;
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) {
+        const int t = t0 + j;
+        if (t >= T) break;
+        const uint16_t* xr = x + (size_t)t * H;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            if (c < nc) {
+                const uint2 xv = __ldg(reinterpret_cast<const uint2*>(xr + (c0 + c) * 128 + 4 * lane));
+                acc[j] = __fmaf_rn(bf16_lo(xv.x), wv[c].x, acc[j]);
+                acc[j] = __fmaf_rn(bf16_hi(xv.x), wv[c].y, acc[j]);
+                acc[j] = __fmaf_rn(bf16_lo(xv.y), wv[c].z, acc[j]);
+                acc[j] = __fmaf_rn(bf16_hi(xv.y), wv[c].w, acc[j]);
+                if (x16 != nullptr)
+                    amx[j] = fmaxf(amx[j], fmaxf(fmaxf(fabsf(bf16_lo(xv.x)), fabsf(bf16_hi(xv.x))),
+                                                 fmaxf(fabsf(bf16_lo(xv.y)), fabsf(bf16_hi(xv.y)))));
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kTok; ++j) {
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) acc[j] = __fadd_rn(acc[j], __shfl_xor_sync(kFull, acc[j], off));
+        if (x16 != nullptr) amx[j] = warp_max_abs(amx[j]);
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int j = 0; j < kTok; ++j) { part[seg][j] = acc[j]; pmax[seg][j] = amx[j]; }
+    }
+    __syncthreads();
+    if (threadIdx.x < kTok) {
+        const int t = t0 + threadIdx.x;
+        if (t < T) {
+            float r = part[0][threadIdx.x];
+            for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
+            z[(size_t)t * E + e] = r;
+        }
+    }
+    // fp16 copy of the tokens for the prefill GEMM (each token scaled by its
+    // power of two), spread over the CTAs
+    if (x16 != nullptr) {
+        for (int j = 0; j < kTok; ++j) {
+            const int t = t0 + j;
+            if (t >= T) break;
+            float m = pmax[0][j];
+            for (int s = 1; s < nseg; ++s) m = fmaxf(m, pmax[s][j]);
+            const int ex = token_exp(m);
+            if (e == 0 && threadIdx.x == 0) xe[t] = ex;
+            for (int k = e * blockDim.x + threadIdx.x; k < H; k += E * blockDim.x)
+                x16[(size_t)t * H + k] = __float2half_rn(ldexpf(bf16_lo(x[(size_t)t * H + k]), -ex));
+        }
+    }
+    // The CTAs also prepare the tokens' activations for the expert-FFN
+    // kernels, spread over all of them: warp `seg` of the CTA of expert e
+    // takes the 32-element blocks 32*seg + e, 32*seg + e + E, ... of its
+    // segment (blocks past the hidden size, up to the 256 padding, are zero).
+    if (xq != nullptr) {
+        const int nsb = (H + 255) / 256;
+        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)nsb * kStatFloats;
+        for (int j = 0; j < kTok; ++j) {
+            const int t = t0 + j;
+            if (t >= T) break;
+            for (int jb = 32 * seg + e; jb < 32 * seg + 32 && jb < 8 * nsb; jb += E) {
+                const int k = 32 * jb + lane;
+                const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
+                prep_block32(v, jb, (1 << kF2) | (1 << kF4) | (1 << kF8), xq + (size_t)t * qstride,
+                             xs + (size_t)t * sstride, nsb);
+            }
+        }
+    }
+    if (!fr.on) return;
+    // Routing fused in: every CTA publishes its logits and prepared tokens
+    // (each thread fences its own writes, then one count per CTA); the CTA
+    // that counts last routes every token and permutes, reading the others'
+    // logits after a fence, then publishes the result with a release store.
+    // The expert-FFN kernel, launched as this grid's dependent, waits on the
+    // count (prepared tokens) and on the release flag (routing result).
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(fr.logits_done, 1u) == fr.n_ctas - 1u;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    route_permute_cta(S, fr.idx, fr.d, fr.offsets, fr.perm, fr.inv, fr.active, fr.plan, z, fr.wts);
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(fr.route_ready), "r"(1u) : "memory");
+}
+
+
 void route_setup() {
     prefer_max_shared(router_logits_kernel);
     prefer_max_shared(router_logits_tile_kernel);
@@ -518,22 +580,37 @@ void route_setup() {
 
 }  // namespace
 
+cudaError_t launch_zero(uint32_t* words, int n, cudaStream_t s) {
+    prof_begin("zero", s);
+    const cudaError_t e = launch_pdl(zero_kernel, dim3(1), dim3(256), 0, s, words, n);
+    prof_end(s);
+    return e;
+}
+
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 __half* x16, int32_t* xe, uint32_t* zero_words, int n_zero, cudaStream_t s) {
+                                 __half* x16, int32_t* xe, const FusedRoute* fused, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
     const int nseg = (d.H / 128 + 7) / 8;
     if (device_setup(kSetupRoute, route_setup) <= 0) return cudaErrorInvalidDevice;
     prof_begin("router_logits", s);
     cudaError_t e;
-    if (xq == nullptr && d.T >= 16 && nseg <= 8) {
+    if (fused == nullptr && xq == nullptr && d.T >= 16 && nseg <= 8) {
         // larger batches without activation preparation: tokens reused across 16 experts
         dim3 grid((d.E + kEB - 1) / kEB, (d.T + kTokT - 1) / kTokT);
-        e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16, xe,
-                       zero_words, n_zero);
+        e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16, xe);
     } else {
         dim3 grid(d.E, (d.T + kTok - 1) / kTok);
-        e = launch_pdl(router_logits_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe,
-                       zero_words, n_zero);
+        FusedRoute fr{};
+        int threads = nseg * 32;
+        size_t smem = 0;
+        if (fused != nullptr) {
+            fr = *fused;
+            fr.on = 1;
+            fr.n_ctas = grid.x * grid.y;
+            threads = (nseg > kPermWarps ? nseg : kPermWarps) * 32;   // the last CTA routes with kPermWarps warps
+            smem = sizeof(PermSmem);
+        }
+        e = launch_pdl(router_logits_kernel, grid, dim3(threads), smem, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe, fr);
     }
     prof_end(s);
     return e;

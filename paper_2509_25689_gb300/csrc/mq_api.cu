@@ -92,8 +92,10 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_plan = take(sizeof(Plan));
     const size_t o_xe = take((size_t)d.T * 4);
     const size_t cnt_bytes = decode_counter_bytes(d);
-    const size_t o_cnt = take(cnt_bytes + 4);   // work counters, then the error word (zeroed per call)
-    const size_t o_err = o_cnt + cnt_bytes;
+    // work counters, the two routing words, then the error word (zeroed per call)
+    const size_t o_cnt = take(cnt_bytes + 12);
+    const size_t o_sync = o_cnt + cnt_bytes;
+    const size_t o_err = o_sync + 8;
     if (w && base) {
         char* b = static_cast<char*>(base);
         w->z = reinterpret_cast<float*>(b + o_z);
@@ -111,12 +113,14 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->plan = reinterpret_cast<Plan*>(b + o_plan);
         w->counters = reinterpret_cast<uint32_t*>(b + o_cnt);
         w->counter_bytes = cnt_bytes;
+        w->logits_done = reinterpret_cast<uint32_t*>(b + o_sync);
+        w->route_ready = reinterpret_cast<uint32_t*>(b + o_sync + 4);
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
         w->xe = reinterpret_cast<int32_t*>(b + o_xe);
         w->x16 = w->xq;   // the prefill path uses these bytes instead of the decode preparation
         w->h16 = w->hq;
         w->zero_words = w->counters;
-        w->n_zero = (int)((cnt_bytes + 4) / 4);
+        w->n_zero = (int)((cnt_bytes + 12) / 4);
     }
     return at;
 }
@@ -221,15 +225,32 @@ int check_common(const mq_layer_cfg* cfg, int32_t T, const void* x, const float*
 
 // Routing, permutation and the per-call set-up of the expert-FFN path:
 // mode 0 = routing only, 1 = decode (prepared tokens + work plan),
-// 2 = prefill (fp16 tokens for the grouped GEMM).
+// 2 = prefill (fp16 tokens for the grouped GEMM).  Forward calls first clear
+// their per-call words.  fuse (decode on the mma.sync kernels): the logits
+// kernel's last CTA routes and permutes, and the expert-FFN kernel follows
+// it directly, waiting on the published flags.
 int run_route(const Dims& d, const void* x, const float* router_w, const float* bias, Work& w,
-              cudaStream_t s, int mode) {
+              cudaStream_t s, int mode, bool fuse = false) {
     const bool fwd = mode != 0;
-    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, mode == 1 ? w.xq : nullptr, w.xs,
-                             mode == 2 ? w.x16 : nullptr, w.xe, fwd ? w.zero_words : nullptr, fwd ? w.n_zero : 0,
-                             s) != cudaSuccess)
-        return MQ_ECUDA;
+    if (fwd && launch_zero(w.zero_words, w.n_zero, s) != cudaSuccess) return MQ_ECUDA;
     Plan* plan = mode == 1 ? w.plan : nullptr;
+    if (fuse) {
+        FusedRoute fr{};
+        fr.d = d;
+        fr.bias = bias;
+        // the expert-FFN kernel reads the plan and the permutation only
+        fr.idx = w.idx; fr.wts = w.wts; fr.offsets = nullptr; fr.perm = w.perm; fr.inv = nullptr;
+        fr.active = nullptr; fr.plan = plan;
+        fr.logits_done = w.logits_done;
+        fr.route_ready = w.route_ready;
+        if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, w.xq, w.xs, nullptr, w.xe, &fr,
+                                 s) != cudaSuccess)
+            return MQ_ECUDA;
+        return MQ_OK;
+    }
+    if (launch_router_logits(d, static_cast<const uint16_t*>(x), router_w, w.z, mode == 1 ? w.xq : nullptr, w.xs,
+                             mode == 2 ? w.x16 : nullptr, w.xe, nullptr, s) != cudaSuccess)
+        return MQ_ECUDA;
     if (d.T <= kFusedRouteTokens) {
         // decode-sized batch: top-k, permutation and work plan in one CTA
         if (launch_route_permute(d, w.z, bias, w.idx, w.wts, w.offsets, w.perm, w.inv, w.active, plan, s) !=
@@ -293,7 +314,7 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     const int pm = path_mode();
     const bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
     const bool tc = !prefill && decode_tc_fits(d) && (pm == 3 || !decode_mma_fits(d));
-    rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1);
+    rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1, !prefill && !tc);
     if (rc != MQ_OK) return rc;
     if (prefill) {
         if (launch_prefill(d, tab, w, out, s) != cudaSuccess) return MQ_ECUDA;

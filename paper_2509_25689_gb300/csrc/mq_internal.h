@@ -60,6 +60,8 @@ struct Work {
     float* pdn;        // [A][H] down outputs per assignment (combined by a last pass)
     uint32_t* counters;  // item counters and last-arriver counts (zeroed per call)
     size_t counter_bytes;
+    uint32_t* logits_done;  // logits CTAs that published their logits and prepared tokens (zeroed per call)
+    uint32_t* route_ready;  // set (release) once the routing result is written (zeroed per call)
     uint32_t* err;     // device error word (bounded waits that ran out)
     __half* x16;       // [T][H] tokens in fp16 for the prefill GEMM (shares xq's bytes),
                        // each token scaled by 2^-xe[t]
@@ -118,9 +120,29 @@ void prefer_max_shared(void (*kernel)(KArgs...)) {
 }
 #endif
 
+// Routing fused into the logits kernel (decode path): the CTA that finishes
+// last routes every token and permutes (idx/wts/offsets/perm/inv/active/plan
+// as the permutation kernel writes them), then sets route_ready with a
+// release store; every CTA first counts itself in logits_done after its
+// logits and prepared tokens are written.  Both words must be zero at launch.
+struct FusedRoute {
+    int on;
+    uint32_t n_ctas;          // filled in by the launcher
+    Dims d;
+    const float* bias;
+    int32_t* idx; float* wts; int32_t* offsets; int32_t* perm; int32_t* inv; int32_t* active;
+    Plan* plan;
+    uint32_t* logits_done;
+    uint32_t* route_ready;
+};
+
+// Clears n words (the per-call counters) once the previous kernel on the
+// stream is done; the first kernel of every forward call.
+cudaError_t launch_zero(uint32_t* words, int n, cudaStream_t s);
+// fused: nullptr, or the routing outputs for the fused last-CTA routing
+// (one CTA per expert x 8 tokens; the logits kernel with activation prep)
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
-                                 __half* x16, int32_t* xe, uint32_t* zero_words, int n_zero,
-                                 cudaStream_t s);
+                                 __half* x16, int32_t* xe, const FusedRoute* fused, cudaStream_t s);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, Plan* plan, cudaStream_t s);

@@ -68,7 +68,8 @@ __device__ __forceinline__ void route_token(const float* __restrict__ z, const f
         const int e = lane + 32 * m;
         s[m] = 0.0f; u[m] = 0.0f; grp[m] = 0;
         if (e < E) {
-            s[m] = canonical_sigmoid(z[(size_t)t * E + e]);
+            // through L2: the logits may come from other CTAs of the same grid
+            s[m] = canonical_sigmoid(__ldcg(z + (size_t)t * E + e));
             u[m] = __fadd_rn(s[m], bias ? bias[e] : 0.0f);
             grp[m] = e / gs;
             uw[e] = u[m];
@@ -173,6 +174,119 @@ __device__ __forceinline__ void route_token(const float* __restrict__ z, const f
         if (lane == j) { sel = bi; mys = sv; }   // lane j keeps slot j
     }
     // weights: s_j / sum(s), summed in slot order, times routed_scale
+    if (lane < K) {
+        idx[(size_t)t * K + lane] = sel;
+        wts[(size_t)t * K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), routed_scale);
+    }
+    if (sel_out != nullptr) *sel_out = sel;
+}
+
+
+// The same selection for one token, written for a cold SM: it runs once per
+// decode call in whichever CTA routes, where every distinct line of
+// instructions costs an instruction fetch from the memory system.  So the
+// per-expert work is a loop (not unrolled), and the top-k is K rounds of a
+// warp-wide "largest key, then lowest id" over each lane's 8 candidates
+// (equal to route_token's per-lane ordering plus head merge).  Scratch:
+// sc[2 * kMaxExperts] floats (u, then s), g_sh[G].  Results are identical to
+// route_token's.
+__device__ __forceinline__ void route_token_compact(const float* __restrict__ z, const float* __restrict__ bias,
+                                                    int E, int G, int Gk, int K, float routed_scale, int t,
+                                                    float* sc, float* g_sh, int32_t* __restrict__ idx,
+                                                    float* __restrict__ wts, int* sel_out) {
+    const int lane = threadIdx.x & 31;
+    const int gs = E / G;
+    float* u_sh = sc;
+    float* s_sh = sc + 256;
+#pragma unroll 1
+    for (int e = lane; e < E; e += 32) {
+        const float sv = canonical_sigmoid(__ldcg(z + (size_t)t * E + e));
+        s_sh[e] = sv;
+        u_sh[e] = __fadd_rn(sv, bias ? bias[e] : 0.0f);
+    }
+    __syncwarp();
+    // group score = sum of the two largest u of the group (as route_token)
+    if (G <= 16) {
+        int P = 2;
+        while (P * 2 * G <= 32) P *= 2;
+        const int g = lane / P, sub = lane % P;
+        float top1 = -INFINITY, top2 = -INFINITY;
+        if (g < G) {
+            const float* ug = u_sh + g * gs;
+#pragma unroll 1
+            for (int i = sub; i < gs; i += P) {
+                const float v = ug[i];
+                top2 = fmaxf(top2, fminf(top1, v));
+                top1 = fmaxf(top1, v);
+            }
+        }
+#pragma unroll 1
+        for (int off = P >> 1; off >= 1; off >>= 1) {
+            const float o1 = __shfl_xor_sync(kFull, top1, off), o2 = __shfl_xor_sync(kFull, top2, off);
+            top2 = fmaxf(fminf(top1, o1), fmaxf(top2, o2));
+            top1 = fmaxf(top1, o1);
+        }
+        if (g < G && sub == 0) g_sh[g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
+    } else {
+#pragma unroll 1
+        for (int g = lane; g < G; g += 32) {
+            float top1 = -INFINITY, top2 = -INFINITY;
+            const float* ug = u_sh + g * gs;
+#pragma unroll 1
+            for (int i = 0; i < gs; ++i) {
+                const float v = ug[i];
+                top2 = fmaxf(top2, fminf(top1, v));
+                top1 = fmaxf(top1, v);
+            }
+            g_sh[g] = gs == 1 ? top1 : __fadd_rn(top1, top2);
+        }
+    }
+    __syncwarp();
+    // kept groups: fewer than topk_group groups rank before them
+    uint64_t kept = 0;
+#pragma unroll 1
+    for (int h = 0; h < 2; ++h) {
+        const int g = lane + 32 * h;
+        bool keep = false;
+        if (g < G) {
+            const uint32_t kg = ord_key(g_sh[g]);
+            int before = 0;
+#pragma unroll 1
+            for (int g2 = 0; g2 < G; ++g2) {
+                const uint32_t k2 = ord_key(g_sh[g2]);
+                before += (k2 > kg || (k2 == kg && g2 < g)) ? 1 : 0;
+            }
+            keep = before < Gk;
+        }
+        kept |= (uint64_t)__ballot_sync(kFull, keep) << (32 * h);
+    }
+    uint32_t key[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        const int e = lane + 32 * m;
+        key[m] = (e < E && ((kept >> (e / gs)) & 1)) ? ord_key(u_sh[e]) : 0u;
+    }
+    int sel = 0;
+    float ssum = 0.0f, mys = 0.0f;
+#pragma unroll 1
+    for (int j = 0; j < K; ++j) {
+        // this lane's best: largest key, the lower id first among equal keys
+        uint32_t bk = 0u;
+        int bm = 0;
+#pragma unroll
+        for (int m = 0; m < 8; ++m)
+            if (key[m] > bk) { bk = key[m]; bm = m; }
+        const uint32_t kmax = __reduce_max_sync(kFull, bk);
+        const int bi = (int)__reduce_min_sync(kFull, bk == kmax ? (uint32_t)(lane + 32 * bm) : 0xffffffffu);
+        if ((bi & 31) == lane) {
+#pragma unroll
+            for (int m = 0; m < 8; ++m)
+                if (m == (bi >> 5)) key[m] = 0u;
+        }
+        const float sv = s_sh[bi];
+        ssum = __fadd_rn(ssum, sv);   // slot order, identical on every lane
+        if (lane == j) { sel = bi; mys = sv; }
+    }
     if (lane < K) {
         idx[(size_t)t * K + lane] = sel;
         wts[(size_t)t * K + lane] = __fmul_rn(__fdiv_rn(mys, ssum), routed_scale);

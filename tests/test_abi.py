@@ -137,6 +137,7 @@ def test_bench_step_bytes_counts_each_touched_expert_once(mq):
     assert b["quantized"] == 6 * (gu + dn) + sh
     assert b["gateup_mma"] == 6 * gu + 2 * mq.mq_packed_size(4, I, H) + H * 2 + (K + 1) * I * 4
     assert b["down_mma"] == 6 * dn + mq.mq_packed_size(4, H, I) + (K + 1) * I * 4 + H * 4
+    assert b["ffn_mma"] == b["gateup_mma"] + b["down_mma"]   # the one decode FFN kernel reads both
     assert b["router_logits"] == E * H * 4 + H * 2 + E * 4
 
 
@@ -153,9 +154,9 @@ def test_binding_refuses_short_buffers(mq):
 
 def test_bench_traffic_only_for_the_captured_workload():
     import bench
-    t = bench._profiled_traffic("gateup_mma")
+    t = bench._profiled_traffic("ffn_mma")
     assert t is None or t > 0
-    assert bench._profiled_traffic("gateup_mma", "v3_decode_t1_k6") is None
+    assert bench._profiled_traffic("ffn_mma", "v3_decode_t1_k6") is None
     assert bench._profiled_traffic("router_logits") is None
 
 
