@@ -71,6 +71,44 @@ def test_never_selected_experts_score_zero_and_go_last():
     assert R.prune(idx, w, 5, 0.5, 0.6)[0] == [0, 1, 2]
 
 
+def test_fixed_weight_rounding_by_hand():
+    # units of 2^-64, ties to even
+    assert R.fixed_weight(1.0) == 2 ** 64
+    assert R.fixed_weight(0.625) == 5 * 2 ** 61
+    assert R.fixed_weight(2.0 ** -70) == 0              # 1/64 unit
+    assert R.fixed_weight(3 * 2.0 ** -66) == 1          # 0.75 unit
+    assert R.fixed_weight(2.0 ** -65) == 0              # exactly half: to even (0)
+    assert R.fixed_weight(3 * 2.0 ** -65) == 2          # 1.5 units: to even (2)
+    assert R.fixed_weight(5 * 2.0 ** -65) == 2          # 2.5 units: to even (2)
+    assert R.fixed_weight(-0.75) == -3 * 2 ** 62
+
+
+def test_weight_sum_is_order_free_and_exact():
+    # 1 + 256 * 2^-60: a running double sum loses every small term
+    # (1 + 2^-60 rounds back to 1); the exact sum is 1 + 2^-52
+    idx = [[0]] * 257
+    w = [[1.0]] + [[2.0 ** -60]] * 256
+    assert R.expert_importance(idx, w, 1, 0.0) == [(1.0 + 2.0 ** -52) / 257]
+    assert R.expert_importance(idx[::-1], w[::-1], 1, 0.0) == [(1.0 + 2.0 ** -52) / 257]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_weight_sums_equal_fsum(seed):
+    # every float32 weight >= 2^-40 is a whole number of 2^-64 units, so the
+    # sum must be the correctly rounded sum of the weights (math.fsum)
+    import math
+    rng = np.random.default_rng(seed)
+    T, K, E = 300, 4, 16
+    idx = np.stack([rng.choice(E, K, replace=False) for _ in range(T)])
+    w = (rng.random((T, K)) * 2.0 ** rng.integers(-40, 20, (T, K))).astype(np.float32)
+    w = np.maximum(w, np.float32(2.0 ** -40))
+    count, fsum = R.expert_counts_and_sums(idx.tolist(), w.tolist(), E)
+    for e in range(E):
+        sel = w[idx == e].astype(np.float64)
+        assert count[e] == sel.size
+        assert fsum[e] / 2 ** 64 == math.fsum(sel.tolist())
+
+
 # --------------------------------------------------- library vs the oracle ---
 @pytest.fixture(scope="module")
 def mq():
