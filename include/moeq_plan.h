@@ -79,13 +79,31 @@ int mq_plan_precision(const mq_plan_cfg* cfg, const mq_plan_tensor* tensors, int
  * 0..n-1.  n >= 0. */
 int mq_binary_partition_order(int32_t n, int32_t* order_out);
 
+/* Hardware-aware activation adjustment (Sec. 3.2).  After pruning to a
+ * retention ratio retain, every layer activates k_pruned = ceil(retain *
+ * k_orig - 1e-12) experts per token; per device the per-layer counts
+ * k_i <= k_pruned are tuned so that FLOPs_active = 2 sum_i k_i P_i (P_i =
+ * params_per_expert[i], one expert of layer i) fits flops_budget: starting
+ * from k_pruned everywhere, one layer at a time gives up one expert, the
+ * layers taken in binary-partition order (as mq_binary_partition_order,
+ * cycling through it), none below 1.  k_out: host int32 [n_layers];
+ * flops_out (or NULL): FLOPs_active of the plan, above flops_budget only when
+ * every k_i is 1.  k_orig in 1..256, retain in (0, 1], n_layers in 0..4096,
+ * every P_i in 1..2^40, flops_budget >= 0; MQ_OK or MQ_EINVAL (nothing
+ * written).  topk_group needs no change: k_i never rises. */
+int mq_activation_plan(int32_t k_orig, double retain, int32_t n_layers, const int64_t* params_per_expert,
+                       int64_t flops_budget, int32_t* k_out, int64_t* flops_out);
+
 /* Expert-importance scores for pruning (Sec. 3.1).  Over a routed
  * calibration stream of n_tokens tokens (moe_quant_route's topk_idx /
  * topk_w copied to the host: int32 / fp32 [n_tokens, top_k], ids in
- * 0..n_experts-1, finite weights):
+ * 0..n_experts-1, finite weights with |w| < 2^32):
  *   f_e = tokens selecting e / n_tokens, s_e = mean weight of e's
- *   selections (0 if none), I_e = alpha f_e + (1 - alpha) s_e,
- * counts and sums taken in token-major slot order in double precision.
+ *   selections (0 if none), I_e = alpha f_e + (1 - alpha) s_e.
+ * The weight sum of e is order-free: every weight rounded to the nearest
+ * multiple of 2^-64 (ties to even; exact for |w| >= 2^-40), the multiples
+ * added exactly, the total rounded once to double and divided by the count.
+ * The device histogram (moeq_stats.h) gives the same bits.
  * The ceil(retain * n_experts) experts of largest I_e (ties to the lower id)
  * are kept: keep_out (host int32, room for n_experts) receives their ids in
  * ascending order and *n_keep_out their number; scores_out (host double

@@ -88,6 +88,12 @@ def _load():
         "mq_binary_partition_order": (ctypes.c_int, [i32, vp]),
         "mq_expert_importance": (ctypes.c_int, [vp, vp, i32, i32, i32, ctypes.c_double, ctypes.c_double, vp, vp,
                                                 ctypes.POINTER(ctypes.c_int32)]),
+        "mq_activation_plan": (ctypes.c_int, [i32, ctypes.c_double, i32, vp, i64, vp, ctypes.POINTER(ctypes.c_int64)]),
+        "mq_expert_stats_bytes": (sz, [i32]),
+        "mq_expert_stats_reset": (ctypes.c_int, [vp, i32, vp]),
+        "mq_expert_stats_add": (ctypes.c_int, [vp, i32, vp, vp, i32, i32, vp]),
+        "mq_expert_stats_scores": (ctypes.c_int, [vp, i32, ctypes.c_double, ctypes.c_double, vp, vp, vp, vp,
+                                                  ctypes.POINTER(ctypes.c_int32), vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -99,7 +105,8 @@ _lib = _load()
 EXPORTED = ("mq_packed_size", "mq_pack", "mq_unpack", "mq_unpack_device", "moe_quant_workspace_size",
             "moe_quant_forward", "moe_quant_forward_noalloc", "moe_quant_route", "mq_strerror", "mq_set_path", "mq_profile_enable",
             "mq_profile_collect", "mq_plan_precision", "mq_binary_partition_order", "moe_quant_status",
-            "moe_quant_status_noalloc", "mq_expert_importance", "mq_test_fail_next_decode")
+            "moe_quant_status_noalloc", "mq_expert_importance", "mq_test_fail_next_decode",
+            "mq_activation_plan", "mq_expert_stats_bytes", "mq_expert_stats_reset", "mq_expert_stats_add", "mq_expert_stats_scores")
 
 
 def _ptr(a):
@@ -332,3 +339,55 @@ def mq_expert_importance(topk_idx, topk_w, n_experts: int, alpha: float = 0.5, r
                                      float(alpha), float(retain), scores.ctypes.data, keep.ctypes.data,
                                      ctypes.byref(nk)))
     return keep[:nk.value], scores[:n_experts]
+
+
+def mq_activation_plan(k_orig: int, retain: float, params_per_expert, flops_budget: int):
+    """Per-layer activated experts k_i and the plan's FLOPs_active (Sec. 3.2)."""
+    import numpy as np
+    P = np.ascontiguousarray(np.asarray(params_per_expert, dtype=np.int64).reshape(-1))
+    k = np.empty(max(P.size, 1), np.int32)
+    fl = ctypes.c_int64(0)
+    _check("mq_activation_plan", _lib.mq_activation_plan(int(k_orig), float(retain), int(P.size), P.ctypes.data,
+                                                         int(flops_budget), k.ctypes.data, ctypes.byref(fl)))
+    return k[:P.size], int(fl.value)
+
+
+# ------------------------------------------- device expert statistics ---
+def mq_expert_stats_bytes(n_experts: int) -> int:
+    return int(_lib.mq_expert_stats_bytes(n_experts))
+
+
+def mq_expert_stats_reset(stats, n_experts: int, stream=None):
+    _need("mq_expert_stats_reset", stats, mq_expert_stats_bytes(n_experts))
+    return _check("mq_expert_stats_reset", _lib.mq_expert_stats_reset(_ptr(stats), n_experts, _stream(stream)))
+
+
+def mq_expert_stats_add(stats, n_experts: int, topk_idx, topk_w, n_tokens: int, top_k: int, stream=None):
+    """stats: device buffer of mq_expert_stats_bytes(n_experts) bytes;
+    topk_idx / topk_w: device int32 / fp32 [n_tokens, top_k]."""
+    _need("mq_expert_stats_add", stats, mq_expert_stats_bytes(n_experts))
+    if n_tokens > 0:
+        _need("mq_expert_stats_add", topk_idx, 4 * n_tokens * top_k)
+        _need("mq_expert_stats_add", topk_w, 4 * n_tokens * top_k)
+    return _check("mq_expert_stats_add", _lib.mq_expert_stats_add(_ptr(stats), n_experts, _ptr(topk_idx),
+                                                                  _ptr(topk_w), n_tokens, top_k, _stream(stream)))
+
+
+def mq_expert_stats_scores(stats, n_experts: int, alpha: float, retain: float, freq=None, mean_w=None, scores=None,
+                           keep=None, stream=None) -> int:
+    """Writes the requested device outputs; returns ceil(retain n_experts),
+    the number of ids written to keep."""
+    _need("mq_expert_stats_scores", stats, mq_expert_stats_bytes(n_experts))
+    nk = ctypes.c_int32(0)
+    # no outputs: only the kept count, nothing enqueued
+    _check("mq_expert_stats_scores", _lib.mq_expert_stats_scores(_ptr(stats), n_experts, float(alpha), float(retain),
+                                                                 None, None, None, None, ctypes.byref(nk), None))
+    for a in (freq, mean_w, scores):
+        if a is not None:
+            _need("mq_expert_stats_scores", a, 8 * n_experts)
+    if keep is not None:
+        _need("mq_expert_stats_scores", keep, 4 * nk.value)
+    _check("mq_expert_stats_scores",
+           _lib.mq_expert_stats_scores(_ptr(stats), n_experts, float(alpha), float(retain), _ptr(freq), _ptr(mean_w),
+                                       _ptr(scores), _ptr(keep), None, _stream(stream)))
+    return int(nk.value)

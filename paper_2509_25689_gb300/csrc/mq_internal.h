@@ -79,7 +79,8 @@ size_t workspace_plan(const Dims& d, void* base, Work* w);
 // init() the first time `slot` is used with the current device (under a
 // process-wide mutex) and returns that device's SM count (0 if the device
 // query failed).  Slots: one per translation unit or kernel group.
-enum SetupSlot : int { kSetupDecode = 0, kSetupPrefill, kSetupTgemv, kSetupRoute, kSetupCombine, kSetupSlots };
+enum SetupSlot : int { kSetupDecode = 0, kSetupPrefill, kSetupTgemv, kSetupRoute, kSetupCombine, kSetupStats,
+                 kSetupSlots };
 int device_setup(int slot, void (*init)());
 
 // Test hook of the bounded waits (mq_test_fail_next_decode): true once after

@@ -10,6 +10,7 @@
 
 #include "moeq.h"
 #include "moeq_plan.h"
+#include "mq_fixsum.h"
 
 extern "C" int mq_expert_importance(const int32_t* topk_idx, const float* topk_w, int32_t n_tokens, int32_t top_k,
                                     int32_t n_experts, double alpha, double retain, double* scores_out,
@@ -19,20 +20,21 @@ extern "C" int mq_expert_importance(const int32_t* topk_idx, const float* topk_w
     if (n_tokens > 0 && (topk_idx == nullptr || topk_w == nullptr)) return MQ_EINVAL;
     if (keep_out == nullptr || n_keep_out == nullptr) return MQ_EINVAL;
     const size_t n = (size_t)n_tokens * (size_t)top_k;
+    std::vector<mq::Fix128> wfix(n);
     for (size_t i = 0; i < n; ++i)
-        if (topk_idx[i] < 0 || topk_idx[i] >= n_experts || !std::isfinite(topk_w[i])) return MQ_EINVAL;
+        if (topk_idx[i] < 0 || topk_idx[i] >= n_experts || !mq::fix_from_float(topk_w[i], wfix[i])) return MQ_EINVAL;
 
-    // counts and weight sums in token-major slot order
+    // counts, and weight sums exact in 2^-64 units (order-free)
     std::vector<int64_t> count(n_experts, 0);
-    std::vector<double> ssum(n_experts, 0.0);
+    std::vector<mq::Fix128> ssum(n_experts, mq::Fix128{0, 0});
     for (size_t i = 0; i < n; ++i) {
         count[topk_idx[i]] += 1;
-        ssum[topk_idx[i]] += (double)topk_w[i];
+        mq::fix_add(ssum[topk_idx[i]], wfix[i]);
     }
     std::vector<double> score(n_experts);
     for (int32_t e = 0; e < n_experts; ++e) {
         const double f = n_tokens > 0 ? (double)count[e] / (double)n_tokens : 0.0;
-        const double s = count[e] > 0 ? ssum[e] / (double)count[e] : 0.0;
+        const double s = count[e] > 0 ? mq::fix_to_double(ssum[e]) / (double)count[e] : 0.0;
         score[e] = alpha * f + (1.0 - alpha) * s;
     }
     const int32_t k = (int32_t)std::ceil(retain * n_experts - 1e-12);

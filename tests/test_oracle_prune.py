@@ -146,3 +146,48 @@ def test_library_argument_checks(mq):
         mq.mq_expert_importance(idx, np.full((2, 2), np.nan, np.float32), 4)
     keep, scores = mq.mq_expert_importance(np.zeros((0, 2), np.int32), np.zeros((0, 2), np.float32), 4, 0.5, 0.5)
     assert list(keep) == [0, 1] and (scores == 0).all()
+
+
+def test_library_exact_sums_hard_weights(mq):
+    # weights over 2^-80 .. 2^31, negatives, zeros, and 1 + 256 * 2^-60 on one
+    # expert: the host routine's fixed-point sums give the oracle's bits
+    rng = np.random.default_rng(5)
+    E, K, T = 40, 4, 800
+    idx = np.stack([rng.choice(E, K, replace=False) for _ in range(T)]).astype(np.int32)
+    w = (rng.random((T, K)) * 2.0 ** rng.integers(-80, 31, (T, K))).astype(np.float32)
+    w[rng.random((T, K)) < 0.1] *= -1
+    w[rng.random((T, K)) < 0.05] = 0.0
+    idx[:257, 0] = 3
+    w[:257, 0] = np.float32(2.0 ** -60)
+    w[0, 0] = np.float32(1.0)
+    for alpha, r in ((0.5, 0.75), (0.0, 0.5)):
+        keep, scores = mq.mq_expert_importance(idx, w, E, alpha, r)
+        rkeep, rscores = R.prune(idx.tolist(), w.tolist(), E, alpha, r)
+        assert list(keep) == rkeep
+        np.testing.assert_array_equal(scores.view(np.uint64), np.array(rscores).view(np.uint64))
+    with pytest.raises(mq.MoeqError):      # |w| >= 2^32 is outside the accumulator's range
+        mq.mq_expert_importance(idx[:1], np.full((1, K), 2.0 ** 32, np.float32), E)
+
+
+def test_device_stats_host_side_checks(mq):
+    # sizes and argument checks that reject (or finish) before any device work
+    assert mq.mq_expert_stats_bytes(0) == 0 and mq.mq_expert_stats_bytes(1025) == 0
+    assert mq.mq_expert_stats_bytes(256) == 16 + 24 * 256
+    buf = np.zeros(mq.mq_expert_stats_bytes(256) + 16, np.uint8)
+    base = buf.ctypes.data
+    stats = base + (-base) % 16
+    assert mq.mq_expert_stats_add(stats, 256, None, None, 0, 8) == 0          # empty batch: nothing enqueued
+    for r, k in ((0.75, 192), (1.0, 256), (0.5, 128), (0.001, 1)):
+        assert mq.mq_expert_stats_scores(stats, 256, 0.5, r) == k == R.keep_count(r, 256)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_reset(stats, 0)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_scores(stats, 256, 1.5, 0.75)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_scores(stats, 256, 0.5, 0.0)
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_add(stats, 256, None, None, 4, 8)                 # null batch
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_add(stats, 256, 16, 16, 4, 33)                    # top_k > 32
+    with pytest.raises(mq.MoeqError):
+        mq.mq_expert_stats_add(stats + 8, 256, 16, 16, 4, 8)                 # misaligned buffer
