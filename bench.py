@@ -145,6 +145,14 @@ def step_bytes(spec, fmts, idx_steps):
     return out
 
 
+def flops_active_per_token(k_layers, P, has_shared):
+    """FLOPs_active = 2 sum_i k_i P_i per token over the layers (Sec. 3.2;
+    P = parameters of one routed expert), and the same with each layer's
+    shared expert (always active) added."""
+    routed = 2 * sum(int(k) for k in k_layers) * P
+    return {"routed": routed, "with_shared": routed + (2 * len(k_layers) * P if has_shared else 0)}
+
+
 def step_flops(spec):
     """Dense-contraction FLOPs per step of the expert FFN kernels: every routed
     assignment and every shared-expert row does gate and up (2 x 2 H I) and
@@ -425,6 +433,8 @@ def measure_layer(spec, K, W, rank=0, world=1, local=0):
                                    f"{spec.n_experts} experts + shared, G={spec.n_groups}/{spec.topk_group}, "
                                    f"top-{spec.top_k}, T={T}", "l2": "flushed (256 MB write) before every step",
                        "parallelism": f"replicas x{world}"},
+            "flops_active_per_token": flops_active_per_token([spec.top_k], spec.expert_param_count(),
+                                                             spec.has_shared),
             "achieved_hbm_gbs": round(gbs, 1), "hbm_frac_of_measured": round(gbs / peak, 4),
             "hbm_frac_of_8tbs": round(gbs / 8000.0, 4), "quantized_bytes_per_step": int(quant_bytes / K),
             "roofline": roof,
@@ -487,8 +497,8 @@ def run_native(args):
             if not args.no_cpu_baseline:
                 r["cpu_baseline"] = cpu_baseline(HostOracleLayer(sp, seed=0), xf, openmp=True)
             subs.append(r)
-        for tokens in (1, 8):
-            subs.append(measure_stack(get_config("v3_stack20"), tokens, 64, 5, rank, world, local,
+        for name, tokens in (("v3_stack20", 1), ("v3_stack20", 8), ("v3_stack20_ki", 1)):
+            subs.append(measure_stack(get_config(name), tokens, 64, 5, rank, world, local,
                                       cpu=not args.no_cpu_baseline))
         result["sub_records"] = subs
     if world > 1:
@@ -508,21 +518,35 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
     from workloads.synth import draw_tokens
     from dataclasses import replace
 
+    import paper_2509_25689_gb300 as mq
     spec = replace(base, tokens=T)
     L = spec.n_layers
-    layers = [BenchLayer(spec, seed=1000 * rank + l) for l in range(L)]
+    P = spec.expert_param_count()
+    ex = spec.extra
+    if "k_orig" in ex:
+        # per-layer activated experts k_i <= ceil(r k_orig) under the
+        # workload's FLOPs budget (the library's activation plan)
+        k_layers, _ = mq.mq_activation_plan(ex["k_orig"], ex["retain"], [P] * L, 2 * ex["budget_expert_acts"] * P)
+        k_layers = [int(v) for v in k_layers]
+    else:
+        k_layers = [spec.top_k] * L
+    kmax = max(k_layers)
+    lspecs = [replace(spec, top_k=k_layers[l]) for l in range(L)]
+    layers = [BenchLayer(lspecs[l], seed=1000 * rank + l) for l in range(L)]
     resident = sum(int(t.numel()) for lay in layers for trip in lay.tensors for t in trip)
     n_pool = max(1, min(W + K, (64 << 20) // (L * T * spec.hidden * 2)))
     x_host = np.stack([np.stack([draw_tokens(5000 + rank * 100003 + i * L + l, T, spec.hidden) for l in range(L)])
                        for i in range(n_pool)])                      # [pool, L, T, H] bf16 bits
     x_dev = torch.from_numpy(x_host.view(np.int16)).cuda()
     xbuf = torch.empty((L, T, spec.hidden), dtype=torch.int16, device="cuda")
-    idx_g = torch.empty((L, T, spec.top_k), dtype=torch.int32, device="cuda")
+    # layer l writes its [T, k_l] ids into its own region of one buffer
+    idx_g = torch.full((L, T * kmax), -1, dtype=torch.int32, device="cuda")
+    idx_views = [idx_g[l, :T * k_layers[l]].view(T, k_layers[l]) for l in range(L)]
     stream = torch.cuda.Stream()
 
     def eager():
         for l, lay in enumerate(layers):
-            lay.forward(xbuf[l], idx_g[l])
+            lay.forward(xbuf[l], idx_views[l])
 
     xbuf.copy_(x_dev[0])
     with torch.cuda.stream(stream):
@@ -537,7 +561,7 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
         graph.replay()
     torch.cuda.synchronize()
 
-    idx_steps = torch.empty((K, L, T, spec.top_k), dtype=torch.int32, device="cuda")
+    idx_steps = torch.empty((K, L, T * kmax), dtype=torch.int32, device="cuda")
     clocks = ClockSampler(local)
     clocks.start()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
@@ -580,10 +604,11 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
     e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in e2e_evs), world, "cuda")
 
     idx_host = idx_steps.cpu().numpy()
+    step_idx = lambda i, l: idx_host[i, l, :T * k_layers[l]].reshape(T, k_layers[l])
     touched = 0
     for i in range(K):
         for l, lay in enumerate(layers):
-            sb = step_bytes(spec, lay.fmts, [idx_host[i, l]])[0]
+            sb = step_bytes(lspecs[l], lay.fmts, [step_idx(i, l)])[0]
             touched += sb["quantized"]
     peak, peak_src = _peaks()
     gbs = touched / (dev_ms / 1e3) / 1e9
@@ -596,10 +621,17 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
             "data": "synthetic (seeded random packed weights on device; fresh N(0,1) bf16 tokens per layer per step)",
             "config": {"workload": f"{spec.name}: {L} independent V3 layers (hidden {spec.hidden}, inter "
                                    f"{spec.inter}, {spec.n_experts} mixed-format experts + shared Q8_0 each), "
-                                   f"T={T} per layer", "resident_weight_bytes": resident,
+                                   f"T={T} per layer" + (f", k_i <= {kmax} per layer (activation plan for "
+                                                         f"{ex['budget_expert_acts']} expert activations per token)"
+                                                         if "k_orig" in ex else ""),
+                       "resident_weight_bytes": resident,
                        "l2": "not flushed: each step reads several GB of weights (> 129 MB L2)",
                        "graph": f"the {L} layer calls captured once in a CUDA graph",
                        "parallelism": f"replicas x{world}"},
+            "activated_experts_per_layer": k_layers,
+            "flops_active_per_token": flops_active_per_token(k_layers, P, spec.has_shared),
+            "activated_experts_per_layer": k_layers,
+            "flops_active_per_token": flops_active_per_token(k_layers, P, spec.has_shared),
             "achieved_hbm_gbs": round(gbs, 1), "hbm_frac_of_measured": round(gbs / peak, 4),
             "hbm_frac_of_8tbs": round(gbs / 8000.0, 4), "quantized_bytes_per_step": int(touched / K),
             "kernels": [{"name": n, "launches": c, "total_ms": round(ms, 4)} for n, c, ms in kstats],
@@ -612,7 +644,7 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
         dominant = max(kstats, key=lambda s: s[2]) if kstats else None
         if dominant:
             name, launches, tot_ms = dominant
-            per_launch = sum(step_bytes(spec, lay.fmts, [idx_host[0, l]])[0].get(name, 0)
+            per_launch = sum(step_bytes(lspecs[l], lay.fmts, [step_idx(0, l)])[0].get(name, 0)
                              for l, lay in enumerate(layers)) / L
             avg_s = tot_ms / launches / 1e3
             result["roofline"] = {"bound": "hbm", "kernel": name, "achieved": round(per_launch / avg_s / 1e9, 1),
@@ -621,10 +653,11 @@ def measure_stack(base, T, K, W, rank=0, world=1, local=0, cpu=True):
                                   "algorithmic_bytes_per_launch": int(per_launch),
                                   "avg_launch_us": round(avg_s * 1e6, 2)}
         if world == 1 and cpu:
-            host = HostOracleLayer(spec, seed=0)
+            host = HostOracleLayer(lspecs[0], seed=0)
             cb = cpu_baseline(host, x_host[0, 0], openmp=True)
             cb["value"] = cb["value"] / L      # a token goes through every layer
-            cb["sample"] = f"one layer of the stack, divided by its {L} layers: " + cb["sample"]
+            cb["sample"] = (f"one layer of the stack (k = {k_layers[0]}), divided by its {L} layers: " +
+                            cb["sample"])
             result["cpu_baseline"] = cb
     del layers, x_dev, xbuf, graph
     torch.cuda.empty_cache()

@@ -143,3 +143,35 @@ extern "C" int mq_plan_precision(const mq_plan_cfg* cfg, const mq_plan_tensor* t
     if (total_bits64_out) *total_bits64_out = total;
     return MQ_OK;
 }
+
+// Activation adjustment (Sec. 3.2): k_pruned = ceil(r k_orig) per layer, then
+// one expert at a time off the layers in binary-partition order (cycling,
+// none below 1) until 2 sum k_i P_i fits the budget.
+extern "C" int mq_activation_plan(int32_t k_orig, double retain, int32_t n_layers, const int64_t* params_per_expert,
+                                  int64_t flops_budget, int32_t* k_out, int64_t* flops_out) {
+    if (k_orig < 1 || k_orig > 256 || !(retain > 0.0 && retain <= 1.0) || n_layers < 0 || n_layers > 4096 ||
+        flops_budget < 0)
+        return MQ_EINVAL;
+    if (n_layers > 0 && (params_per_expert == nullptr || k_out == nullptr)) return MQ_EINVAL;
+    for (int32_t i = 0; i < n_layers; ++i)
+        if (params_per_expert[i] < 1 || params_per_expert[i] > (int64_t(1) << 40)) return MQ_EINVAL;
+    const int32_t kp = (int32_t)std::ceil(retain * k_orig - 1e-12);
+    std::vector<int32_t> k(n_layers, kp);
+    // 2 * 256 * 2^40 * 4096 < 2^63
+    int64_t flops = 0;
+    for (int32_t i = 0; i < n_layers; ++i) flops += 2 * (int64_t)kp * params_per_expert[i];
+    std::vector<int32_t> order;
+    bp_order(n_layers, order);
+    int64_t above_one = kp > 1 ? n_layers : 0;   // layers that can still give up an expert
+    for (size_t pos = 0; flops > flops_budget && above_one > 0; ++pos) {
+        const int32_t l = order[pos % order.size()];
+        if (k[l] > 1) {
+            --k[l];
+            flops -= 2 * params_per_expert[l];
+            if (k[l] == 1) --above_one;
+        }
+    }
+    std::copy(k.begin(), k.end(), k_out);
+    if (flops_out) *flops_out = flops;
+    return MQ_OK;
+}

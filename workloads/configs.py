@@ -92,18 +92,13 @@ CONFIGS = {
     # 5: 20 independent layers, decode at batch 1 and 8, 64 steps
     "v3_stack20": _v3(name="v3_stack20", tokens=1, mixed=True, n_layers=20, steps=64,
                       extra={"batches": (1, 8)}),
+    # 5 with per-layer activated experts (Sec. 3.2): k_pruned = ceil(0.75 * 8)
+    # = 6, then k_i <= 6 tuned to a budget of 110 expert activations per token
+    # over the 20 layers (FLOPs_active = 2 * 110 * P), 10 layers at 5 and 10 at 6
+    "v3_stack20_ki": _v3(name="v3_stack20_ki", tokens=1, mixed=True, n_layers=20, steps=64, top_k=6,
+                         extra={"batches": (1, 8), "k_orig": 8, "retain": 0.75, "budget_expert_acts": 110}),
 }
 
 
 def get_config(name: str) -> LayerSpec:
     return CONFIGS[name]
-
-
-def activation_adjusted_k(r: float, k_orig: int) -> int:
-    """k_pruned = ceil(r * k_orig) (Sec. 3.2, Hardware-Aware Activation Adjustment)."""
-    return int(math.ceil(r * k_orig - 1e-12))
-
-
-def flops_active(k_per_layer, params_per_expert) -> float:
-    """FLOPs_active ~= 2 * sum_i k_i P_i per token (Sec. 3.2)."""
-    return 2.0 * sum(k * p for k, p in zip(k_per_layer, params_per_expert))
