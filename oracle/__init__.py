@@ -20,8 +20,8 @@ _SO = os.path.join(_HERE, f"liboracle_{platform.machine()}.so")
 # threads, identical arithmetic per row/token (OMP_NUM_THREADS sets the count)
 _SO_OMP = os.path.join(_HERE, f"liboracle_omp_{platform.machine()}.so")
 
-Q2_K, Q3_K, Q4_K, Q8_0 = 1, 2, 3, 4
-FORMATS = {"Q2_K": Q2_K, "Q3_K": Q3_K, "Q4_K": Q4_K, "Q8_0": Q8_0}
+Q2_K, Q3_K, Q4_K, Q8_0, Q6_K, BF16 = 1, 2, 3, 4, 5, 6
+FORMATS = {"Q2_K": Q2_K, "Q3_K": Q3_K, "Q4_K": Q4_K, "Q8_0": Q8_0, "Q6_K": Q6_K, "BF16": BF16}
 
 
 class OracleLayer(ctypes.Structure):

@@ -11,7 +11,9 @@
  * What each part follows, and what pins it (tests/test_oracle_*.py):
  *
  *  - Block formats (Sec. 3.3: tensors stored in llama.cpp-style k-quant
- *    block formats Q2_K/Q3_K/Q4_K and Q8; Sec. 4.1 implementation details).
+ *    block formats Q2_K/Q3_K/Q4_K/Q6_K and Q8, the planner's upgrade
+ *    targets for small and medium tensors being Q8 and Q6; a bf16 format
+ *    for tensors kept unquantized; Sec. 4.1 implementation details).
  *    The paper gives no byte layout, so the layout below is this project's
  *    own "-style" definition: every format blocks along the contraction
  *    (column) axis, rows are padded to whole blocks with zero weights and
@@ -21,7 +23,12 @@
  *    bytes are cut in 64-byte units, unit-major; see unit_at).  Code bits
  *    are placed in "pair order" (see code_pos_*: the two codes of a pair
  *    sit 16 bits apart in one word), sub-block scale fields in "slot
- *    order" (slot_of); Q8_0 codes are stored offset by 128.
+ *    order" (slot_of); Q8_0 codes are stored offset by 128.  Q6_K: 16
+ *    sub-blocks of 16, fp16 d, an 8-bit scale per sub-block stored offset
+ *    by 128, 6-bit codes q in 0..63 for the value d * sc * (q - 32), kept
+ *    as a low-nibble plane (code_pos_4bit16) and a high-two-bit plane
+ *    (code_pos_2bit).  BF16: 32-weight blocks of raw bf16 values in MMA
+ *    fragment order (bf16_pos).
  *      PINNED by hand-built blocks (tests/golden/hand_blocks.json), by
  *      single-bit placement tests, by grid blocks that must re-pack to
  *      themselves, and by nearest-grid-point brute force on random blocks.
@@ -92,6 +99,13 @@ static uint16_t float_to_half(float f) {
 
 static float bf16_to_float(uint16_t b) { return bits_to_f32((uint32_t)b << 16); }
 
+/* fp32 -> bf16, round to nearest even (finite inputs) */
+static uint16_t float_to_bf16(float f) {
+    uint32_t u = f32_to_bits(f);
+    uint32_t lsb = (u >> 16) & 1u;
+    return (uint16_t)((u + 0x7FFFu + lsb) >> 16);
+}
+
 /* ------------------------------------------------------------------ */
 /* Format geometry                                                      */
 /* ------------------------------------------------------------------ */
@@ -121,6 +135,11 @@ static int get_geom(int fmt, geom* g) {
     case ORC_Q8_0: g->qk = 32; g->nplanes = 2;
         g->bytes[0] = 2; g->bytes[1] = 32;
         g->unit[0] = 2; g->unit[1] = 32; return 0;
+    case ORC_Q6_K: g->qk = 256; g->nplanes = 4;
+        g->bytes[0] = 2; g->bytes[1] = 16; g->bytes[2] = 128; g->bytes[3] = 64;
+        g->unit[0] = 2; g->unit[1] = 16; g->unit[2] = 64; g->unit[3] = 64; return 0;
+    case ORC_BF16: g->qk = 32; g->nplanes = 1;
+        g->bytes[0] = 64; g->unit[0] = 64; return 0;
     default: return -1;
     }
 }
@@ -198,6 +217,21 @@ static void code_pos_8bit(int k, int* word, int* bit) {
     *word = m >> 1;
     *bit = 16 * e + 8 * (m & 1);
 }
+
+/* 4-bit codes of 16-wide sub-blocks (Q6_K low nibbles): 32 words/block,
+   two 64-byte units (unit = j / 8).  Sub-block j takes words
+   16 (j / 8) + 4 (j % 4) + 2 ((j / 4) % 2) + 0..1; pair m at word m / 4,
+   bit 4 (m % 4). */
+static void code_pos_4bit16(int k, int* word, int* bit) {
+    int j = k >> 4, p = k & 15, m = p >> 1, e = p & 1;
+    *word = 16 * (j >> 3) + 4 * (j & 3) + 2 * ((j >> 2) & 1) + (m >> 2);
+    *bit = 16 * e + 4 * (m & 3);
+}
+
+/* BF16 block of 32: position (in 16-bit units) of weight k, so that the
+   four words a tensor-core fragment takes for k = 2t, 2t+1, 8+2t, 9+2t,
+   16+2t, 17+2t, 24+2t, 25+2t are contiguous. */
+static int bf16_pos(int k) { return 8 * ((k & 7) >> 1) + 2 * (k >> 3) + (k & 1); }
 
 static uint32_t get_word(const uint8_t* p, int w) {
     const uint8_t* b = p + 4 * w;
@@ -352,6 +386,39 @@ int oracle_pack(int fmt, const float* w, int64_t rows, int64_t cols,
                         code_pos_1bit(k, &wd, &bt); put_field(rec[3], wd, bt, 1, (uint32_t)(code >> 2));
                     }
                 }
+            } else if (fmt == ORC_Q6_K) {
+                /* symmetric: per sub-block the element of largest |w| maps to
+                   code -32; 8-bit sub-block scales against d = max|scale| / 127 */
+                float scale[16], maxabs = 0.0f;
+                for (int j = 0; j < 16; j++) {
+                    float amax = wb[16 * j];
+                    for (int i = 1; i < 16; i++)
+                        if (fabsf(wb[16 * j + i]) > fabsf(amax)) amax = wb[16 * j + i];
+                    scale[j] = amax / -32.0f;
+                    if (fabsf(scale[j]) > maxabs) maxabs = fabsf(scale[j]);
+                }
+                uint16_t dh = float_to_half(maxabs / 127.0f);
+                float df = half_to_float(dh);
+                wr16(rec[0], dh);
+                for (int j = 0; j < 16; j++) {
+                    int scj = df > 0.0f ? clampi(rn(scale[j] / df), -128, 127) : 0;
+                    rec[1][slot_of(j)] = (uint8_t)(scj + 128);
+                    float den = df * (float)scj;
+                    for (int i = 0; i < 16; i++) {
+                        int k = 16 * j + i;
+                        int qi = den != 0.0f ? clampi(rn(wb[k] / den), -32, 31) : 0;
+                        int code = qi + 32;
+                        int wd, bt;
+                        code_pos_4bit16(k, &wd, &bt); put_field(rec[2], wd, bt, 4, (uint32_t)(code & 15));
+                        code_pos_2bit(k, &wd, &bt); put_field(rec[3], wd, bt, 2, (uint32_t)(code >> 4));
+                    }
+                }
+            } else if (fmt == ORC_BF16) {
+                for (int k = 0; k < 32; k++) {
+                    uint16_t h = float_to_bf16(wb[k]);
+                    if ((h & 0x7F80u) == 0x7F80u) return -2;   /* rounds beyond the bf16 range */
+                    wr16(rec[0] + 2 * bf16_pos(k), h);
+                }
             } else { /* Q8_0 */
                 float amax = 0.0f;
                 for (int k = 0; k < 32; k++) if (fabsf(wb[k]) > amax) amax = fabsf(wb[k]);
@@ -420,6 +487,17 @@ int oracle_unpack(int fmt, const uint8_t* src, int64_t rows, int64_t cols, float
                     int hi = (int)get_field(rec[3], wd, bt, 1);
                     int q = lo | (hi << 2);
                     v = (df * (float)(s - 32)) * (float)(q - 4);
+                } else if (fmt == ORC_Q6_K) {
+                    float df = half_to_float(rd16(rec[0]));
+                    int s = (int)rec[1][slot_of(k / 16)] - 128;
+                    code_pos_4bit16(k, &wd, &bt);
+                    int lo = (int)get_field(rec[2], wd, bt, 4);
+                    code_pos_2bit(k, &wd, &bt);
+                    int hi = (int)get_field(rec[3], wd, bt, 2);
+                    int q = lo | (hi << 4);
+                    v = (df * (float)s) * (float)(q - 32);
+                } else if (fmt == ORC_BF16) {
+                    v = bf16_to_float(rd16(rec[0] + 2 * bf16_pos(k)));
                 } else {
                     float df = half_to_float(rd16(rec[0]));
                     code_pos_8bit(k, &wd, &bt);

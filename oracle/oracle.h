@@ -16,8 +16,9 @@
  *     "Framework Overview" of Sec. 3.
  *   - num_experts_per_tok (k) and topk_group over the pruned expert set:
  *     Sec. 3.2 (Hardware-Aware Activation Adjustment).
- *   - k-quant style block formats (Q2_K/Q3_K/Q4_K) and Q8: Sec. 3.3 and
- *     the implementation details of Sec. 4.1.  The paper defers the byte
+ *   - k-quant style block formats (Q2_K/Q3_K/Q4_K/Q6_K) and Q8, and bf16
+ *     tensors kept unquantized: Sec. 3.3 (the level ladder of the
+ *     precision planner) and the implementation details of Sec. 4.1.  The paper defers the byte
  *     layout to llama.cpp; the layouts here are this project's own
  *     definitions of "-style" formats (not GGUF byte-compatible).
  *
@@ -33,7 +34,7 @@
 extern "C" {
 #endif
 
-enum { ORC_Q2_K = 1, ORC_Q3_K = 2, ORC_Q4_K = 3, ORC_Q8_0 = 4 };
+enum { ORC_Q2_K = 1, ORC_Q3_K = 2, ORC_Q4_K = 3, ORC_Q8_0 = 4, ORC_Q6_K = 5, ORC_BF16 = 6 };
 
 typedef struct {
     int32_t hidden, inter, n_experts, n_groups, topk_group, top_k;
