@@ -9,7 +9,8 @@
  *     topk_group kept groups over the pruned experts and
  *     num_experts_per_tok = k experts per token (Sec. 3.2),
  *   - each expert tensor stored in its own k-quant style format
- *     (Q2_K/Q3_K/Q4_K) or Q8_0 (Sec. 3.3; Sec. 4.1 implementation details),
+ *     (Q2_K/Q3_K/Q4_K/Q6_K), Q8_0, or kept unquantized in bf16 (Sec. 3.3,
+ *     the planner's level ladder; Sec. 4.1 implementation details),
  *   - SwiGLU expert FFNs, router-weighted combine and an always-on shared
  *     expert (Fig. 1, framework overview of Sec. 3).
  *
@@ -27,12 +28,14 @@
  *
  * Packed tensor format (all formats): a tensor has `rows` output rows and
  * `cols` contraction columns.  Each row is cut into blocks of QK weights
- * along the columns (QK = 256 for Q2_K/Q3_K/Q4_K, 32 for Q8_0), the last
+ * along the columns (QK = 256 for Q2_K/Q3_K/Q4_K/Q6_K, 32 for Q8_0 and
+ * BF16), the last
  * block padded with zero weights, and rows are padded with zero rows to a
  * multiple of 32 (a tile).  Every field of a block lives in its own plane,
  * starting at a multiple of 256 bytes from the tensor base.  A field's
  * record (the field of one row and one block) is stored in units of at most
- * 64 bytes (only the Q4_K codes have two units), and unit u of the record of
+ * 64 bytes (the Q4_K and Q6_K 4-bit codes have two units), and unit u of
+ * the record of
  * (row r, block b) sits at byte
  *   ((((r / 32) * nb + b) * nu + u) * 32 + r % 32) * unit_bytes
  * of its plane (nb blocks per row, nu units per record), so any block range
@@ -44,22 +47,33 @@
  *   Q3_K: d fp16 | 12 B 6-bit sub-scales (stored sc+32) | 64 B low 2 bits | 32 B high bit
  *         w = (d*(s-32))*(q-4),         sub-blocks of 16
  *   Q8_0: d fp16 | 32 B codes stored as q+128,  w = d*q
+ *   Q6_K: d fp16 | 16 B 8-bit sub-scales (stored sc+128) | 128 B low 4 bits
+ *         of q | 64 B high 2 bits of q,
+ *         w = (d*(s-128))*(q-32),       sub-blocks of 16
+ *   BF16: 64 B: the block's 32 weights as bf16, weight k at 16-bit slot
+ *         8((k%8)/2) + 2(k/8) + k%2,  w = the bf16 value
  * Inside a block, weight k is in sub-block j = k/n (n = 16 for 2-bit and
- * 1-bit codes, 32 for 4-bit and 8-bit codes) at pair m = (k%n)/2, e = k%2.
- * Codes are little-endian 32-bit words ("pair order"):
- *   2-bit: word 4(j%4) + j/4,          bit 16e + 2m
+ * 1-bit codes and for the Q6_K low 4 bits, 32 for Q4_K and 8-bit codes) at
+ * pair m = (k%n)/2, e = k%2.  Codes are little-endian 32-bit words ("pair
+ * order"):
+ *   2-bit: word 4(j%4) + j/4,          bit 16e + 2m   (Q2_K; Q3_K low bits;
+ *                                                      Q6_K high bits)
  *   1-bit: word 2(j%4) + j/8,          bit 16e + 8((j/4)%2) + m
- *   4-bit: word 16(j/4) + 4(j%4) + m/4, bit 16e + 4(m%4)
+ *   4-bit: word 16(j/4) + 4(j%4) + m/4, bit 16e + 4(m%4)   (Q4_K)
+ *   Q6_K 4-bit: word 16(j/8) + 4(j%4) + 2((j/4)%2) + m/4, bit 16e + 4(m%4)
  *   8-bit: word m/2,                   bit 16e + 8(m%2)
- * Sub-block j of Q2_K/Q3_K sits in slot u = 4((j%8)/2) + 2(j/8) + j%2:
+ * Sub-block j of Q2_K/Q3_K/Q6_K sits in slot u = 4((j%8)/2) + 2(j/8) + j%2:
  *   Q2_K: byte u = sc | m << 4.
+ *   Q6_K: byte u = sc + 128.
  *   Q3_K: bits 4u..4u+3 of bytes 0-7 (LE) = low nibble of s,
  *         bits 2u..2u+1 of bytes 8-11 (LE) = high two bits of s.
  * Q4_K sub-block j (< 8): byte j = (sc & 15) | (m & 15) << 4; bits 4j..4j+1
  *   of bytes 8-11 (LE) = sc >> 4, bits 4j+2..4j+3 = m >> 4.
  * These are this library's own "-style" layouts; the paper defers layouts to
  * llama.cpp and they are not GGUF byte-compatible.  Every decoded weight is
- * exact in fp32 except for the single rounding of the final subtraction.
+ * exact in fp32 except for the single rounding of the final subtraction
+ * (Q2_K/Q4_K) or product (Q6_K: d*(s-128) is exact, its product with q-32
+ * is rounded once).
  */
 #ifndef MOEQ_H
 #define MOEQ_H
@@ -71,7 +85,7 @@
 extern "C" {
 #endif
 
-typedef enum { MQ_Q2_K = 1, MQ_Q3_K = 2, MQ_Q4_K = 3, MQ_Q8_0 = 4 } mq_format;
+typedef enum { MQ_Q2_K = 1, MQ_Q3_K = 2, MQ_Q4_K = 3, MQ_Q8_0 = 4, MQ_Q6_K = 5, MQ_BF16 = 6 } mq_format;
 
 enum {
     MQ_OK = 0,
@@ -112,9 +126,9 @@ size_t mq_packed_size(int fmt, int64_t rows, int64_t cols);
 
 /* Host quantizer (Sec. 3.3 quantizes tensors to a block format; the rule is
  * this library's deterministic nearest-grid rule).  w: host fp32
- * [rows, cols] row-major, finite; dst: host buffer of dst_bytes >=
- * mq_packed_size.  Returns MQ_OK, MQ_EINVAL (incl. non-finite w) or
- * MQ_EFORMAT. */
+ * [rows, cols] row-major, finite (for BF16: rounding to a finite bf16);
+ * dst: host buffer of dst_bytes >= mq_packed_size.  Returns MQ_OK,
+ * MQ_EINVAL (incl. non-finite w) or MQ_EFORMAT. */
 int mq_pack(int fmt, const float* w, int64_t rows, int64_t cols, void* dst, size_t dst_bytes);
 
 /* Host dequantizer: src host packed tensor -> dst host fp32 [rows, cols]
@@ -151,7 +165,16 @@ size_t moe_quant_workspace_size(const mq_layer_cfg* cfg, int32_t n_tokens);
  * output still beyond the fp16 range after that scaling (it needs
  * |h| > 65504 * 2^2e, far outside trained models) is not passed on silently:
  * the call's error word gets bit 16 and moe_quant_status returns
- * MQ_EDEVICE.
+ * MQ_EDEVICE.  Weights: the decode kernels take every format's decoded
+ * values as they are (BF16 tensors as bf16 MMA operands, the token or h
+ * split into bf16 hi + lo); the prefill grouped GEMM decodes weights to
+ * fp16, which holds every BF16 weight with 2^-14 <= |w| < 65520 exactly
+ * (smaller ones to the nearest fp16 subnormal); a BF16 weight of |w| >=
+ * 65520 sets bit 64 of the error word instead.  The tcgen05 decode GEMV
+ * (mq_set_path mode 3) takes Q2_K/Q3_K/Q4_K/Q8_0 only: a layer with a
+ * Q6_K or BF16 tensor is refused there (MQ_EFORMAT) and, when that kernel
+ * would be chosen automatically (hidden or inter not a multiple of 256),
+ * runs on the grouped GEMM instead.
  * Shape rules (MQ_ESHAPE): hidden and inter multiples of 128 (hidden <=
  * 32768, inter <= 16384), 1 <= n_experts <= 256, n_experts % n_groups == 0,
  * n_groups <= 64, 1 <= topk_group <= n_groups, 1 <= top_k <= 32 and
@@ -195,7 +218,8 @@ int moe_quant_forward_noalloc(const mq_layer_cfg* cfg, int32_t n_tokens, const v
  * 1 / 2 a decode GEMV consumer / producer gave up a wait, 32 a decode down
  * item gave up waiting for its expert's SwiGLU output, 4 a prefill GEMM
  * wait, 8 a tcgen05 GEMV wait, 16 a prefill SwiGLU output beyond the fp16
- * range (see moe_quant_forward).  This call
+ * range, 64 a BF16 weight beyond the prefill GEMM's fp16 range (see
+ * moe_quant_forward).  This call
  * waits for the stream (cudaStreamSynchronize), reads the word and returns
  * MQ_OK (0 bits), MQ_EDEVICE (some bit set; err_bits, or NULL, receives the
  * bits), or the argument codes of moe_quant_forward (MQ_EWORKSPACE for a

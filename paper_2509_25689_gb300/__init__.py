@@ -14,8 +14,8 @@ import os
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libmoeq.so")
 
-MQ_Q2_K, MQ_Q3_K, MQ_Q4_K, MQ_Q8_0 = 1, 2, 3, 4
-FORMATS = {"Q2_K": MQ_Q2_K, "Q3_K": MQ_Q3_K, "Q4_K": MQ_Q4_K, "Q8_0": MQ_Q8_0}
+MQ_Q2_K, MQ_Q3_K, MQ_Q4_K, MQ_Q8_0, MQ_Q6_K, MQ_BF16 = 1, 2, 3, 4, 5, 6
+FORMATS = {"Q2_K": MQ_Q2_K, "Q3_K": MQ_Q3_K, "Q4_K": MQ_Q4_K, "Q8_0": MQ_Q8_0, "Q6_K": MQ_Q6_K, "BF16": MQ_BF16}
 MQ_OK = 0
 MQ_EINVAL, MQ_EFORMAT, MQ_EALIGN, MQ_ESHAPE, MQ_EWORKSPACE, MQ_ECUDA, MQ_EDEVICE, MQ_ERANGE = range(-1, -9, -1)
 

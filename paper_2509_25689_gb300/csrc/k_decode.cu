@@ -53,6 +53,14 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// bf16 x bf16 -> fp32 (the BF16 weight tiles)
+__device__ __forceinline__ void mma16816_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                              uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 __device__ __forceinline__ float h2f(uint32_t bits16) { return __half2float(__ushort_as_half((unsigned short)bits16)); }
 
 struct VecSrc {
@@ -185,26 +193,26 @@ struct __align__(16) Hdr {
 // token pieces in a stage: the family fragments and the per-superblock
 // statistics, each for the stage's ks superblocks
 struct TokLay { int x, s, stride; };
+// (BF16: the bf16 hi and lo operands of the token instead)
 __host__ __device__ __forceinline__ TokLay tok_lay(int fmt, int ks) {
-    (void)fmt;
     TokLay t;
     int at = 0;
     t.x = at; at += ks * 512;
-    t.s = at; at += ks * kStatFloats * 4;
+    t.s = at; at += ks * (fmt == kBF16 ? 512 : kStatFloats * 4);
     t.stride = (at + 127) & ~127;
     return t;
 }
 
 __host__ __device__ __forceinline__ int weight_stage_bytes(int fmt, int ks) {
     const PlaneBytes pb = plane_bytes(fmt);
-    const int nblk = fmt == kQ80 ? 8 * ks : ks;
+    const int nblk = block_len(fmt) == 32 ? 8 * ks : ks;
     int at = 0;
     for (int p = 0; p < pb.n; ++p) at += (32 * nblk * pb.b[p] + 127) & ~127;
     return at;
 }
 // superblocks per stage for a format and token count (fits a ring slot)
 __host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok, int stage_bytes) {
-    int ks = fmt == kQ80 ? kStageSb / 2 : kStageSb;
+    int ks = fmt == kQ80 ? kStageSb / 2 : fmt == kBF16 ? 2 : kStageSb;
     while (ks > 1 && weight_stage_bytes(fmt, ks) + ntok * tok_lay(fmt, ks).stride > stage_bytes) --ks;
     return ks;
 }
@@ -231,7 +239,7 @@ __host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int f
     const int nsb = down ? (d.I + 255) / 256 : (d.H + 255) / 256;
     const TensorLayout L = tensor_layout(fmt, down ? d.H : d.I, down ? d.I : d.H);
     const PlaneBytes pb = plane_bytes(fmt);
-    const int bmul = fmt == kQ80 ? 8 : 1;
+    const int bmul = block_len(fmt) == 32 ? 8 : 1;   // Q8_0 / BF16: 8 blocks of 32 per superblock
     G.per = (int16_t)stage_sb(fmt, ntok, kSlotBytes);
     G.nst = (int16_t)((nsb + G.per - 1) / G.per);
     G.npl = (int16_t)pb.n;
@@ -264,7 +272,7 @@ struct DecodeArgs {
     uint32_t* err;
     uint64_t wait_ns;        // limit of every bounded wait
     int fail_first_stage;    // test hook: the producer posts nothing for its first stage
-    Geo geo[2][4][kDecodeTok];   // [down][format][tokens], computed on the host
+    Geo geo[2][kNumFormats][kDecodeTok];   // [down][format][tokens], computed on the host
 };
 
 struct ItemDesc {            // decoded item (producer side)
@@ -468,6 +476,99 @@ __device__ __forceinline__ void tile_mma(const Geo& h, uint32_t st, int jj, int 
                              (sub4(cB[2 * tl + 1], wi) >> sh) & mk, XA[hm][mm], XB[hm][mm]);
             }
         }
+    } else if (FMT == kQ6K) {
+        // q = low nibble + 16 * high two bits.  Nibble MMAs as Q4_K's (operand
+        // family F4: pair m carries 2^(4 (m & 1))) on 16-wide sub-blocks; the
+        // high two bits sit in the Q2_K code order and go into the same
+        // accumulators weighed by 16: each pair's field is moved by one of
+        // three shifts of its word (<< 4, none, >> 6) to a bit position p
+        // <= 8 of its fp16 half, and the F4 operand is scaled by the exact
+        // power of two 2^(4 + 4 (m & 1) - p) (at most 2^2 / 2^6 for even / odd
+        // m, which the F4 range leaves room for).
+        uint4 n0[NR], n1[NR], c[NR];   // nibbles: unit 0 (sub-blocks t, t+4), unit 1 (t+8, t+12); high bits
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int r = rec_of(i) - jj * 32;
+            n0[i] = lds128(st + w2 + ((jj * 2 + 0) * 32 + r) * 64 + 16 * t);
+            n1[i] = lds128(st + w2 + ((jj * 2 + 1) * 32 + r) * 64 + 16 * t);
+            c[i] = lds128(st + w3 + rec_of(i) * 64 + 16 * t);
+        }
+        uint32_t XA[2][8], XB[2][8];
+#pragma unroll
+        for (int gm = 0; gm < 2; ++gm) {
+            ld_frag8(own0 ? xb + 32 * (8 * gm + t) : zaddr, XA[gm]);
+            ld_frag8(own1 ? xb + 32 * (8 * gm + 4 + t) : zaddr, XB[gm]);
+        }
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const uint32_t mk = (m & 1) ? 0x00F000F0u : 0x000F000Fu;
+            const int sh = (m & 2) ? 8 : 0;
+            const int wi = m >> 2;   // word of the pair within a sub-block's two
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm)
+#pragma unroll
+                for (int tl = 0; tl < NT; ++tl) {
+                    const uint4& ua = gm ? n1[2 * tl] : n0[2 * tl];
+                    const uint4& ub = gm ? n1[2 * tl + 1] : n0[2 * tl + 1];
+                    mma16816(T.DD[tl][gm][m & 1], (sub4(ua, wi) >> sh) & mk, (sub4(ub, wi) >> sh) & mk,
+                             (sub4(ua, 2 + wi) >> sh) & mk, (sub4(ub, 2 + wi) >> sh) & mk, XA[gm][m], XB[gm][m]);
+                }
+        }
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            // word shift (left 4 / none / right 6), resulting bit position, operand scale 2^e
+            const int shl = m <= 1 ? 4 : 0, shr = m >= 5 ? 6 : 0;
+            const int pos = 2 * m + shl - shr;
+            const int e = 4 + 4 * (m & 1) - pos;
+            const uint32_t mk = 0x00030003u << pos;
+            const uint32_t sc16 = (uint32_t)(15 + e) << 10;
+            const __half2 scl = __halves2half2(__ushort_as_half((unsigned short)sc16), __ushort_as_half((unsigned short)sc16));
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm) {
+                uint32_t ua = XA[gm][m], ub = XB[gm][m];
+                if (e != 0) {
+                    const __half2 xa = __hmul2(*reinterpret_cast<const __half2*>(&ua), scl);
+                    const __half2 xb2 = __hmul2(*reinterpret_cast<const __half2*>(&ub), scl);
+                    ua = *reinterpret_cast<const uint32_t*>(&xa);
+                    ub = *reinterpret_cast<const uint32_t*>(&xb2);
+                }
+#pragma unroll
+                for (int tl = 0; tl < NT; ++tl) {
+                    const uint32_t qa0 = sub4(c[2 * tl], 2 * gm), qa1 = sub4(c[2 * tl + 1], 2 * gm);
+                    const uint32_t qb0 = sub4(c[2 * tl], 2 * gm + 1), qb1 = sub4(c[2 * tl + 1], 2 * gm + 1);
+                    mma16816(T.DD[tl][gm][(m + 1) & 1], ((qa0 << shl) >> shr) & mk, ((qa1 << shl) >> shr) & mk,
+                             ((qb0 << shl) >> shr) & mk, ((qb1 << shl) >> shr) & mk, ua, ub);
+                }
+            }
+        }
+    } else if (FMT == kBF16) {
+        // bf16 weights times the token's bf16 hi and lo operands (family FB /
+        // FBL), blocks 8 jj + (0..7) of 32; fragment order puts a lane's four
+        // words of a row (k = 2t.., 8+2t.., 16+2t.., 24+2t..) together.  Only
+        // lanes g = 0 supply the token (column 0 of B), so column 0 of D is the
+        // row's dot product and the other columns stay zero.
+        const uint32_t hb = tb + h.tx + jj * 512, lb = tb + h.ts + jj * 512;
+        const bool own = g == 0;
+#pragma unroll 2
+        for (int b = 0; b < 8; ++b) {
+            const uint4 Bh = lds128(own ? hb + 64 * b + 16 * t : zaddr);
+            const uint4 Bl = lds128(own ? lb + 64 * b + 16 * t : zaddr);
+            uint4 a[NR];
+#pragma unroll
+            for (int i = 0; i < NR; ++i) {
+                const int r = rec_of(i) - jj * 32;
+                a[i] = lds128(st + h.woff[0] + ((8 * jj + b) * 32 + r) * 64 + 16 * t);
+            }
+#pragma unroll
+            for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+                for (int tl = 0; tl < NT; ++tl) {
+                    const uint32_t a0 = sub4(a[2 * tl], 2 * kc), a1 = sub4(a[2 * tl + 1], 2 * kc);
+                    const uint32_t a2 = sub4(a[2 * tl], 2 * kc + 1), a3 = sub4(a[2 * tl + 1], 2 * kc + 1);
+                    mma16816_bf16(T.DD[tl][kc][0], a0, a1, a2, a3, sub4(Bh, 2 * kc), sub4(Bh, 2 * kc + 1));
+                    mma16816_bf16(T.DD[tl][kc][1], a0, a1, a2, a3, sub4(Bl, 2 * kc), sub4(Bl, 2 * kc + 1));
+                }
+        }
     } else {   // Q8_0: blocks 8 jj + (0..7), pairs 8 half .. 8 half + 7, four accumulators per row tile
         uint4 cA[NR], cB[NR];   // rows: blocks t and t+4
 #pragma unroll
@@ -502,7 +603,16 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
     const int rbase = jj * 32 + 16 * rt0 + g;
     auto rec_of = [&](int i) { return rbase + 16 * (i >> 1) + 8 * (i & 1); };
 
-    if (FMT == kQ2K || FMT == kQ3K) {
+    if (FMT == kBF16) {
+        // column 0 of D holds each row's sum (the other columns are zero)
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int tl = i >> 1, hl = i & 1;
+            acc[i] += (T.DD[tl][0][0][2 * hl] + T.DD[tl][0][1][2 * hl]) + (T.DD[tl][1][0][2 * hl] + T.DD[tl][1][1][2 * hl]);
+        }
+        return;
+    }
+    if (FMT == kQ2K || FMT == kQ3K || FMT == kQ6K) {
         // slot-ordered scale fields of each row: slot 4t + b (b = 2 * group + col)
         // holds the lane's sub-block of D[group][col].  Fields are turned into
         // fp16 pairs (b0, b2) / (b1, b3) whose values are field * 2^-24 (masked
@@ -524,7 +634,21 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
                     D[gm][cc] = T.DD[tl][gm][0][2 * hl + cc] + T.DD[tl][gm][1][2 * hl + cc];
             const int rec = rec_of(i);
             const float d = h2f(lds16(st + w0 + rec * 2)) * 16777216.0f;
-            if (FMT == kQ2K) {
+            if (FMT == kQ6K) {
+                // scale bytes hold s + 128: masked into fp16 subnormal pairs
+                // (s + 128) * 2^-24, minus 128 * 2^-24 (exact), widened; the
+                // 2^24 is folded into d
+                const uint32_t f = lds32(st + w1 + rec * 16 + 4 * t);
+                const uint32_t fa = f & 0x00FF00FFu, fb = (f >> 8) & 0x00FF00FFu;
+                const __half2 o128 = __halves2half2(__ushort_as_half((unsigned short)128), __ushort_as_half((unsigned short)128));
+                const __half2 va = __hsub2(*reinterpret_cast<const __half2*>(&fa), o128);
+                const __half2 vb = __hsub2(*reinterpret_cast<const __half2*>(&fb), o128);
+                const float2 s02 = __half22float2(va), s13 = __half22float2(vb);   // slots (0, 2), (1, 3)
+                const float P0 = fmaf(D[0][0], cf0, -32.0f * S[0]), P1 = fmaf(D[0][1], cf0, -32.0f * S[1]);
+                const float P2 = fmaf(D[1][0], cf1, -32.0f * S[2]), P3 = fmaf(D[1][1], cf1, -32.0f * S[3]);
+                const float a = fmaf(s13.y, P3, fmaf(s02.y, P2, fmaf(s13.x, P1, s02.x * P0)));
+                acc[i] = fmaf(d, a, acc[i]);
+            } else if (FMT == kQ2K) {
                 // byte b = sc | m << 4; bytes 1 and 3 moved down to bytes 0 and 2
                 const float dm = h2f(lds16(st + w1 + rec * 2)) * 1048576.0f;   // m sits 4 bits up: 2^-20
                 const uint32_t f = lds32(st + w2 + rec * 16 + 4 * t);
@@ -629,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     __shared__ int s_fail;           // a bounded wait ran out somewhere in the CTA
     __shared__ int s_touch;
     __shared__ __align__(16) uint32_t zero_blk[8];   // operand B of the lanes that supply none
-    __shared__ Geo geo[2][4][kDecodeTok];
+    __shared__ Geo geo[2][kNumFormats][kDecodeTok];
     const Dims& d = A.d;
     // ---- set-up that does not depend on the routing result runs before the
     // wait for the previous kernel (overlapping its tail)
@@ -682,8 +806,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // most one copy: lanes 0..3 a weight plane, lanes 4.. one piece of one
         // token (family fragments or statistics).  A stage then only advances
         // the source by the stage's first superblock.
-        const VecSrc vx{A.xq, A.xs, (size_t)4 * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
-        const VecSrc vh{A.hq, A.hs, (size_t)4 * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi};
+        const VecSrc vx{A.xq, A.xs, (size_t)kFamSlots * A.nsbx * 256, (size_t)A.nsbx * kStatFloats, A.nsbx};
+        const VecSrc vh{A.hq, A.hs, (size_t)kFamSlots * A.nsbi * 256, (size_t)A.nsbi * kStatFloats, A.nsbi};
         int cur_gu = 0, cur_dn = 0, p_q = 0;
         // weights are read once per call: evict-first in L2, so they do not
         // displace the activations, h and partial outputs the kernel shares
@@ -857,10 +981,15 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         for (int t2 = 1; t2 < kDecodeTok; ++t2) if (tk == t2) v = P.vec[t2];
                         const uint8_t* qv = reinterpret_cast<const uint8_t*>(vs.q + (size_t)v * vs.q_stride);
                         const uint8_t* sv = reinterpret_cast<const uint8_t*>(vs.st + (size_t)v * vs.st_stride);
-                        const int fam = fmt == kQ2K || fmt == kQ3K ? kF2 : fmt == kQ4K ? kF4 : kF8;
+                        const int fam = fmt == kQ2K || fmt == kQ3K ? kF2
+                                      : fmt == kQ4K || fmt == kQ6K ? kF4 : fmt == kBF16 ? kFB : kF8;
                         const uint32_t tb = G->tok0 + tk * G->tstride;
                         if (piece == 0) { c_src = qv + (size_t)fam * vs.nsb * 512; c_stride = 512; c_dst = tb + G->tx; }
-                        if (piece == 1) { c_src = sv; c_stride = kStatFloats * 4; c_dst = tb + G->ts; }
+                        if (piece == 1 && fmt == kBF16) {   // the lo operands instead of statistics
+                            c_src = qv + (size_t)kFBL * vs.nsb * 512; c_stride = 512; c_dst = tb + G->ts;
+                        } else if (piece == 1) {
+                            c_src = sv; c_stride = kStatFloats * 4; c_dst = tb + G->ts;
+                        }
                     }
                 }
                 const int per = G->per;
@@ -967,8 +1096,12 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     tile_cols<kQ2K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 } else if (fmt == kQ3K) {
                     tile_cols<kQ3K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
-                } else {
+                } else if (fmt == kQ4K) {
                     tile_cols<kQ4K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
+                } else if (fmt == kQ6K) {
+                    tile_cols<kQ6K>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
+                } else {
+                    tile_cols<kBF16>(GS, stage, wcol, ks, rt0, tk, zaddr, cur[tk]);
                 }
             }
             // fields needed after the slot is released to the producer
@@ -1030,7 +1163,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     const float w = e_shared ? 1.0f : __ldcg(A.wts + a);
                     const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
                     const int fam = families_of(tab.fmt[e_e][2]);
-                    __half* hq = A.hq + (size_t)a * 4 * A.nsbi * 256;
+                    __half* hq = A.hq + (size_t)a * kFamSlots * A.nsbi * 256;
                     float* hs = A.hs + (size_t)a * A.nsbi * kStatFloats;
                     prep_block32(hv, e_rb, fam, hq, hs, A.nsbi);
                     const int n_rb = d.I / 32;
@@ -1110,7 +1243,7 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     uint64_t test_ns = 0;
     if (take_wait_test(&test_ns)) { A.wait_ns = test_ns; A.fail_first_stage = 1; }
     for (int dn = 0; dn < 2; ++dn)
-        for (int f = 1; f <= 4; ++f)
+        for (int f = 1; f <= kNumFormats; ++f)
             for (int n = 1; n <= kDecodeTok; ++n) make_geo(A.geo[dn][f - 1][n - 1], d, dn == 1, f, n);
     // one token: every item carries one, and the accumulators shrink to one token's
     const bool one = d.T == 1;

@@ -49,6 +49,7 @@ constexpr int kBBytes = kNT * kKC * 2;         // one activation chunk, 32 KB
 constexpr int kSlotBytes = 2 * kABytes + kBBytes;
 constexpr uint32_t kErrMma = 4u;
 constexpr uint32_t kErrRange = 16u;            // an fp16 SwiGLU output would overflow (see the epilogue)
+constexpr uint32_t kErrWeightRange = 64u;      // a BF16 weight beyond the fp16 operand range
 
 struct PrefillArgs {
     Dims d;
@@ -133,6 +134,7 @@ struct Packed {
     uint32_t dd;      // d | dmin << 16 (Q8_0: d of the two blocks)
 };
 
+__device__ __forceinline__ uint2 ldg64u(const uint8_t* p) { return __ldg(reinterpret_cast<const uint2*>(p)); }
 __device__ __forceinline__ uint32_t ldg16u(const uint8_t* p) { return __ldg(reinterpret_cast<const unsigned short*>(p)); }
 
 // Start of one weight row's records in each plane; the record of
@@ -149,6 +151,15 @@ __device__ __forceinline__ RowPtrs row_ptrs(int fmt, const uint8_t* base, const 
 }
 
 __device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, int hf, Packed& P) {
+    if (fmt == kBF16) {
+        // block 2c + hf: only the address of its 64-byte record is carried (the
+        // decode step loads it), which keeps the prefetched fields of the other
+        // formats in registers
+        const uintptr_t bp = reinterpret_cast<uintptr_t>(RP.row[0] + (int64_t)(2 * c + hf) * (32 * 64));
+        P.w[0] = (uint32_t)bp;
+        P.w[1] = (uint32_t)((uint64_t)bp >> 32);
+        return;
+    }
     if (fmt == kQ80) {
         const int64_t b = 2 * c + hf;
         const uint8_t* cp = RP.row[1] + b * (32 * 32);
@@ -168,6 +179,21 @@ __device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, in
         const int j = 2 * cc + hf;
         const uint4 w = ldg128(RP.row[3] + s * (32 * 128) + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
         P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
+        return;
+    }
+    if (fmt == kQ6K) {
+        const uint4 sv = ldg128(RP.row[1] + s * (32 * 16));
+        P.sc[0] = sv.x; P.sc[1] = sv.y; P.sc[2] = sv.z; P.sc[3] = sv.w;
+        // low nibbles: sub-block j = 4 cc + i in unit cc / 2, words 4 i + 2 (cc % 2) + 0..1
+        const uint8_t* np = RP.row[2] + s * (32 * 128) + (cc >> 1) * (kRowTile * 64);
+        const uint8_t* hp = RP.row[3] + s * (32 * 64);
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            const int i = 2 * hf + ii;
+            const uint2 nw = ldg64u(np + 4 * (4 * i + 2 * (cc & 1)));
+            P.w[2 * ii] = nw.x; P.w[2 * ii + 1] = nw.y;
+            P.w[4 + ii] = ldg32(hp + 4 * (4 * i + cc));
+        }
         return;
     }
     if (fmt == kQ2K) {
@@ -201,7 +227,6 @@ struct SBlk {
     uint32_t sc[4];   // scale record
     uint32_t dd;      // d | dmin << 16
 };
-__device__ __forceinline__ uint2 ldg64u(const uint8_t* p) { return __ldg(reinterpret_cast<const uint2*>(p)); }
 __device__ __forceinline__ void load_sblk(int fmt, const RowPtrs& RP, int sb, int hf, SBlk& B) {
     const int64_t s = sb;
     B.dd = ldg16u(RP.row[0] + s * (32 * 2));
@@ -255,12 +280,68 @@ __device__ __forceinline__ uint32_t byte_of(const uint32_t (&w)[4], int i) {
     return (v >> (8 * (i & 3))) & 0xffu;
 }
 
+// Q6_K and BF16 chunks, kept out of line: the formats of most units keep
+// their registers (an out-of-line call saves only what is live around it).
+__device__ __noinline__ bool dequant_store_rare(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
+    if (fmt == kBF16) {
+        const uint8_t* bp = reinterpret_cast<const uint8_t*>((uintptr_t)P.w[0] | ((uintptr_t)P.w[1] << 32));
+        uint32_t wd[16];   // the record: pair p of the block in word 4 (p % 4) + p / 4
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const uint4 q = ldg128(bp + 16 * v);
+            wd[4 * v] = q.x; wd[4 * v + 1] = q.y; wd[4 * v + 2] = q.z; wd[4 * v + 3] = q.w;
+        }
+        bool over = false;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {   // core-matrix row 4 hf + q: k = 8q .. 8q+7 of the block
+            uint32_t o[4];
+#pragma unroll
+            for (int pp = 0; pp < 4; ++pp) {
+                const uint32_t wv = wd[4 * pp + q];   // the pair k = 8q + 2pp, +1
+                const float lo = __uint_as_float(wv << 16), hi = __uint_as_float(wv & 0xFFFF0000u);
+                over |= fmaxf(fabsf(lo), fabsf(hi)) >= 65520.0f;
+                o[pp] = h2u(__floats2half2_rn(lo, hi));
+            }
+            sts128(dst + ((4 * hf + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+        }
+        return over;
+    }
+    if (fmt == kQ6K) {
+        const int cc = c & 3;
+        const float d = half_lo(P.dd);
+        const __half2 k1056 = __float2half2_rn(1056.0f);   // 1024 + the code offset 32
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            const int i = 2 * hf + ii, j = 4 * cc + i;
+            const int sv = (int)byte_of(P.sc, q16_slot(j)) - 128;
+            const __half2 a2 = __float2half2_rn(d * (float)sv);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                uint32_t o[4];
+#pragma unroll
+                for (int mm = 0; mm < 4; ++mm) {
+                    const int m = 4 * q + mm;
+                    const uint32_t nib = (P.w[2 * ii + (m >> 2)] >> (4 * (m & 3))) & 0x000F000Fu;
+                    const uint32_t hi2 = (P.w[4 + ii] >> (2 * m)) & 0x00030003u;
+                    o[mm] = h2u(__hmul2(a2, __hsub2(u2h(nib | (hi2 << 4) | 0x64006400u), k1056)));
+                }
+                sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
+            }
+        }
+        return false;
+    }
+    return false;
+}
+
 // Decode the 64 weights of chunk c of one row (fields in P) to fp16 and store
 // them as 8 core-matrix rows at dst, dst + 128*16, ...  Values follow the
 // format definitions of include/moeq.h; the per-sub-block products d*sc and
-// dmin*m are rounded to fp16 once.
-__device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
+// dmin*m are rounded to fp16 once.  BF16 weights convert exactly where
+// 2^-14 <= |w| < 65520 (below, to the nearest fp16 subnormal); the return
+// value is true if one of them is beyond the fp16 range.
+__device__ __forceinline__ bool dequant_store(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
     const __half2 k1024 = __float2half2_rn(1024.0f);
+    if (fmt == kBF16 || fmt == kQ6K) return dequant_store_rare(fmt, P, c, hf, dst);
     if (fmt == kQ80) {
         const __half2 k1152 = __float2half2_rn(1152.0f);
         {
@@ -277,7 +358,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, i
                 sts128(dst + ((4 * bb + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
         }
-        return;
+        return false;
     }
     const int cc = c & 3;
     const float d = half_lo(P.dd);
@@ -299,7 +380,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, i
                 sts128(dst + ((4 * jj + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
         }
-        return;
+        return false;
     }
     if (fmt == kQ2K) {
         const float dmin = half_hi(P.dd);
@@ -319,7 +400,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, i
                 sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
             }
         }
-        return;
+        return false;
     }
     // Q3_K
     const __half2 k1028 = __float2half2_rn(1028.0f);
@@ -343,6 +424,7 @@ __device__ __forceinline__ void dequant_store(int fmt, const Packed& P, int c, i
             sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
         }
     }
+    return false;
 }
 
 __device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
@@ -450,6 +532,7 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
     int gchunk = 0;        // chunks posted by this CTA so far (ring position and parities)
     int last_committed = -1;   // without the MMA warp: the last chunk thread 0 committed
     bool failed = false;
+    bool w_over = false;   // a BF16 weight of this thread's rows beyond the fp16 range
     int cursor = 0;
 
     // units are claimed from a global counter (their cost varies with the
@@ -524,8 +607,9 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
             if (pl < pb.n) {
                 const TensorLayout& Lx = lane < 4 ? L0 : L1;
                 pf_src = rec_ptr((lane < 4 ? b0 : b1) + Lx.plane[pl], Lx, pb.b[pl], (int64_t)mt * kMT + 32 * warp, 0);
-                pf_bytes = (uint32_t)(32 * pb.b[pl] * (fmt == kQ80 ? 8 : 1));
-                pf_nsb = (int)(fmt == kQ80 ? Lx.blocks_per_row / 8 : Lx.blocks_per_row);
+                const bool b32 = block_len(fmt) == 32;   // Q8_0 / BF16: groups of 8 blocks
+                pf_bytes = (uint32_t)(32 * pb.b[pl] * (b32 ? 8 : 1));
+                pf_nsb = (int)(b32 ? Lx.blocks_per_row / 8 : Lx.blocks_per_row);
                 if ((reinterpret_cast<uintptr_t>(pf_src) & 15u) != 0 || (pf_bytes & 15u) != 0) pf_src = nullptr;
             }
         }
@@ -544,8 +628,8 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
             const uint32_t sbase = ring + s * kSlotBytes;
-            dequant_store(f0, Q0, c, hf, sbase + rr * 16);
-            if (!kDown) dequant_store(f1, Q1, c, hf, sbase + kABytes + rr * 16);
+            if (dequant_store(f0, Q0, c, hf, sbase + rr * 16)) w_over = true;
+            if (!kDown && dequant_store(f1, Q1, c, hf, sbase + kABytes + rr * 16)) w_over = true;
             asm volatile("cp.async.wait_group 1;" ::: "memory");
             // this thread's shared-memory writes (and landed copies) before the
             // tensor cores read them
@@ -562,7 +646,8 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
             last_committed = g;
             return true;
         };
-        if (f0 != kQ80 && (kDown || f1 != kQ80)) {
+        auto sblk_fmt = [](int f) { return f == kQ2K || f == kQ3K || f == kQ4K; };
+        if (sblk_fmt(f0) && (kDown || sblk_fmt(f1))) {
             // superblock-granular fields (Q2_K, Q3_K, Q4_K), one superblock ahead
             const int nS = (nC + 3) / 4;
             SBlk Sa0, Sa1, Sb0, Sb1;
@@ -593,7 +678,7 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
                 if (sb + 1 < nS && !sblock(sb + 1, Sb0, Sb1, Sa0, Sa1)) { failed = true; break; }
             }
         } else {
-            // Q8_0 in the unit: per-chunk fields (blocks of 32), one chunk ahead
+            // Q8_0, Q6_K or BF16 in the unit: per-chunk fields, one chunk ahead
             Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
             load_chunk(f0, RP0, 0, hf, P0);
             if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
@@ -673,6 +758,7 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
         if (tid == 0) s_info[s] = -1;
         mbar_arrive(fbar0 + 8 * s);
     }
+    if (w_over) atomicOr(A.err, kErrWeightRange);
     }   // workers
     __syncthreads();
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");

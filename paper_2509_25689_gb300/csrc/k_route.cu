@@ -452,7 +452,7 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
                                                              int E, float* __restrict__ z,
                                                              __half* __restrict__ xq, float* __restrict__ xs,
                                                              __half* __restrict__ x16, int32_t* __restrict__ xe,
-                                                             const FusedRoute fr) {
+                                                             int x_fams, const FusedRoute fr) {
     __shared__ float part[32][kTok];
     __shared__ float pmax[32][kTok];   // per segment: largest |x| of each token (prefill copy only)
     __shared__ int s_last;
@@ -539,14 +539,14 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     // segment (blocks past the hidden size, up to the 256 padding, are zero).
     if (xq != nullptr) {
         const int nsb = (H + 255) / 256;
-        const size_t qstride = (size_t)4 * nsb * 256, sstride = (size_t)nsb * kStatFloats;
+        const size_t qstride = (size_t)kFamSlots * nsb * 256, sstride = (size_t)nsb * kStatFloats;
         for (int j = 0; j < kTok; ++j) {
             const int t = t0 + j;
             if (t >= T) break;
             for (int jb = 32 * seg + e; jb < 32 * seg + 32 && jb < 8 * nsb; jb += E) {
                 const int k = 32 * jb + lane;
                 const float v = k < H ? bf16_lo(x[(size_t)t * H + k]) : 0.0f;
-                prep_block32(v, jb, (1 << kF2) | (1 << kF4) | (1 << kF8), xq + (size_t)t * qstride,
+                prep_block32(v, jb, x_fams, xq + (size_t)t * qstride,
                              xs + (size_t)t * sstride, nsb);
             }
         }
@@ -610,7 +610,8 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
             threads = (nseg > kPermWarps ? nseg : kPermWarps) * 32;   // the last CTA routes with kPermWarps warps
             smem = sizeof(PermSmem);
         }
-        e = launch_pdl(router_logits_kernel, grid, dim3(threads), smem, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe, fr);
+        e = launch_pdl(router_logits_kernel, grid, dim3(threads), smem, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe,
+                       d.x_fams, fr);
     }
     prof_end(s);
     return e;

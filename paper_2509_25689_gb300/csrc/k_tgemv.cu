@@ -539,7 +539,7 @@ __global__ void __launch_bounds__(kTThreads, 1) tgemv_kernel(const __grid_consta
     const int nsb = kDown ? A.nsbi : A.nsbx;
     const __half* vq = kDown ? A.hq : A.xq;
     const float* vs = kDown ? A.hs : A.xs;
-    const size_t q_stride = (size_t)4 * nsb * 256, s_stride = (size_t)nsb * kStatFloats;
+    const size_t q_stride = (size_t)kFamSlots * nsb * 256, s_stride = (size_t)nsb * kStatFloats;
     int cursor = 0, uc = 0, last_fmt = -1;
     bool ok = true, alive = true;
     // gate/up: both groups take the same item (gate rows, up rows); down: one item per group
@@ -607,7 +607,7 @@ __global__ void __launch_bounds__(kTThreads, 1) tgemv_kernel(const __grid_consta
                     const float gv = acc[tk];
                     const float w = it.shared ? 1.0f : A.wts[a];
                     const float hv = gv / (1.0f + expf(-gv)) * xch[r][tk] * w;
-                    __half* hq = A.hq + (size_t)a * 4 * A.nsbi * 256;
+                    __half* hq = A.hq + (size_t)a * kFamSlots * A.nsbi * 256;
                     float* hs = A.hs + (size_t)a * A.nsbi * kStatFloats;
                     prep_block32(hv, jb, famd, hq, hs, A.nsbi);
                     if (jb == n32 - 1)

@@ -13,20 +13,34 @@
 //   - fp16 copies of xt in natural element order, one per code family, each
 //     element divided by the power of two its code carries: F2 (2-bit code
 //     positions: Q2_K, and Q3_K whose high bit the kernels place right above
-//     the pair's 2-bit code), F4 (4-bit codes: Q4_K), F8 (8-bit codes: Q8_0,
-//     none); slot 1 of the layout is not used;
+//     the pair's 2-bit code), F4 (4-bit codes: Q4_K, and Q6_K whose high two
+//     bits the kernels weigh through shifts and exact operand scalings), F8
+//     (8-bit codes: Q8_0, none);
+//   - for bf16 weights (MMA operands of one type: bf16 x bf16), the value
+//     itself split into bf16 hi = bf16(v) and lo = bf16(v - hi) (hi + lo
+//     holds v to about 16 bits; for a bf16 token lo is 0), each in the
+//     tensor-core fragment order of the BF16 weight blocks (families FB and
+//     FBL);
 //   - the sums sigma * sum(xt) over every 16- and 32-element sub-block (the
 //     sub-block min terms of Q2_K / Q4_K, the -4 offset of Q3_K codes and the
 //     +128 offset of Q8_0 codes).
-// Layout per vector: halves [4 family slots][nsb][256] and, per superblock, a
-// 32-float record {c[8] | S16[16] in slot order | S32[8]}.
+// Layout per vector: halves [kFamSlots family slots][nsb][256] and, per
+// superblock, a 32-float record {c[8] | S16[16] in slot order | S32[8]}.
 #pragma once
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <stdint.h>
 
+#include "mq_layout.h"
+
 namespace mq {
 
-enum Family : int { kF2 = 0, kF4 = 2, kF8 = 3 };
+enum Family : int { kF2 = 0, kFB = 1, kF4 = 2, kF8 = 3, kFBL = 4 };
+constexpr int kFamSlots = 5;
+// families every prepared token gets (the bf16 pair only when a gate or up
+// tensor of the layer is BF16)
+constexpr int kCodeFams = (1 << kF2) | (1 << kF4) | (1 << kF8);
+constexpr int kBf16Fams = (1 << kFB) | (1 << kFBL);
 
 constexpr int kStatFloats = 32;   // floats of statistics per superblock
 constexpr int kStatC = 0, kStatS16 = 8, kStatS32 = 24;
@@ -69,6 +83,13 @@ __device__ __forceinline__ void prep_block32(float v, int jb, int fam_mask, __ha
     if (fam_mask & (1 << kF2)) qs[kF2 * fam_stride] = __float2half_rn(ldexpf(xt, -pair_shift2(m16)));
     if (fam_mask & (1 << kF4)) qs[kF4 * fam_stride] = __float2half_rn(ldexpf(xt, -pair_shift4(m32)));
     if (fam_mask & (1 << kF8)) qs[kF8 * fam_stride] = __float2half_rn(xt);
+    if (fam_mask & (1 << kFB)) {
+        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));   // v - hi is exact
+        unsigned short* fb = reinterpret_cast<unsigned short*>(q + (size_t)s * 256 + ((jb & 7) << 5) + bf16_slot(lane));
+        fb[kFB * fam_stride] = __bfloat16_as_ushort(hi);
+        fb[kFBL * fam_stride] = __bfloat16_as_ushort(lo);
+    }
     const float s16 = half_warp_sum(xt);
     const float s32 = s16 + __shfl_xor_sync(0xffffffffu, s16, 16);
     float* rec = st + (size_t)s * kStatFloats;
@@ -84,7 +105,9 @@ __device__ __forceinline__ void prep_block32(float v, int jb, int fam_mask, __ha
 
 // family mask needed by a weight format
 __host__ __device__ __forceinline__ int families_of(int fmt) {
-    return fmt == 1 || fmt == 2 ? (1 << kF2) : fmt == 3 ? (1 << kF4) : (1 << kF8);
+    return fmt == kQ2K || fmt == kQ3K ? (1 << kF2)
+         : fmt == kQ4K || fmt == kQ6K ? (1 << kF4)
+         : fmt == kBF16 ? kBf16Fams : (1 << kF8);
 }
 
 }  // namespace mq

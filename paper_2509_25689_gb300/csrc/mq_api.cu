@@ -59,6 +59,7 @@ Dims dims_of(const mq_layer_cfg* c, int32_t T) {
     Dims d;
     d.H = c->hidden; d.I = c->inter; d.E = c->n_experts; d.G = c->n_groups; d.Gk = c->topk_group;
     d.K = c->top_k; d.T = T; d.has_shared = c->has_shared; d.routed_scale = c->routed_scale;
+    d.x_fams = kCodeFams;
     return d;
 }
 
@@ -84,9 +85,9 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_off = take((size_t)(d.E + 1) * 4);
     const size_t o_perm = take(TK * 4), o_inv = take(TK * 4);
     const size_t o_act = take((size_t)(d.E + 2) * 4);
-    const size_t o_xq = take((size_t)d.T * 4 * nsbx * 256 * 2);
+    const size_t o_xq = take((size_t)d.T * kFamSlots * nsbx * 256 * 2);
     const size_t o_xs = take((size_t)d.T * nsbx * kStatFloats * 4);
-    const size_t o_hq = take(A * 4 * nsbi * 256 * 2);
+    const size_t o_hq = take(A * kFamSlots * nsbi * 256 * 2);
     const size_t o_hs = take(A * nsbi * kStatFloats * 4);
     const size_t o_pdn = take(A * d.H * 4);
     const size_t o_plan = take(sizeof(Plan));
@@ -291,18 +292,22 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     if (!table || !table->experts || !fmt) return MQ_EINVAL;
     if (cfg->has_shared && !table->shared) return MQ_EINVAL;
     if (n_tokens > 0 && !out) return MQ_EINVAL;
-    const Dims d = dims_of(cfg, n_tokens);
+    Dims d = dims_of(cfg, n_tokens);
     static thread_local ExpertTab tab;
     const int n = d.E + d.has_shared;
+    bool new_fmts = false;   // Q6_K / BF16 tensors: not on the tcgen05 GEMV kernels
     for (int e = 0; e < n; ++e) {
         const mq_expert_weights& ew = e < d.E ? table->experts[e] : *table->shared;
         const void* ps[3] = {ew.gate, ew.up, ew.down};
         for (int j = 0; j < 3; ++j) {
-            if (!valid_format(fmt[3 * e + j])) return MQ_EFORMAT;
+            const int f = fmt[3 * e + j];
+            if (!valid_format(f)) return MQ_EFORMAT;
             if (!ps[j]) return MQ_EINVAL;
             if (!aligned16(ps[j])) return MQ_EALIGN;
             tab.p[e][j] = static_cast<const uint8_t*>(ps[j]);
-            tab.fmt[e][j] = fmt[3 * e + j];
+            tab.fmt[e][j] = (uint8_t)f;
+            new_fmts |= f == kQ6K || f == kBF16;
+            if (f == kBF16 && j < 2) d.x_fams |= kBf16Fams;   // bf16 operands of the tokens
         }
     }
     if (n_tokens == 0) return MQ_OK;
@@ -312,8 +317,14 @@ extern "C" int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, cons
     if (topk_idx) w.idx = topk_idx;
     if (topk_w) w.wts = topk_w;
     const int pm = path_mode();
-    const bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
+    bool prefill = pm == 2 || (pm == 0 && n_tokens >= g_prefill_threshold);
     const bool tc = !prefill && decode_tc_fits(d) && (pm == 3 || !decode_mma_fits(d));
+    if (tc && new_fmts) {
+        // the tcgen05 GEMV kernels take Q2_K/Q3_K/Q4_K/Q8_0 only: a forced
+        // request is refused, an automatic choice goes to the grouped GEMM
+        if (pm == 3) return MQ_EFORMAT;
+        prefill = true;
+    }
     rc = run_route(d, x, router_w, bias, w, s, prefill ? 2 : 1, !prefill && !tc);
     if (rc != MQ_OK) return rc;
     if (prefill) {

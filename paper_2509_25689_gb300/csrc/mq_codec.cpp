@@ -11,6 +11,11 @@
 //     d = fp16(max |scale| / 31), sc = clamp(rne(scale/d), -32, 31),
 //     q = clamp(rne(w / (d*sc)), -4, 3); stored sc+32 and q+4
 //   Q8_0: d = fp16(max|w| / 127), q = clamp(rne(w/d), -127, 127), stored q+128
+//   Q6_K: as Q3_K with codes -32..31 and 8-bit scales: scale = a / -32,
+//     d = fp16(max |scale| / 127), sc = clamp(rne(scale/d), -128, 127),
+//     q = clamp(rne(w / (d*sc)), -32, 31); stored sc+128 and q+32
+//   BF16: each weight rounded to bf16 (nearest, ties to even); a weight that
+//     rounds past the largest finite bf16 is rejected
 // All arithmetic is IEEE fp32 (this file is built with -ffp-contract=off),
 // rne = round half to even; a zero denominator gives code 0.
 #include <cmath>
@@ -82,7 +87,50 @@ void quantize_asym(const float* w, int sub, int L, int S, AsymBlock& out) {
     }
 }
 
+// bf16 of a finite float, nearest-even; false if it rounds to infinity
+bool to_bf16_rne(float f, uint16_t& out) {
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    const uint32_t low = u & 0xffffu, keep = u >> 16;
+    const bool up = low > 0x8000u || (low == 0x8000u && (keep & 1u));
+    const uint32_t h = keep + (up ? 1u : 0u);
+    out = (uint16_t)h;
+    return ((h >> 7) & 0xffu) != 0xffu;
+}
+
 void encode_block(int f, const float* w, uint8_t* const planes[4]) {
+    if (f == kBF16) {
+        for (int k = 0; k < 32; ++k) {
+            uint16_t h = 0;
+            to_bf16_rne(w[k], h);   // range checked before encoding
+            store16(planes[0] + 2 * bf16_slot(k), h);
+        }
+        return;
+    }
+    if (f == kQ6K) {
+        float scale[16], top = 0.0f;
+        for (int j = 0; j < 16; ++j) {
+            float a = w[16 * j];
+            for (int i = 1; i < 16; ++i) if (std::fabs(w[16 * j + i]) > std::fabs(a)) a = w[16 * j + i];
+            scale[j] = a / -32.0f;
+            top = std::fabs(scale[j]) > top ? std::fabs(scale[j]) : top;
+        }
+        const uint16_t dh = to_half_rne(top / 127.0f);
+        const float d = half_bits_to_float(dh);
+        store16(planes[0], dh);
+        for (int j = 0; j < 16; ++j) {
+            const int sc = d > 0.0f ? clip(rne(scale[j] / d), -128, 127) : 0;
+            planes[1][q16_slot(j)] = (uint8_t)(sc + 128);
+            const float den = d * (float)sc;
+            for (int i = 0; i < 16; ++i) {
+                const int k = 16 * j + i;
+                const int q = (den != 0.0f ? clip(rne(w[k] / den), -32, 31) : 0) + 32;
+                set_bits(planes[2], pos4s(k), (uint32_t)q, 15u);
+                set_bits(planes[3], pos2(k), (uint32_t)(q >> 4), 3u);
+            }
+        }
+        return;
+    }
     if (f == kQ80) {
         float amax = 0.0f;
         for (int k = 0; k < 32; ++k) amax = std::fabs(w[k]) > amax ? std::fabs(w[k]) : amax;
@@ -154,8 +202,11 @@ extern "C" int mq_pack(int fmt, const float* w, int64_t rows, int64_t cols, void
     if (rows < 0 || cols < 0 || !dst || (rows * cols > 0 && !w)) return MQ_EINVAL;
     const TensorLayout L = tensor_layout(fmt, rows, cols);
     if (dst_bytes < (size_t)L.total) return MQ_EINVAL;
-    for (int64_t i = 0; i < rows * cols; ++i)
+    for (int64_t i = 0; i < rows * cols; ++i) {
         if (!std::isfinite(w[i])) return MQ_EINVAL;
+        uint16_t h;
+        if (fmt == kBF16 && !to_bf16_rne(w[i], h)) return MQ_EINVAL;
+    }
     uint8_t* out = static_cast<uint8_t*>(dst);
     std::memset(out, 0, (size_t)L.total);
     const int qk = block_len(fmt);

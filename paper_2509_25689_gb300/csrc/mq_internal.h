@@ -22,6 +22,7 @@ struct Dims {
     int H, I, E, G, Gk, K, T;
     int has_shared;
     float routed_scale;
+    int x_fams;   // activation families prepared for the tokens (mq_actprep.cuh)
 };
 
 // Decode work plan: the expert-FFN kernels cut work into items of 32 rows x

@@ -14,7 +14,8 @@
 
 namespace mq {
 
-enum Format : int { kQ2K = 1, kQ3K = 2, kQ4K = 3, kQ80 = 4 };
+enum Format : int { kQ2K = 1, kQ3K = 2, kQ4K = 3, kQ80 = 4, kQ6K = 5, kBF16 = 6 };
+constexpr int kNumFormats = 6;
 
 constexpr int kPlaneAlign = 256;
 constexpr int kRowTile = 32;         // records are grouped in tiles of 32 rows
@@ -22,13 +23,13 @@ constexpr int kMaxExperts = 256;     // routed experts per layer
 constexpr int kMaxTopK = 32;
 constexpr int kMaxGroups = 64;
 
-MQ_HD bool valid_format(int f) { return f >= kQ2K && f <= kQ80; }
+MQ_HD bool valid_format(int f) { return f >= kQ2K && f <= kBF16; }
 
 // weights per block along the contraction axis
-MQ_HD int block_len(int f) { return f == kQ80 ? 32 : 256; }
+MQ_HD int block_len(int f) { return f == kQ80 || f == kBF16 ? 32 : 256; }
 
 // bytes per (row, block) record of each plane, planes in storage order; a
-// record is stored in units of at most 64 bytes (only Q4_K codes have 2)
+// record is stored in units of at most 64 bytes (Q4_K and Q6_K codes have 2)
 struct PlaneBytes { int n; int b[4]; };
 MQ_HD PlaneBytes plane_bytes(int f) {
     PlaneBytes p{0, {0, 0, 0, 0}};
@@ -36,6 +37,8 @@ MQ_HD PlaneBytes plane_bytes(int f) {
     else if (f == kQ2K) { p.n = 4; p.b[0] = 2; p.b[1] = 2; p.b[2] = 16; p.b[3] = 64; }
     else if (f == kQ3K) { p.n = 4; p.b[0] = 2; p.b[1] = 12; p.b[2] = 64; p.b[3] = 32; }
     else if (f == kQ80) { p.n = 2; p.b[0] = 2; p.b[1] = 32; }
+    else if (f == kQ6K) { p.n = 4; p.b[0] = 2; p.b[1] = 16; p.b[2] = 128; p.b[3] = 64; }
+    else if (f == kBF16) { p.n = 1; p.b[0] = 64; }
     return p;
 }
 MQ_HD int unit_bytes(int record_bytes) { return record_bytes > 64 ? 64 : record_bytes; }
@@ -96,6 +99,16 @@ MQ_HD CodePos pos8(int k) {   // Q8_0 codes (stored q + 128), k < 32
     const int m = k >> 1, e = k & 1;
     return CodePos{m >> 1, 16 * e + 8 * (m & 1)};
 }
+// Q6_K low nibbles (16-wide sub-blocks): two 64-byte units, unit = j / 8;
+// sub-block j in words 16 (j / 8) + 4 (j % 4) + 2 ((j / 4) % 2) + 0..1
+MQ_HD CodePos pos4s(int k) {
+    const int j = k >> 4, m = (k & 15) >> 1, e = k & 1;
+    return CodePos{16 * (j >> 3) + 4 * (j & 3) + 2 * ((j >> 2) & 1) + (m >> 2), 16 * e + 4 * (m & 3)};
+}
+// BF16 block of 32: 16-bit position of weight k (tensor-core fragment order:
+// the words for k = 2t, 2t+1 | 8+2t, 9+2t | 16+2t, 17+2t | 24+2t, 25+2t
+// are contiguous)
+MQ_HD int bf16_slot(int k) { return 8 * ((k & 7) >> 1) + 2 * (k >> 3) + (k & 1); }
 
 // slot of sub-block j (< 16) in the Q2_K / Q3_K scale fields
 MQ_HD int q16_slot(int j) { return 4 * ((j & 7) >> 1) + 2 * (j >> 3) + (j & 1); }
@@ -152,6 +165,18 @@ MQ_HD float dequant_at(int f, const uint8_t* base, const TensorLayout& L, int64_
     const int64_t b = c / qk;
     const int k = (int)(c % qk);
     const PlaneBytes pb = plane_bytes(f);
+    if (f == kBF16) {
+        const uint16_t h = load_le16(rec_ptr(base + L.plane[0], L, 64, r, b) + 2 * bf16_slot(k));
+        union { uint32_t u; float f; } c; c.u = (uint32_t)h << 16; return c.f;
+    }
+    if (f == kQ6K) {
+        const float d = half_bits_to_float(load_le16(rec_ptr(base + L.plane[0], L, 2, r, b)));
+        const int s = (int)rec_ptr(base + L.plane[1], L, 16, r, b)[q16_slot(k >> 4)] - 128;
+        const CodePos pl = pos4s(k), ph = pos2(k);
+        const int lo = (int)((rec_word(base + L.plane[2], L, 128, r, b, pl.word) >> pl.bit) & 15u);
+        const int hi = (int)((rec_word(base + L.plane[3], L, 64, r, b, ph.word) >> ph.bit) & 3u);
+        return (d * (float)s) * (float)((lo | (hi << 4)) - 32);
+    }
     const float d = half_bits_to_float(load_le16(rec_ptr(base + L.plane[0], L, 2, r, b)));
     if (f == kQ80) {
         const CodePos p = pos8(k);

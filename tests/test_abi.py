@@ -40,7 +40,7 @@ def test_library_exports_every_declared_symbol(mq):
         assert n in mq.EXPORTED, n
 
 
-@pytest.mark.parametrize("fmt", ["Q2_K", "Q3_K", "Q4_K", "Q8_0"])
+@pytest.mark.parametrize("fmt", ["Q2_K", "Q3_K", "Q4_K", "Q8_0", "Q6_K", "BF16"])
 @pytest.mark.parametrize("shape", [(1, 32), (3, 256), (5, 300), (16, 1024), (7, 2051)])
 def test_host_pack_unpack_match_oracle(mq, orc, fmt, shape):
     rng = np.random.default_rng(hash((fmt, shape)) % 2**32)
@@ -52,7 +52,7 @@ def test_host_pack_unpack_match_oracle(mq, orc, fmt, shape):
     assert mq.mq_packed_size(fmt, *shape) == orc.packed_size(fmt, *shape)
 
 
-@pytest.mark.parametrize("fmt", [1, 2, 3, 4])
+@pytest.mark.parametrize("fmt", [1, 2, 3, 4, 5, 6])
 def test_host_unpack_random_planes_match_oracle(mq, orc, fmt):
     from workloads.synth import random_packed, rng_for
     p = random_packed(fmt, 9, 768, rng_for(fmt))
@@ -66,6 +66,8 @@ def test_bad_format_and_sizes(mq):
         mq.mq_pack(9, np.zeros((1, 32), np.float32))
     with pytest.raises(mq.MoeqError):
         mq.mq_pack("Q8_0", np.full((1, 32), np.inf, np.float32))
+    with pytest.raises(mq.MoeqError):       # rounds past the largest bf16
+        mq.mq_pack("BF16", np.full((1, 32), np.finfo(np.float32).max, np.float32))
 
 
 @pytest.mark.parametrize("field,value,code", [
@@ -112,7 +114,7 @@ def test_strerror(mq):
     assert "workspace" in mq.mq_strerror(-5)
 
 
-@pytest.mark.parametrize("fmt", [1, 2, 3, 4])
+@pytest.mark.parametrize("fmt", [1, 2, 3, 4, 5, 6])
 def test_generator_sizes_match_library_and_oracle(mq, orc, fmt):
     # the input generators and bench.py's byte accounting size packed tensors
     # themselves; they must agree with both codecs

@@ -9,8 +9,8 @@ from __future__ import annotations
 import math
 from dataclasses import dataclass, field
 
-Q2_K, Q3_K, Q4_K, Q8_0 = 1, 2, 3, 4
-FMT_NAMES = {Q2_K: "Q2_K", Q3_K: "Q3_K", Q4_K: "Q4_K", Q8_0: "Q8_0"}
+Q2_K, Q3_K, Q4_K, Q8_0, Q6_K, BF16 = 1, 2, 3, 4, 5, 6
+FMT_NAMES = {Q2_K: "Q2_K", Q3_K: "Q3_K", Q4_K: "Q4_K", Q8_0: "Q8_0", Q6_K: "Q6_K", BF16: "BF16"}
 
 # bytes per block in each plane, and weights per block (format geometry used
 # only for byte accounting and for filling planes with random content)
@@ -19,6 +19,8 @@ PLANES = {
     Q2_K: (256, [("f16", 2), ("f16", 2), ("u8", 16), ("u8", 64)]),
     Q3_K: (256, [("f16", 2), ("u8", 12), ("u8", 64), ("u8", 32)]),
     Q8_0: (32, [("f16", 2), ("u8", 32)]),
+    Q6_K: (256, [("f16", 2), ("u8", 16), ("u8", 128), ("u8", 64)]),
+    BF16: (32, [("bf16", 64)]),
 }
 PLANE_ALIGN = 256
 

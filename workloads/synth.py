@@ -11,13 +11,14 @@ Recipe (stated here and in the design notes):
   bias        fp32 ~ N(0, bias_std)    (0.01 on V3 layers, 0 on the tiny layer)
   codes/fields uniform random bytes
   d, dmin     fp16 = base * U(0.5, 1.5), base per format (FP16_BASE)
+  bf16 tensor bf16 ~ N(0, 0.02)        (BF16 format: values, not fields)
   pruned set  sorted draw of n_experts of the original 256 ids
 """
 from __future__ import annotations
 
 import numpy as np
 
-from .configs import PLANES, PLANE_ALIGN, Q2_K, Q3_K, Q4_K, Q8_0, ROW_TILE, LayerSpec, packed_bytes
+from .configs import PLANES, PLANE_ALIGN, Q2_K, Q3_K, Q4_K, Q6_K, Q8_0, ROW_TILE, LayerSpec, packed_bytes
 
 # fp16 scale bases: decoded weights then have mean ~0 and std ~0.02
 FP16_BASE = {
@@ -25,7 +26,9 @@ FP16_BASE = {
     Q3_K: (4.7e-4,),
     Q4_K: (7.7e-5, 5.8e-4),
     Q8_0: (2.7e-4,),
+    Q6_K: (6.5e-5,),      # d straddles the smallest normal fp16 (6.1e-5): both kinds occur
 }
+BF16_STD = 0.02
 
 
 def rng_for(seed: int) -> np.random.Generator:
@@ -135,6 +138,9 @@ def random_packed(fmt: int, rows: int, cols: int, r: np.random.Generator) -> np.
             fi += 1
             v = (base * (0.5 + r.random(nblk, dtype=np.float32))).astype(np.float16)
             buf[off:off + n] = v.view(np.uint8)
+        elif kind == "bf16":
+            v = f32_to_bf16_bits(r.standard_normal(n // 2, dtype=np.float32) * np.float32(BF16_STD))
+            buf[off:off + n] = v.view(np.uint8)
         else:
             buf[off:off + n] = np.frombuffer(r.bytes(n), np.uint8)
     return buf
@@ -152,6 +158,9 @@ def random_packed_device(fmt: int, rows: int, cols: int, gen, device):
             base = FP16_BASE[fmt][fi]
             fi += 1
             v = (base * (0.5 + torch.rand(nblk, generator=gen, device=device))).to(torch.float16)
+            buf[off:off + n] = v.view(torch.uint8)
+        elif kind == "bf16":
+            v = (torch.randn(n // 2, generator=gen, device=device) * BF16_STD).to(torch.bfloat16)
             buf[off:off + n] = v.view(torch.uint8)
         else:
             buf[off:off + n] = torch.randint(0, 256, (n,), generator=gen, device=device,
