@@ -196,7 +196,7 @@ int moe_quant_forward(const mq_layer_cfg* cfg, int32_t n_tokens, const void* x,
  *   device that loads it until the process exits.  A call whose
  *   moe_quant_workspace_size(cfg, n_tokens) exceeds 16 MiB returns MQ_ERANGE
  *   and enqueues nothing (a V3-shaped layer, hidden 7168 / inter 2048 /
- *   top-8 + shared expert, fits up to 35 tokens).
+ *   top-8 + shared expert, fits up to 29 tokens).
  *   The first call on a device looks the array's device address up
  *   (cudaGetSymbolAddress, with that device current); make that first call
  *   before any stream capture.  It allocates nothing itself.

@@ -188,6 +188,7 @@ struct __align__(16) Hdr {
     int32_t ks, fmt, tensor, ntok;   // tensor: 0 gate, 1 up, 2 down rows rb, 3 down rows rb + 1
     int32_t rb, e, shared, slot;
     int32_t asg[kDecodeTok];
+    int32_t kb, half, pad0, pad1;      // first superblock of the item's K range; K half (-1: whole K)
 };
 
 // token pieces in a stage: the family fragments and the per-superblock
@@ -266,17 +267,21 @@ struct DecodeArgs {
     float* pdn;              // [A][H]
     uint32_t* next;          // item counter
     uint32_t* hready;        // [kMaxExperts + 1] per slot: published h blocks (tokens x 32-row blocks)
+    uint32_t* scount;        // [T][I / 32] halves of a shared gate/up block finished (K split)
+    float* spart;            // [T][2 halves][2 (gate, up)][I] the halves' sums
     const uint32_t* logits_done;   // logits CTAs done (their prepared tokens are written)
     const uint32_t* route_ready;   // non-zero once the routing result is written
     uint32_t n_logit_ctas;
     uint32_t* err;
     uint64_t wait_ns;        // limit of every bounded wait
     int fail_first_stage;    // test hook: the producer posts nothing for its first stage
+    int split_shared;        // the shared expert's gate/up blocks are split in two K halves
     Geo geo[2][kNumFormats][kDecodeTok];   // [down][format][tokens], computed on the host
 };
 
 struct ItemDesc {            // decoded item (producer side)
     int e, rb, tg, ntok, shared, nst0, nst, down, slot;
+    int kb, ke, half;        // superblock range [kb, ke) of K; half of a split item (-1: whole K)
     int vec[kDecodeTok], asg[kDecodeTok];
 };
 
@@ -293,10 +298,22 @@ __device__ __forceinline__ void decode_item(const DecodeArgs& A, const SlotCache
     const int p = cursor;
     it.slot = p;
     it.down = down ? 1 : 0;
-    const int local = lid - pre[p];
+    int local = lid - pre[p];
     const Dims& d = A.d;
-    // gate/up items: one 32-row block of gate and up; down items: two 32-row blocks
+    // gate/up items: one 32-row block of gate and up; down items: two 32-row blocks.
+    // The shared expert's gate/up blocks are split in two K halves (two items,
+    // the halves of a block claimed one after the other), so that every CTA has
+    // shared-expert work while the routing result is computed.
     const int nrb = down ? d.H / 64 : d.I / 32;
+    const int nsb = down ? A.nsbi : A.nsbx;
+    it.half = -1; it.kb = 0; it.ke = nsb;
+    if (!down && p < d.has_shared && A.split_shared) {
+        it.half = local & 1;
+        local >>= 1;
+        const int mid = nsb / 2;
+        it.kb = it.half ? mid : 0;
+        it.ke = it.half ? nsb : mid;
+    }
     it.tg = local / nrb;
     it.rb = (local - it.tg * nrb) * (down ? 2 : 1);
     it.e = sc.e[p];
@@ -790,7 +807,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     // the wait for the routing kernel.  (The tokens' prepared activations come
     // from the logits kernel, which completed before the routing kernel let
     // this grid launch.)
-    const int n_sh_items = d.has_shared ? (d.I / 32) * ((d.T + kDecodeTok - 1) / kDecodeTok) : 0;
+    const int n_sh_blocks = d.has_shared ? (d.I / 32) * ((d.T + kDecodeTok - 1) / kDecodeTok) : 0;
+    const int n_sh_items = A.split_shared ? 2 * n_sh_blocks : n_sh_blocks;
     if (threadIdx.x == 0 && n_sh_items > 0) {
         sc.pre_gu[0] = 0; sc.pre_gu[1] = n_sh_items;
         sc.e[0] = d.E; sc.first[0] = 0; sc.ntot[0] = d.T;
@@ -866,7 +884,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                         ntot = __ldcg(&A.plan->slot_ntot[i]);
                     }
                 }
-                sc.pre_gu[i] = pg;
+                // the plan counts one gate/up item per shared block; with the K
+                // split the shared slot has two
+                sc.pre_gu[i] = pg + (i >= 1 && A.split_shared ? n_sh_blocks : 0);
                 sc.pre_dn[i] = pd;
                 if (i < n_slots) {
                     sc.e[i] = e;
@@ -912,14 +932,20 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             const int id = id_next;
             if (!routed && id >= n_sh_items) wait_routing();
             const int item = id < n_items ? id : -1;
-            // claim the following item now; the atomic's latency hides behind this item's stages
-            if (item >= 0) id_next = claim();
+            // claim the following item now, so that the atomic's latency hides
+            // behind this item's stages; before the routing result is in, only
+            // after this item's stages are posted, so that the shared expert's
+            // items spread over the CTAs instead of going two to a CTA
+            const bool claim_early = routed || !A.split_shared;
+            if (item >= 0 && claim_early) id_next = claim();
             if (item >= 0) {
                 decode_item(A, sc, s_perm, n_slots, n_gu, item, cur_gu, cur_dn, P);
                 fmt0 = tab.fmt[P.e][P.down ? 2 : 0];
                 fmt1 = tab.fmt[P.e][P.down ? 2 : 1];
-                P.nst0 = geo[P.down][fmt0 - 1][P.ntok - 1].nst;
-                P.nst = P.down ? 2 * P.nst0 : P.nst0 + geo[0][fmt1 - 1][P.ntok - 1].nst;
+                const int span = P.ke - P.kb;
+                const int per0 = geo[P.down][fmt0 - 1][P.ntok - 1].per, per1 = geo[0][fmt1 - 1][P.ntok - 1].per;
+                P.nst0 = (span + per0 - 1) / per0;
+                P.nst = P.down ? 2 * P.nst0 : P.nst0 + (span + per1 - 1) / per1;
             }
             const int nst = item >= 0 ? P.nst : 1;
             bool failed = false;
@@ -993,7 +1019,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     }
                 }
                 const int per = G->per;
-                const int s0 = (pj - phase_j) * per, ks = min(per, (P.down ? A.nsbi : A.nsbx) - s0);
+                const int s0 = P.kb + (pj - phase_j) * per, ks = min(per, P.ke - s0);
                 const uint32_t stage = ring + slot * kSlotBytes;
                 const uint32_t bytes = c_src ? (uint32_t)ks * c_stride : 0u;
                 uint32_t total = bytes;
@@ -1005,6 +1031,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     H[1] = make_int4(ks, fmt, tensor, P.ntok);
                     H[2] = make_int4(P.rb, P.e, P.shared, P.slot);
                     H[3] = make_int4(P.asg[0], P.asg[1], P.asg[2], P.asg[3]);
+                    H[4] = make_int4(P.kb, P.half, 0, 0);
                     s_posted[slot] = p_q;
                     mbar_arrive_tx(full, total);
                 }
@@ -1042,6 +1069,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             if (failed) { if (lane == 0) { atomicOr(A.err, kErrEmpty); s_fail = 1; } break; }
             if (item < 0) break;
+            if (!claim_early) id_next = claim();
         }
     } else {
         // ============================ consumer warps =============================
@@ -1074,7 +1102,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             // multiple of kCols
             const int s_item = H.s0 + ((H.tensor & 1) ? (dn ? A.nsbi : A.nsbx) : 0);
             const int wcol = (col - s_item % kCols + kCols) % kCols;
-            if ((H.tensor & 1) && H.s0 == 0) {
+            if ((H.tensor & 1) && H.s0 == H.kb) {
                 // first stage of the second phase: the first phase's sums are complete
 #pragma unroll
                 for (int tk = 0; tk < MT; ++tk)
@@ -1106,10 +1134,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             // fields needed after the slot is released to the producer
             const bool item_end = H.j == H.nst - 1;
-            int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0, e_slot = 0;
+            int e_rb = 0, e_ntok = 0, e_shared = 0, e_e = 0, e_slot = 0, e_half = -1;
             int e_asg[kDecodeTok];
             if (item_end) {
-                e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e; e_slot = H.slot;
+                e_rb = H.rb; e_ntok = H.ntok; e_shared = H.shared; e_e = H.e; e_slot = H.slot; e_half = H.half;
 #pragma unroll
                 for (int tk = 0; tk < kDecodeTok; ++tk) e_asg[tk] = H.asg[tk];
             }
@@ -1153,7 +1181,30 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     v0 += red[buf][c2][0][tk][lane];
                     v1 += red[buf][c2][1][tk][lane];
                 }
-                if (dn) {
+                bool finish = true;
+                if (!dn && e_half >= 0) {
+                    // K half of a shared-expert block: publish this half's sums; the
+                    // half that counts second adds the other's (a + b, the same bits
+                    // in either order) and finishes the block
+                    const int t = a - d.T * d.K;   // the token (shared-expert assignment)
+                    float* sp = A.spart + (size_t)t * 4 * d.I;
+                    sp[(2 * e_half + 0) * d.I + 32 * e_rb + lane] = v0;
+                    sp[(2 * e_half + 1) * d.I + 32 * e_rb + lane] = v1;
+                    __threadfence();
+                    __syncwarp();
+                    uint32_t before = 0;
+                    if (lane == 0) before = atomicAdd(A.scount + (size_t)t * (d.I / 32) + e_rb, 1u);
+                    before = __shfl_sync(kFull, before, 0);
+                    finish = before == 1u;
+                    if (finish) {
+                        __threadfence();
+                        const int o = 1 - e_half;
+                        v0 += __ldcg(sp + (2 * o + 0) * d.I + 32 * e_rb + lane);
+                        v1 += __ldcg(sp + (2 * o + 1) * d.I + 32 * e_rb + lane);
+                    }
+                }
+                if (!finish) {
+                } else if (dn) {
                     A.pdn[(size_t)a * d.H + 32 * e_rb + lane] = v0;
                     A.pdn[(size_t)a * d.H + 32 * (e_rb + 1) + lane] = v1;
                 } else {
@@ -1215,8 +1266,9 @@ void combine_setup() { prefer_max_shared(combine_kernel); }
 }  // namespace
 
 size_t decode_counter_bytes(const Dims& d) {
-    (void)d;
-    return 4 + 4 * (kMaxExperts + 1);   // the item counter, then one h counter per expert slot
+    // the item counter, one h counter per expert slot, then one half-count per
+    // (token, 32-row block) of the shared expert's K-split gate/up blocks
+    return 4 + 4 * (kMaxExperts + 1) + 4 * (size_t)d.T * (d.I / 32);
 }
 
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
@@ -1234,6 +1286,9 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.pdn = w.pdn;
     A.next = w.counters;
     A.hready = w.counters + 1;
+    A.scount = w.counters + 1 + (kMaxExperts + 1);
+    A.spart = w.spart;
+    A.split_shared = d.T == 1 && d.has_shared && A.nsbx >= 2 ? 1 : 0;   // one token: the routing front
     A.logits_done = w.logits_done;
     A.route_ready = w.route_ready;
     A.n_logit_ctas = (uint32_t)(d.E * ((d.T + 7) / 8));   // the logits kernel's grid (experts x 8-token groups)

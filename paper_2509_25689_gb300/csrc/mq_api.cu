@@ -92,6 +92,7 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
     const size_t o_pdn = take(A * d.H * 4);
     const size_t o_plan = take(sizeof(Plan));
     const size_t o_xe = take((size_t)d.T * 4);
+    const size_t o_spart = take((size_t)d.T * 4 * d.I * 4);   // shared gate/up K halves (decode)
     const size_t cnt_bytes = decode_counter_bytes(d);
     // work counters, the two routing words, then the error word (zeroed per call)
     const size_t o_cnt = take(cnt_bytes + 12);
@@ -118,6 +119,7 @@ size_t workspace_plan(const Dims& d, void* base, Work* w) {
         w->route_ready = reinterpret_cast<uint32_t*>(b + o_sync + 4);
         w->err = reinterpret_cast<uint32_t*>(b + o_err);
         w->xe = reinterpret_cast<int32_t*>(b + o_xe);
+        w->spart = reinterpret_cast<float*>(b + o_spart);
         w->x16 = w->xq;   // the prefill path uses these bytes instead of the decode preparation
         w->h16 = w->hq;
         w->zero_words = w->counters;

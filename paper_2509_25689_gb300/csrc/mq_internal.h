@@ -68,6 +68,7 @@ struct Work {
                        // each token scaled by 2^-xe[t]
     int32_t* xe;       // [T] per-token power-of-two exponents of x16 (prefill path)
     __half* h16;       // [A][I] fp16 SwiGLU outputs for the prefill GEMM (shares hq's bytes)
+    float* spart;         // decode: the shared expert's gate/up K halves [T][2][2][I]
     uint32_t* zero_words; // counters + error word, cleared by the first kernel of a call
     int n_zero;
 };
