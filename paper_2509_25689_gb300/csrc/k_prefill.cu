@@ -150,8 +150,11 @@ __device__ __forceinline__ RowPtrs row_ptrs(int fmt, const uint8_t* base, const 
     return P;
 }
 
+// kRare: the launch's layer has Q6_K or BF16 tensors (their code paths exist
+// only in that instantiation, so the common one keeps its registers)
+template <bool kRare>
 __device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, int hf, Packed& P) {
-    if (fmt == kBF16) {
+    if (kRare && fmt == kBF16) {
         // block 2c + hf: only the address of its 64-byte record is carried (the
         // decode step loads it), which keeps the prefetched fields of the other
         // formats in registers
@@ -181,7 +184,7 @@ __device__ __forceinline__ void load_chunk(int fmt, const RowPtrs& RP, int c, in
         P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
         return;
     }
-    if (fmt == kQ6K) {
+    if (kRare && fmt == kQ6K) {
         const uint4 sv = ldg128(RP.row[1] + s * (32 * 16));
         P.sc[0] = sv.x; P.sc[1] = sv.y; P.sc[2] = sv.z; P.sc[3] = sv.w;
         // low nibbles: sub-block j = 4 cc + i in unit cc / 2, words 4 i + 2 (cc % 2) + 0..1
@@ -282,9 +285,15 @@ __device__ __forceinline__ uint32_t byte_of(const uint32_t (&w)[4], int i) {
 
 // Q6_K and BF16 chunks, kept out of line: the formats of most units keep
 // their registers (an out-of-line call saves only what is live around it).
-__device__ __noinline__ bool dequant_store_rare(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
+// The fields come as scalars (a reference would make every caller keep its
+// packed fields in local memory).
+__device__ __noinline__ bool dequant_store_rare(int fmt, uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
+                                                uint32_t w4, uint32_t w5, uint32_t sc0, uint32_t sc1, uint32_t sc2,
+                                                uint32_t sc3, uint32_t dd, int c, int hf, uint32_t dst) {
+    const uint32_t Pw[6] = {w0, w1, w2, w3, w4, w5};
+    const uint32_t Psc[4] = {sc0, sc1, sc2, sc3};
     if (fmt == kBF16) {
-        const uint8_t* bp = reinterpret_cast<const uint8_t*>((uintptr_t)P.w[0] | ((uintptr_t)P.w[1] << 32));
+        const uint8_t* bp = reinterpret_cast<const uint8_t*>((uintptr_t)w0 | ((uintptr_t)w1 << 32));
         uint32_t wd[16];   // the record: pair p of the block in word 4 (p % 4) + p / 4
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
@@ -308,12 +317,12 @@ __device__ __noinline__ bool dequant_store_rare(int fmt, const Packed& P, int c,
     }
     if (fmt == kQ6K) {
         const int cc = c & 3;
-        const float d = half_lo(P.dd);
+        const float d = half_lo(dd);
         const __half2 k1056 = __float2half2_rn(1056.0f);   // 1024 + the code offset 32
 #pragma unroll
         for (int ii = 0; ii < 2; ++ii) {
             const int i = 2 * hf + ii, j = 4 * cc + i;
-            const int sv = (int)byte_of(P.sc, q16_slot(j)) - 128;
+            const int sv = (int)byte_of(Psc, q16_slot(j)) - 128;
             const __half2 a2 = __float2half2_rn(d * (float)sv);
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
@@ -321,8 +330,8 @@ __device__ __noinline__ bool dequant_store_rare(int fmt, const Packed& P, int c,
 #pragma unroll
                 for (int mm = 0; mm < 4; ++mm) {
                     const int m = 4 * q + mm;
-                    const uint32_t nib = (P.w[2 * ii + (m >> 2)] >> (4 * (m & 3))) & 0x000F000Fu;
-                    const uint32_t hi2 = (P.w[4 + ii] >> (2 * m)) & 0x00030003u;
+                    const uint32_t nib = (Pw[2 * ii + (m >> 2)] >> (4 * (m & 3))) & 0x000F000Fu;
+                    const uint32_t hi2 = (Pw[4 + ii] >> (2 * m)) & 0x00030003u;
                     o[mm] = h2u(__hmul2(a2, __hsub2(u2h(nib | (hi2 << 4) | 0x64006400u), k1056)));
                 }
                 sts128(dst + ((2 * i + q) * kMT) * 16, o[0], o[1], o[2], o[3]);
@@ -339,9 +348,12 @@ __device__ __noinline__ bool dequant_store_rare(int fmt, const Packed& P, int c,
 // dmin*m are rounded to fp16 once.  BF16 weights convert exactly where
 // 2^-14 <= |w| < 65520 (below, to the nearest fp16 subnormal); the return
 // value is true if one of them is beyond the fp16 range.
+template <bool kRare>
 __device__ __forceinline__ bool dequant_store(int fmt, const Packed& P, int c, int hf, uint32_t dst) {
     const __half2 k1024 = __float2half2_rn(1024.0f);
-    if (fmt == kBF16 || fmt == kQ6K) return dequant_store_rare(fmt, P, c, hf, dst);
+    if (kRare && (fmt == kBF16 || fmt == kQ6K))
+        return dequant_store_rare(fmt, P.w[0], P.w[1], P.w[2], P.w[3], P.w[4], P.w[5], P.sc[0], P.sc[1], P.sc[2],
+                                  P.sc[3], P.dd, c, hf, dst);
     if (fmt == kQ80) {
         const __half2 k1152 = __float2half2_rn(1152.0f);
         {
@@ -429,7 +441,7 @@ __device__ __forceinline__ bool dequant_store(int fmt, const Packed& P, int c, i
 
 __device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
 
-template <bool kDown>
+template <bool kDown, bool kRare>
 __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(const __grid_constant__ ExpertTab tab,
                                                                             const __grid_constant__ PrefillArgs A) {
     constexpr bool kWS = mma_warp(kDown);
@@ -628,8 +640,8 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
             const uint32_t sbase = ring + s * kSlotBytes;
-            if (dequant_store(f0, Q0, c, hf, sbase + rr * 16)) w_over = true;
-            if (!kDown && dequant_store(f1, Q1, c, hf, sbase + kABytes + rr * 16)) w_over = true;
+            if (dequant_store<kRare>(f0, Q0, c, hf, sbase + rr * 16)) w_over = true;
+            if (!kDown && dequant_store<kRare>(f1, Q1, c, hf, sbase + kABytes + rr * 16)) w_over = true;
             asm volatile("cp.async.wait_group 1;" ::: "memory");
             // this thread's shared-memory writes (and landed copies) before the
             // tensor cores read them
@@ -680,8 +692,8 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
         } else {
             // Q8_0, Q6_K or BF16 in the unit: per-chunk fields, one chunk ahead
             Packed P0, P1;                 // this chunk's packed fields, gate (or down) and up
-            load_chunk(f0, RP0, 0, hf, P0);
-            if (!kDown) load_chunk(f1, RP1, 0, hf, P1);
+            load_chunk<kRare>(f0, RP0, 0, hf, P0);
+            if (!kDown) load_chunk<kRare>(f1, RP1, 0, hf, P1);
             for (int c = 0; c < nC; ++c) {
                 // pull the records of this warp's 32-row tile for the next superblock
                 // into L2, so the per-thread loads of the coming chunks hit L2
@@ -690,8 +702,8 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
                                  ::"l"(pf_src + (int64_t)((c >> 2) + 1) * pf_bytes), "r"(pf_bytes) : "memory");
                 Packed N0, N1;             // the next chunk's, loaded while this one is decoded
                 if (c + 1 < nC) {
-                    load_chunk(f0, RP0, c + 1, hf, N0);
-                    if (!kDown) load_chunk(f1, RP1, c + 1, hf, N1);
+                    load_chunk<kRare>(f0, RP0, c + 1, hf, N0);
+                    if (!kDown) load_chunk<kRare>(f1, RP1, c + 1, hf, N1);
                 }
                 if (!chunk_body(c, P0, P1)) { failed = true; break; }
                 P0 = N0;
@@ -771,8 +783,10 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
 
 void prefill_setup() {
     const int smem = kPSlots * kSlotBytes;
-    cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(prefill_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(prefill_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(prefill_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(prefill_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
 
 }  // namespace
@@ -787,12 +801,19 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     A.offsets = w.offsets; A.perm = w.perm; A.active = w.active; A.wts = w.wts;
     A.x16 = w.x16; A.xe = w.xe; A.h16 = w.h16; A.pdn = w.pdn; A.err = w.err;
     A.next = w.counters;
+    bool rare = false;   // a Q6_K or BF16 tensor anywhere in the layer
+    for (int e = 0; e < d.E + d.has_shared; ++e)
+        for (int j = 0; j < 3; ++j) rare |= tab.fmt[e][j] == kQ6K || tab.fmt[e][j] == kBF16;
     prof_begin("gateup_tc", s);
-    cudaError_t err = launch_pdl(prefill_kernel<false>, dim3(g_psms), dim3(prefill_threads(false)), smem, s, tab, A);
+    cudaError_t err = rare ? launch_pdl(prefill_kernel<false, true>, dim3(g_psms), dim3(prefill_threads(false)), smem,
+                                        s, tab, A)
+                           : launch_pdl(prefill_kernel<false, false>, dim3(g_psms), dim3(prefill_threads(false)), smem,
+                                        s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     prof_begin("down_tc", s);
-    err = launch_pdl(prefill_kernel<true>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A);
+    err = rare ? launch_pdl(prefill_kernel<true, true>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A)
+               : launch_pdl(prefill_kernel<true, false>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);
