@@ -145,6 +145,27 @@ def test_forward_largest_routing_shapes(torch_cuda, orc, T, decode_kernel):
     assert_close(y, ry)
 
 
+@pytest.mark.parametrize("hidden", [256, 768, 1280])
+def test_forward_one_token_shared_k_halves(torch_cuda, orc, hidden):
+    """One token: the shared expert's gate/up blocks are split in two K halves
+    (K = hidden) whose sums the second-finishing half adds.  1, 3 and 5
+    superblocks: no split, then unequal halves."""
+    mq = mq_lib()
+    spec = LayerSpec(name="k_halves", hidden=hidden, inter=256, n_experts=12, n_groups=4, topk_group=2, top_k=3,
+                     tokens=1, has_shared=True, mixed=True, router_std=1 / hidden ** 0.5, bias_std=0.01)
+    fm = np.array([[1, 2, 3], [2, 3, 4], [3, 4, 1], [4, 1, 2]] * 3 + [[4, 4, 4]], np.uint8)
+    layer = DeviceLayer(spec, hidden, fmts=fm)
+    x = tokens(spec, hidden)
+    mq.mq_set_path(1)
+    try:
+        y, idx, w = layer.forward(x)
+    finally:
+        mq.mq_set_path(0)
+    ry, ridx, rw = layer.oracle_forward(orc, x)
+    np.testing.assert_array_equal(idx, ridx)
+    assert_close(y, ry)
+
+
 @pytest.mark.parametrize("T", [1, 3])
 def test_forward_sizes_not_multiple_of_256(torch_cuda, orc, T, decode_kernel):
     """Hidden 384 and inter 128 (multiples of 128 only) with every format,
