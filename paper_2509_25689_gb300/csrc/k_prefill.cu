@@ -58,6 +58,7 @@ struct PrefillArgs {
     const int32_t* xe;       // [T] the tokens' exponents
     __half* h16;             // [A][I] SwiGLU outputs (routing weight folded in), scaled by 2^-2 xe[t]
     float* pdn;              // [A][H]
+    uint8_t* xp;             // warp-specialised GEMM: the tokens in slot-position order, tiled (shares pdn's bytes)
     uint32_t* next;          // unit counters (gate/up, down), zeroed per call
     uint32_t* err;
 };
@@ -81,10 +82,12 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    if (mbar_try(bar, parity)) return true;
+    for (int i = 0; i < 32; ++i)
+        if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (;;) {
-        if (mbar_try(bar, parity)) return true;
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try(bar, parity)) return true;
         if (global_ns() - t0 > 1000000000ull) return false;
     }
 }
@@ -781,12 +784,698 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
     }
 }
 
+// ---------------------------------------------------------------------------
+// Warp-specialised form of the same GEMM, for layers whose tensors are all
+// Q2_K, Q3_K, Q4_K or Q8_0.  Each CTA runs four roles at once, so that the
+// record loads, the weight decode, the activation gather and the MMAs of
+// different chunks overlap instead of following one another:
+//   - a producer warp claims the units, publishes each one (slot, rows,
+//     tokens) in a two-deep unit ring and streams the unit's packed records
+//     into a two-stage ring with bulk copies (one per tensor, plane and
+//     32-row tile; a stage holds one superblock, or 128 contraction columns
+//     when a tensor is Q8_0, whose K-quant partner then comes twice);
+//   - sixteen worker warps decode the records from shared memory into the
+//     fp16 operand of each 64-wide chunk (the values dequant_store gives;
+//     gate/up: eight warps per tensor, down: eight per chunk parity) and, at
+//     the unit's end, run the epilogue out of tensor memory; the gate/up
+//     epilogue writes h straight into the down GEMM's activation layout;
+//   - an activation warp moves the chunk's activation rows with eight bulk
+//     copies from the tile-ordered copy of the tokens (xperm_kernel) or of h;
+//   - an MMA warp issues a chunk's MMAs once the workers and the activation
+//     warp have filled its operand slot (a two-slot ring) and commits them
+//     to the slot's empty barrier.
+// Every wait is bounded and reports to the error word.
+// 16 worker warps (gate/up: 8 per tensor; down: 8 per chunk parity), then
+// the producer, activation and MMA warps
+__host__ __device__ constexpr int g_workers(bool down) { return 16; }
+__host__ __device__ constexpr int g_threads(bool down) { return (g_workers(down) + 3) * 32; }
+constexpr int kGNT = 256;                      // tokens per unit (MMA N up to 256)
+constexpr int kGSlotBytes = 2 * kABytes + kGNT * kKC * 2;   // operand slot: A gate | A up | B, 64 KB
+constexpr int kGOps = 2;                       // operand slots (a third one fits only with 128-token
+                                               // units, measured slower on the Zipf prefill)
+constexpr int kGPk = 2;                        // packed-record stages
+constexpr int kGPkBytes = 36 * 1024;           // Q4_K + Q4_K superblock of 128 rows: 2 x 18,432
+constexpr int kGSmem = kGOps * kGSlotBytes + kGPk * kGPkBytes;
+
+// Activation rows of the warp-specialised GEMM in the order its units read
+// them: slot positions r (the permutation's order for the routed experts,
+// T*K + t for the shared expert), cut into tiles of up to kGNT rows of one
+// slot.  In a tile of N rows starting at position r0, the 16-byte piece p
+// (columns 8p .. 8p+7) of row n sits (p * N + n) * 16 bytes after r0 * K * 2,
+// so a 64-column chunk of a tile is eight contiguous runs of N x 16 bytes:
+// one bulk copy each into the canonical operand layout.
+__device__ __forceinline__ size_t perm_piece(int r0, int K, int N, int p, int n) {
+    return (size_t)r0 * K * 2 + ((size_t)p * N + n) * 16;
+}
+
+// The tokens (fp16, as the logits kernel scaled them) in that layout.
+__global__ void __launch_bounds__(256) xperm_kernel(const __half* __restrict__ x16,
+                                                    const int32_t* __restrict__ offsets,
+                                                    const int32_t* __restrict__ perm, const Dims d,
+                                                    uint8_t* __restrict__ xp) {
+    pdl_wait();
+    __shared__ int32_t s_off[kMaxExperts + 1];
+    const int E = d.E, TK = d.T * d.K, A = TK + (d.has_shared ? d.T : 0);
+    for (int i = threadIdx.x; i <= E; i += blockDim.x) s_off[i] = offsets[i];
+    __syncthreads();
+    const int lane = threadIdx.x & 31, np = d.H / 8;
+    for (int r = blockIdx.x * 8 + (threadIdx.x >> 5); r < A; r += gridDim.x * 8) {
+        int pos0, ntot, t;
+        if (r < TK) {
+            // the expert of position r: the last e with offsets[e] <= r
+            int lo = 0, hi = E - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (s_off[mid] <= r) lo = mid; else hi = mid - 1;
+            }
+            pos0 = s_off[lo]; ntot = s_off[lo + 1] - pos0; t = perm[r] / d.K;
+        } else {
+            pos0 = TK; ntot = d.T; t = r - TK;
+        }
+        const int q = r - pos0, tt = q / kGNT, n = q - tt * kGNT, N = min(kGNT, ntot - tt * kGNT);
+        const int r0 = pos0 + tt * kGNT;
+        const uint4* src = reinterpret_cast<const uint4*>(x16 + (size_t)t * d.H);
+        for (int p = lane; p < np; p += 32)
+            *reinterpret_cast<uint4*>(xp + perm_piece(r0, d.H, N, p, n)) = __ldg(src + p);
+    }
+    pdl_launch();
+}
+
+// per-CTA slot table of the warp-specialised GEMM (the pointers come from
+// the expert table by the slot's expert id)
+struct GSlots {
+    int32_t first[kMaxExperts + 1], ntot[kMaxExperts + 1], pre[kMaxExperts + 2], e[kMaxExperts + 1];
+    uint8_t fmt[kMaxExperts + 1][2];
+};
+
+struct GUnit {
+    int u;               // unit id, -1 once there are none left
+    int p, mt, N, Npad;
+    int r0;              // the tile's first slot position
+    int ks;              // contraction columns per packed stage: 256, or 128 when a tensor is Q8_0
+};
+
+// where each plane of each tensor sits in a packed stage (tile 0; tile t at + t * tile)
+struct GStage {
+    int off[2][4], tile[2][4], ub[2][4];
+    int total;
+};
+__device__ __forceinline__ GStage gstage(int f0, int f1, int ntens, int ks) {
+    GStage G;
+    int at = 0;
+#pragma unroll
+    for (int z = 0; z < 2; ++z) {
+        const int f = z == 0 ? f0 : f1;
+        const PlaneBytes pb = plane_bytes(f);
+        const int nb = f == kQ80 ? ks / 32 : 1;
+#pragma unroll
+        for (int pl = 0; pl < 4; ++pl) {
+            const bool on = z < ntens && pl < pb.n;
+            G.off[z][pl] = at;
+            G.tile[z][pl] = on ? nb * 32 * pb.b[pl] : 0;
+            G.ub[z][pl] = on ? unit_bytes(pb.b[pl]) : 0;
+            at += 4 * G.tile[z][pl];
+        }
+    }
+    G.total = at;
+    return G;
+}
+
+__device__ __forceinline__ void g_mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void g_arrive_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void g_bulk(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar, uint64_t pol) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(pol) : "memory");
+}
+__device__ __forceinline__ uint4 g_lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint2 g_lds64(uint32_t a) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint32_t g_lds32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint32_t g_lds16(uint32_t a) {
+    unsigned short v;
+    asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
+    return v;
+}
+
+// One superblock's fields of this thread's row (records at rec[pl] in the
+// stage), as load_sblk reads them from global memory.
+__device__ __forceinline__ void load_sblk_s(int fmt, const uint32_t (&rec)[4], int hf, SBlk& B) {
+    B.dd = g_lds16(rec[0]);
+    if (fmt == kQ4K) {
+        B.dd |= g_lds16(rec[1]) << 16;
+        B.sc[0] = g_lds32(rec[2]); B.sc[1] = g_lds32(rec[2] + 4); B.sc[2] = g_lds32(rec[2] + 8);
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            const int j = 2 * cc + hf;
+            B.cw[cc] = g_lds128(rec[3] + (j >> 2) * (kRowTile * 64) + 16 * (j & 3));
+        }
+    } else if (fmt == kQ2K) {
+        B.dd |= g_lds16(rec[1]) << 16;
+        const uint4 sv = g_lds128(rec[2]);
+        B.sc[0] = sv.x; B.sc[1] = sv.y; B.sc[2] = sv.z; B.sc[3] = sv.w;
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) B.cw[ii] = g_lds128(rec[3] + 16 * (2 * hf + ii));
+    } else {   // Q3_K
+        B.sc[0] = g_lds32(rec[1]); B.sc[1] = g_lds32(rec[1] + 4); B.sc[2] = g_lds32(rec[1] + 8);
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            B.cw[ii] = g_lds128(rec[2] + 16 * (2 * hf + ii));
+            B.hw[ii] = g_lds64(rec[3] + 8 * (2 * hf + ii));
+        }
+    }
+}
+// make_packed for a chunk index known only at run time (selects instead of
+// an indexed register array, which would live in local memory)
+__device__ __forceinline__ uint4 pick4(const uint4 (&v)[4], int i) {
+    const uint4 a = (i & 1) ? v[1] : v[0], b = (i & 1) ? v[3] : v[2];
+    return (i & 2) ? b : a;
+}
+__device__ __forceinline__ void make_packed_rt(int fmt, const SBlk& B, int cc, Packed& P) {
+    P.dd = B.dd;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) P.sc[i] = B.sc[i];
+    if (fmt == kQ4K) {
+        const uint4 w = pick4(B.cw, cc);
+        P.w[0] = w.x; P.w[1] = w.y; P.w[2] = w.z; P.w[3] = w.w;
+    } else {
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+            const uint4 w = B.cw[ii];
+            const uint32_t lo = (cc & 1) ? w.y : w.x, hi = (cc & 1) ? w.w : w.z;
+            P.w[ii] = (cc & 2) ? hi : lo;
+            P.w[4 + ii] = (cc >> 1) ? B.hw[ii].y : B.hw[ii].x;
+        }
+    }
+}
+// Q8_0 block lb of the stage for this thread's row, as load_chunk reads it
+__device__ __forceinline__ void load_q80_s(const uint32_t (&rec)[4], int lb, Packed& P) {
+    const uint32_t cp = rec[1] + lb * (32 * 32);
+    const uint4 w0 = g_lds128(cp), w1 = g_lds128(cp + 16);
+    P.w[0] = w0.x; P.w[1] = w0.y; P.w[2] = w0.z; P.w[3] = w0.w;
+    P.w[4] = w1.x; P.w[5] = w1.y; P.w[6] = w1.z; P.w[7] = w1.w;
+    P.dd = g_lds16(rec[0] + lb * (32 * 2));
+}
+
+// ---- chunk decode for the warp-specialised GEMM: the values dequant_store
+// produces (the same fp16 roundings: d * sc and dmin * m are exact products
+// rounded once, then one fused multiply-add per weight pair), with fewer
+// instructions: a code field at bit s <= 8 of each 16-bit half, OR-ed into
+// the fp16 pair 2^(10 - s), reads as 2^(10 - s) + code exactly (the field
+// lands in the mantissa at unit weight), so one AND-OR and one subtraction
+// give the code without a shift; the scale fields of two sub-blocks are
+// widened as one fp16 pair.  Stores are plain shared-memory stores the
+// compiler may schedule (the proxy fence after them orders them for the
+// tensor cores).
+__device__ __forceinline__ constexpr uint32_t magic_bits(int s) {
+    return ((uint32_t)(25 - s) << 10) | ((uint32_t)(25 - s) << 26);
+}
+__device__ __forceinline__ __half2 magic_val(int s) { return u2h(magic_bits(s)); }
+__device__ __forceinline__ uint32_t pick_word(const uint32_t (&w)[4], int i) {
+    const uint32_t a = (i & 1) ? w[1] : w[0], b = (i & 1) ? w[3] : w[2];
+    return (i & 2) ? b : a;
+}
+__device__ __forceinline__ void st_row(uint4* dst, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    *dst = make_uint4(a, b, c, d);
+}
+
+// Q2_K: sub-blocks 2 hf, 2 hf + 1 of chunk cc (16 weights each)
+__device__ __forceinline__ void dq_q2k(const SBlk& B, int cc, int hf, uint4* dst) {
+    const uint32_t dd = B.dd;
+    const __half2 d2 = u2h((dd & 0xFFFFu) * 0x00010001u);
+    const __half2 nm2 = u2h(((dd >> 16) * 0x00010001u) ^ 0x80008000u);   // -dmin
+    const int s0 = q16_slot(4 * cc + 2 * hf);   // the two sub-blocks' slots: s0, s0 + 1 (s0 even)
+    const uint32_t x = __byte_perm(pick_word(B.sc, s0 >> 2), 0u, (s0 & 2) ? 0x4342u : 0x4140u);
+    const __half2 k1024 = magic_val(0);
+    const __half2 scp = __hsub2(u2h((x & 0x000F000Fu) | 0x64006400u), k1024);
+    const __half2 mp = __hsub2(u2h(((x >> 4) & 0x000F000Fu) | 0x64006400u), k1024);
+    const __half2 ap = __hmul2(d2, scp), np = __hmul2(nm2, mp);
+#pragma unroll
+    for (int ii = 0; ii < 2; ++ii) {
+        const int i = 2 * hf + ii;
+        const __half2 a2 = ii ? __high2half2(ap) : __low2half2(ap);
+        const __half2 n2 = ii ? __high2half2(np) : __low2half2(np);
+        const uint4 cw = B.cw[ii];
+        const uint32_t lo = (cc & 1) ? cw.y : cw.x, hi = (cc & 1) ? cw.w : cw.z;
+        const uint32_t w = (cc & 2) ? hi : lo, wh = w >> 10;
+        uint32_t o[8];
+        o[0] = h2u(__hfma2(a2, __hsub2(u2h((w & 0x00030003u) | magic_bits(0)), magic_val(0)), n2));
+        o[1] = h2u(__hfma2(a2, __hsub2(u2h((w & 0x000C000Cu) | magic_bits(2)), magic_val(2)), n2));
+        o[2] = h2u(__hfma2(a2, __hsub2(u2h((w & 0x00300030u) | magic_bits(4)), magic_val(4)), n2));
+        o[3] = h2u(__hfma2(a2, __hsub2(u2h((w & 0x00C000C0u) | magic_bits(6)), magic_val(6)), n2));
+        o[4] = h2u(__hfma2(a2, __hsub2(u2h((w & 0x03000300u) | magic_bits(8)), magic_val(8)), n2));
+        o[5] = h2u(__hfma2(a2, __hsub2(u2h((wh & 0x00030003u) | magic_bits(0)), magic_val(0)), n2));
+        o[6] = h2u(__hfma2(a2, __hsub2(u2h((wh & 0x000C000Cu) | magic_bits(2)), magic_val(2)), n2));
+        o[7] = h2u(__hfma2(a2, __hsub2(u2h((wh & 0x00300030u) | magic_bits(4)), magic_val(4)), n2));
+        st_row(dst + (2 * i) * kMT, o[0], o[1], o[2], o[3]);
+        st_row(dst + (2 * i + 1) * kMT, o[4], o[5], o[6], o[7]);
+    }
+}
+
+// Q3_K: code q = low two bits + 4 * high bit, weight d * (s - 32) * (q - 4)
+__device__ __forceinline__ void dq_q3k(const SBlk& B, int cc, int hf, uint4* dst) {
+    const __half2 d2 = u2h((B.dd & 0xFFFFu) * 0x00010001u);
+    const int u = q16_slot(4 * cc + 2 * hf);   // slots u, u + 1 (u even)
+    const uint32_t lo = (pick_word(B.sc, u >> 3) >> (8 * ((u >> 1) & 3))) & 0xFFu;   // nibbles of slots u, u + 1
+    const uint32_t hb = (B.sc[2] >> (8 * (u >> 2) + 2 * (u & 3))) & 0xFu;            // high bits: 2 per slot
+    const uint32_t sx = (lo & 15u) | ((hb & 3u) << 4) | (((lo >> 4) | ((hb >> 2) << 4)) << 16);
+    const __half2 ap = __hmul2(d2, __hsub2(u2h(sx | 0x64006400u), u2h(0x64206420u)));
+    #pragma unroll
+    for (int ii = 0; ii < 2; ++ii) {
+        const int i = 2 * hf + ii;
+        const __half2 a2 = ii ? __high2half2(ap) : __low2half2(ap);
+        const uint4 cw = B.cw[ii];
+        const uint32_t l0 = (cc & 1) ? cw.y : cw.x, l1 = (cc & 1) ? cw.w : cw.z;
+        const uint32_t wl = (cc & 2) ? l1 : l0, wl8 = wl >> 8;
+        const uint32_t wh = ((cc >> 1) ? B.hw[ii].y : B.hw[ii].x) >> (8 * (cc & 1));
+        // pair m: low bits at 2m (m < 4) or 2m - 8 of wl >> 8 (m >= 4); its
+        // high bit (bit m of wh) moved two bits above them
+        uint32_t o[8];
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const int p = m < 4 ? 2 * m : 2 * m - 8;          // low bits' position
+            const int sh = p + 2 - m;                          // high bit: m -> p + 2
+            const uint32_t hsh = sh >= 0 ? (wh << sh) : (wh >> -sh);
+            const uint32_t lm = 0x00030003u << p, hm = 0x00010001u << (p + 2);
+            const uint32_t t = ((m < 4 ? wl : wl8) & lm) | (hsh & hm) | magic_bits(p);
+            // (2^(10-p) + q) - (2^(10-p) + 4) = q - 4, exact
+            o[m] = h2u(__hmul2(a2, __hsub2(u2h(t), u2h(magic_bits(p) + (4u << p) * 0x00010001u))));
+        }
+        st_row(dst + (2 * i) * kMT, o[0], o[1], o[2], o[3]);
+        st_row(dst + (2 * i + 1) * kMT, o[4], o[5], o[6], o[7]);
+    }
+}
+
+// Q4_K: sub-block j = 2 cc + hf (32 weights), weight d * sc * q - dmin * m
+__device__ __forceinline__ void dq_q4k(const SBlk& B, int cc, int hf, uint4* dst) {
+    const int j = 2 * cc + hf;
+    const uint32_t lo = (pick_word(B.sc, j >> 2) >> (8 * (j & 3))) & 0xFFu, high = B.sc[2] >> (4 * j);
+    const uint32_t sc = (lo & 15u) | ((high & 3u) << 4), mn = (lo >> 4) | (((high >> 2) & 3u) << 4);
+    // (d, -dmin) * (sc, m): both products in one pair
+    const __half2 dm = u2h((B.dd & 0xFFFFu) | ((B.dd & 0xFFFF0000u) ^ 0x80000000u));
+    const __half2 pr = __hmul2(dm, __hsub2(u2h((sc | (mn << 16)) | 0x64006400u), magic_val(0)));
+    const __half2 a2 = __low2half2(pr), n2 = __high2half2(pr);
+    const uint4 cw = pick4(B.cw, cc);
+    const uint32_t W[4] = {cw.x, cw.y, cw.z, cw.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint32_t w = W[q], w8 = w >> 8;
+        const uint32_t o0 = h2u(__hfma2(a2, __hsub2(u2h((w & 0x000F000Fu) | magic_bits(0)), magic_val(0)), n2));
+        const uint32_t o1 = h2u(__hfma2(a2, __hsub2(u2h((w & 0x00F000F0u) | magic_bits(4)), magic_val(4)), n2));
+        const uint32_t o2 = h2u(__hfma2(a2, __hsub2(u2h((w8 & 0x000F000Fu) | magic_bits(0)), magic_val(0)), n2));
+        const uint32_t o3 = h2u(__hfma2(a2, __hsub2(u2h((w8 & 0x00F000F0u) | magic_bits(4)), magic_val(4)), n2));
+        st_row(dst + (4 * hf + q) * kMT, o0, o1, o2, o3);
+    }
+}
+
+// Q8_0: block 2 c + hf of the chunk (32 weights), weight d * (q - 128)
+__device__ __forceinline__ void dq_q80(const uint32_t (&w)[8], uint32_t d16, int hf, uint4* dst) {
+    const __half2 d2 = u2h((d16 & 0xFFFFu) * 0x00010001u);
+    const __half2 k1152 = u2h(0x64806480u);   // 1024 + 128
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint32_t o[4];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const uint32_t v = w[2 * q + h];
+            o[2 * h] = h2u(__hmul2(d2, __hsub2(u2h((v & 0x00FF00FFu) | 0x64006400u), k1152)));
+            o[2 * h + 1] = h2u(__hmul2(d2, __hsub2(u2h(((v >> 8) & 0x00FF00FFu) | 0x64006400u), k1152)));
+        }
+        st_row(dst + (4 * hf + q) * kMT, o[0], o[1], o[2], o[3]);
+    }
+}
+
+template <bool kDown>
+__global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __grid_constant__ ExpertTab tab,
+                                                                      const __grid_constant__ PrefillArgs A) {
+    constexpr int kTens = kDown ? 1 : 2;
+    constexpr int kW = g_workers(kDown);            // worker warps
+    constexpr int kThr = g_threads(kDown);
+    constexpr int kWarpP = kW, kWarpB = kW + 1, kWarpM = kW + 2;
+    pdl_wait();
+    pdl_launch();
+    extern __shared__ __align__(1024) uint8_t smem[];
+    __shared__ GSlots sl;
+    __shared__ GUnit s_unit[2];
+    __shared__ int32_t s_row[2][kGNT], s_asg[2][kGNT], s_ex[2][kGNT];
+    __shared__ float s_w[2][kGNT];
+    __shared__ __align__(8) uint64_t op_full[kGOps], op_empty[kGOps], pk_full[kGPk], pk_empty[kGPk];
+    __shared__ __align__(8) uint64_t u_full[2], u_empty[2];
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    const Dims& d = A.d;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n_mt = (kDown ? d.H : d.I) / kMT;
+    const int K = kDown ? d.I : d.H;
+    const int nC = K / kKC;
+    const int n_slots = A.active[0] + d.has_shared;
+    for (int i = tid; i < n_slots; i += kThr) {
+        int e;
+        if (i < d.has_shared) { e = d.E; sl.first[i] = d.T * d.K; sl.ntot[i] = d.T; }
+        else {
+            e = A.active[1 + i - d.has_shared];
+            sl.first[i] = A.offsets[e]; sl.ntot[i] = A.offsets[e + 1] - A.offsets[e];
+        }
+        sl.e[i] = e;
+        sl.fmt[i][0] = tab.fmt[e][kDown ? 2 : 0];
+        sl.fmt[i][1] = tab.fmt[e][1];
+    }
+    __syncthreads();
+    const uint32_t ring = (uint32_t)__cvta_generic_to_shared(smem);
+    const uint32_t pk0 = ring + kGOps * kGSlotBytes;
+    const uint32_t opf = (uint32_t)__cvta_generic_to_shared(op_full), ope = (uint32_t)__cvta_generic_to_shared(op_empty);
+    const uint32_t pkf = (uint32_t)__cvta_generic_to_shared(pk_full), pke = (uint32_t)__cvta_generic_to_shared(pk_empty);
+    const uint32_t uf = (uint32_t)__cvta_generic_to_shared(u_full), ue = (uint32_t)__cvta_generic_to_shared(u_empty);
+    if (tid == 0) {
+        int run = 0;
+        for (int i = 0; i < n_slots; ++i) { sl.pre[i] = run; run += n_mt * ((sl.ntot[i] + kGNT - 1) / kGNT); }
+        sl.pre[n_slots] = run;
+        s_fail = 0;
+        // operand slot: the worker warps that decode a chunk (all 16 for
+        // gate/up, 8 for down) and the activation warp's expect-tx arrival; packed stage and unit slot: one
+        // arrival per worker warp (+ the activation and MMA warps)
+        for (int i = 0; i < kGOps; ++i) { g_mbar_init(opf + 8 * i, 32 * (kDown ? kW / 2 : kW) + 1); g_mbar_init(ope + 8 * i, 1); }
+        for (int i = 0; i < kGPk; ++i) { g_mbar_init(pkf + 8 * i, 1); g_mbar_init(pke + 8 * i, kW); }
+        for (int i = 0; i < 2; ++i) { g_mbar_init(uf + 8 * i, 1); g_mbar_init(ue + 8 * i, kW + 2); }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    constexpr int kCols = kDown ? kGNT : 2 * kGNT;
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     ::"r"((uint32_t)__cvta_generic_to_shared(&s_tmem)), "r"(kCols) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tbase = s_tmem;
+    const int n_units = sl.pre[n_slots];
+    auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
+    auto fail = [&]() { atomicOr(A.err, kErrMma); s_fail = 1; };
+
+    if (warp == kWarpP) {
+        // ---- producer: units and packed records
+        const uint64_t pol = [] { uint64_t p; asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p)); return p; }();
+        int cursor = 0, pq = 0;
+        for (int ui = 0;; ++ui) {
+            const int us = ui & 1;
+            if (ui >= 2 && !mbar_wait(ue + 8 * us, ((ui - 2) >> 1) & 1)) { if (lane == 0) fail(); break; }
+            int u = 0;
+            if (lane == 0) u = (int)atomicAdd(A.next + (kDown ? 1 : 0), 1u);
+            u = __shfl_sync(0xffffffffu, u, 0);
+            if (u >= n_units || failed()) {
+                if (lane == 0) { s_unit[us].u = -1; mbar_arrive(uf + 8 * us); }
+                break;
+            }
+            while (cursor + 1 < n_slots && sl.pre[cursor + 1] <= u) ++cursor;
+            const int p = cursor, local = u - sl.pre[p];
+            const int tt = local / n_mt, mt = local - tt * n_mt;
+            const int n0 = tt * kGNT, N = min(kGNT, sl.ntot[p] - n0);
+            const bool shared = p < d.has_shared;
+            for (int n = lane; n < kGNT; n += 32) {
+                int a = -1, row = 0, ex = 0;
+                float w = 0.0f;
+                if (n < N) {
+                    const int q = n0 + n;
+                    if (shared) { a = d.T * d.K + q; row = q; w = 1.0f; }
+                    else { a = A.perm[sl.first[p] + q]; row = a / d.K; w = A.wts[a]; }
+                    ex = A.xe[row];
+                    if (kDown) row = a;
+                }
+                s_row[us][n] = row; s_asg[us][n] = a; s_w[us][n] = w; s_ex[us][n] = ex;
+            }
+            const int f0 = sl.fmt[p][0], f1 = kDown ? f0 : sl.fmt[p][1];
+            const int ks = (f0 == kQ80 || f1 == kQ80) ? 128 : 256;
+            const GStage G = gstage(f0, f1, kTens, ks);
+            if (G.total > kGPkBytes) {   // only the four formats above come here
+                if (lane == 0) { fail(); s_unit[us].u = -1; mbar_arrive(uf + 8 * us); }
+                break;
+            }
+            if (lane == 0) {
+                GUnit g;
+                g.u = u; g.p = p; g.mt = mt; g.N = N; g.Npad = (N + 15) & ~15; g.ks = ks; g.r0 = sl.first[p] + n0;
+                s_unit[us] = g;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(uf + 8 * us);
+            // this lane's copy: tensor z, plane pl, tile tl (lane = 16 z + 4 pl + tl)
+            // (the per-lane choices are unrolled selects, so nothing is indexed at run time)
+            const int z = lane >> 4, pl = (lane >> 2) & 3, tl = lane & 3;
+            const int fz = z == 0 ? f0 : f1;
+            const uint8_t* src0 = nullptr;
+            int64_t sstep = 0;
+            uint32_t bytes = 0, doff = 0;
+#pragma unroll
+            for (int zz = 0; zz < kTens; ++zz) {
+                const int fm = zz == 0 ? f0 : f1;
+                const PlaneBytes pb = plane_bytes(fm);
+                const TensorLayout L = tensor_layout(fm, kDown ? d.H : d.I, K);
+#pragma unroll
+                for (int pp = 0; pp < 4; ++pp) {
+                    if (zz == z && pp == pl && pp < pb.n) {
+                        src0 = tab.p[sl.e[p]][zz == 0 ? (kDown ? 2 : 0) : 1] + L.plane[pp] +
+                               unit_offset(L.blocks_per_row, pb.b[pp], (int64_t)mt * kMT + 32 * tl, 0, 0);
+                        bytes = (uint32_t)G.tile[zz][pp];
+                        doff = (uint32_t)(G.off[zz][pp] + tl * G.tile[zz][pp]);
+                        sstep = (int64_t)32 * pb.b[pp];   // bytes per block of one tile
+                    }
+                }
+            }
+            const bool mine = bytes != 0;
+            const int cps = ks / kKC;
+            const int nst = (nC + cps - 1) / cps;   // a last K-quant superblock may hold 128 columns only
+            bool bad = false;
+            for (int st = 0; st < nst; ++st, ++pq) {
+                const int ps = pq % kGPk;
+                if (pq >= kGPk && !mbar_wait(pke + 8 * ps, ((pq - kGPk) / kGPk) & 1)) { bad = true; break; }
+                if (failed()) { bad = true; break; }
+                if (lane == 0) g_arrive_tx(pkf + 8 * ps, (uint32_t)G.total);
+                __syncwarp();
+                if (mine) {
+                    const int64_t blk = fz == kQ80 ? (int64_t)st * (ks / 32) : (int64_t)st * ks / 256;
+                    g_bulk(pk0 + ps * kGPkBytes + doff, src0 + blk * sstep, bytes, pkf + 8 * ps, pol);
+                }
+            }
+            if (bad) { if (lane == 0) fail(); break; }
+        }
+        // the stages still in flight land before the CTA exits
+        for (int q = max(0, pq - kGPk); q < pq; ++q) (void)mbar_wait(pkf + 8 * (q % kGPk), (q / kGPk) & 1);
+    } else if (warp == kWarpB) {
+        // ---- activations: the chunk's rows of the unit's tile, eight bulk copies
+        // (one per 8-column piece) into the operand slot; the MMA may read rows
+        // N .. Npad - 1 of an earlier chunk: they only reach accumulator
+        // columns the epilogue never reads
+        const uint8_t* src = kDown ? reinterpret_cast<const uint8_t*>(A.h16) : A.xp;
+        int gq = 0;
+        for (int ui = 0;; ++ui) {
+            const int us = ui & 1;
+            if (!mbar_wait(uf + 8 * us, (ui >> 1) & 1)) { if (lane == 0) fail(); break; }
+            const GUnit U = s_unit[us];
+            if (U.u < 0) break;
+            bool bad = false;
+            for (int c = 0; c < nC; ++c, ++gq) {
+                const int s = gq % kGOps;
+                if (gq >= kGOps && !mbar_wait(ope + 8 * s, ((gq - kGOps) / kGOps) & 1)) { bad = true; break; }
+                if (failed()) { bad = true; break; }
+                if (lane == 0) g_arrive_tx(opf + 8 * s, (uint32_t)(U.N * 128));
+                __syncwarp();
+                if (lane < 8)
+                    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                                 ::"r"(ring + s * kGSlotBytes + 2 * kABytes + lane * kGNT * 16),
+                                   "l"(src + perm_piece(U.r0, K, U.N, c * 8 + lane, 0)), "r"((uint32_t)(U.N * 16)),
+                                   "r"(opf + 8 * s) : "memory");
+            }
+            if (bad) { if (lane == 0) fail(); break; }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(ue + 8 * us);
+        }
+    } else if (warp == kWarpM) {
+        // ---- MMA issue
+        int mq = 0, last = -1;
+        for (int ui = 0;; ++ui) {
+            const int us = ui & 1;
+            if (!mbar_wait(uf + 8 * us, (ui >> 1) & 1)) { if (lane == 0) fail(); break; }
+            const GUnit U = s_unit[us];
+            if (U.u < 0) break;
+            bool bad = false;
+            for (int c = 0; c < nC; ++c, ++mq) {
+                const int s = mq % kGOps;
+                if (!mbar_wait(opf + 8 * s, (mq / kGOps) & 1)) { bad = true; break; }
+                if (lane == 0) {
+                    // (the workers fenced their operand stores; the activations came by bulk copy)
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t idesc = idesc_f16(kMT, U.Npad);
+                    const uint32_t sbase = ring + s * kGSlotBytes, bsm = sbase + 2 * kABytes;
+#pragma unroll
+                    for (int kk = 0; kk < kKC / 16; ++kk) {
+                        const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;
+                        const uint64_t db = sdesc(bsm + 2 * kk * kGNT * 16, kGNT * 16, 128);
+                        mma_f16(tbase, sdesc(sbase + 2 * kk * kMT * 16, kMT * 16, 128), db, idesc, acc);
+                        if (!kDown)
+                            mma_f16(tbase + kGNT, sdesc(sbase + kABytes + 2 * kk * kMT * 16, kMT * 16, 128), db, idesc, acc);
+                    }
+                    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                                 ::"r"(ope + 8 * s) : "memory");
+                }
+                __syncwarp();
+                last = mq;
+            }
+            if (bad) { if (lane == 0) fail(); break; }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(ue + 8 * us);
+        }
+        // tensor memory is released only after the MMAs issued here are done
+        if (last >= 0) (void)mbar_wait(ope + 8 * (last % kGOps), (last / kGOps) & 1);
+    } else {
+        // ---- workers: decode and epilogue.  Gate/up: warps 0-7 decode the gate
+        // tensor, 8-15 the up tensor, of every chunk; down: warps 0-7 the even
+        // chunks, 8-15 the odd ones.  Warp w takes the weight rows of tile w % 4
+        // and half (w / 4) % 2 of its chunks.
+        constexpr int nG = kDown ? 2 : 1;          // chunk groups
+        const int z = kDown ? 0 : (warp >> 3);
+        const int gsel = kDown ? (warp >> 3) : 0;
+        const int tl = warp & 3, hf = (warp >> 2) & 1;
+        const int rr = 32 * tl + lane;
+        uint4* const sv4 = reinterpret_cast<uint4*>(smem);
+        int gbase = 0, pbase = 0;   // chunks and packed stages of the earlier units
+        for (int ui = 0;; ++ui) {
+            const int us = ui & 1;
+            if (!mbar_wait(uf + 8 * us, (ui >> 1) & 1)) { if (lane == 0) fail(); break; }
+            const GUnit U = s_unit[us];
+            if (U.u < 0) break;
+            const int f0 = sl.fmt[U.p][0], f1 = kDown ? f0 : sl.fmt[U.p][1];
+            const int fz = z ? f1 : f0;
+            const GStage G = gstage(f0, f1, kTens, U.ks);
+            uint32_t rec[4];   // this thread's records in stage 0 (stage s at + s * kGPkBytes)
+#pragma unroll
+            for (int pl = 0; pl < 4; ++pl)
+                rec[pl] = pk0 + (uint32_t)((z ? G.off[1][pl] : G.off[0][pl]) + tl * (z ? G.tile[1][pl] : G.tile[0][pl]) +
+                                           lane * (z ? G.ub[1][pl] : G.ub[0][pl]));
+            const int cps = U.ks / kKC;
+            bool bad = false;
+            SBlk B;
+            uint32_t so = 0;
+            int ps = 0, cur = -1;
+            for (int c = gsel; c < nC; c += nG) {
+                const int g = gbase + c, s = g % kGOps, st = c / cps, cl = c - st * cps;
+                if (st != cur) {
+                    cur = st;
+                    const int q = pbase + st;
+                    ps = q % kGPk;
+                    if (!mbar_wait(pkf + 8 * ps, (q / kGPk) & 1)) { bad = true; break; }
+                    so = (uint32_t)(ps * kGPkBytes);
+                    if (fz != kQ80) {
+                        const uint32_t r[4] = {rec[0] + so, rec[1] + so, rec[2] + so, rec[3] + so};
+                        load_sblk_s(fz, r, hf, B);
+                    }
+                }
+                if (g >= kGOps && !mbar_wait(ope + 8 * s, ((g - kGOps) / kGOps) & 1)) { bad = true; break; }
+                if (failed()) { bad = true; break; }
+                uint4* const dst = sv4 + (s * kGSlotBytes + z * kABytes) / 16 + rr;
+                if (fz == kQ2K) {
+                    dq_q2k(B, c & 3, hf, dst);
+                } else if (fz == kQ3K) {
+                    dq_q3k(B, c & 3, hf, dst);
+                } else if (fz == kQ4K) {
+                    dq_q4k(B, c & 3, hf, dst);
+                } else {   // Q8_0: block 2 cl + hf of the stage
+                    const int lb = 2 * cl + hf;
+                    const uint32_t cp = rec[1] + so + lb * (32 * 32);
+                    const uint4 w0 = g_lds128(cp), w1 = g_lds128(cp + 16);
+                    const uint32_t w[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+                    dq_q80(w, g_lds16(rec[0] + so + lb * (32 * 2)), hf, dst);
+                }
+                // this thread's operand stores before the tensor cores read them
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                mbar_arrive(opf + 8 * s);
+                if (c + nG >= nC || (c + nG) / cps != st) {   // this warp's last chunk of the stage
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(pke + 8 * ps);
+                }
+            }
+            gbase += nC;
+            pbase += (nC + cps - 1) / cps;
+            if (bad) { if (lane == 0) fail(); break; }
+            // the unit's MMAs are done once its last chunk's commit arrived.  The
+            // slots' commits are awaited in chunk order: a phase-parity wait may
+            // run at most one phase ahead of its barrier, and a warp that skipped
+            // the other group's chunks has seen only every second completion
+            for (int gg = max(0, gbase - kGOps); gg < gbase && !bad; ++gg)
+                bad = !mbar_wait(ope + 8 * (gg % kGOps), (gg / kGOps) & 1);
+            if (bad) { if (lane == 0) fail(); break; }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            // epilogue: TMEM lane 32 (w % 4) + lane = weight row; the worker
+            // warps of a lane quarter take every (kW / 4)-th group of 8 columns
+            const int row = U.mt * kMT + 32 * tl + lane;
+            bool over = false;
+            for (int n = 8 * (warp >> 2); n < U.Npad; n += 2 * kW) {
+                uint32_t g8[8], u8[8];
+                const uint32_t ta = tbase + ((uint32_t)(32 * tl) << 16) + (uint32_t)n;
+                asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                             : "=r"(g8[0]), "=r"(g8[1]), "=r"(g8[2]), "=r"(g8[3]), "=r"(g8[4]), "=r"(g8[5]),
+                               "=r"(g8[6]), "=r"(g8[7]) : "r"(ta));
+                if (!kDown)
+                    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                                 : "=r"(u8[0]), "=r"(u8[1]), "=r"(u8[2]), "=r"(u8[3]), "=r"(u8[4]), "=r"(u8[5]),
+                                   "=r"(u8[6]), "=r"(u8[7]) : "r"(ta + kGNT));
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int nn = n + j;
+                    if (nn >= U.N) break;
+                    const int a = s_asg[us][nn], ex = s_ex[us][nn];
+                    if (kDown) {
+                        A.pdn[(size_t)a * d.H + row] = ldexpf(__uint_as_float(g8[j]), 2 * ex);
+                    } else {
+                        const float gv = ldexpf(__uint_as_float(g8[j]), ex), uv = ldexpf(__uint_as_float(u8[j]), ex);
+                        const float hs = ldexpf(silu(gv) * uv * s_w[us][nn], -2 * ex);
+                        over |= !(fabsf(hs) <= 65504.0f);
+                        // h in the down GEMM's activation layout (slot position U.r0 + nn)
+                        *reinterpret_cast<__half*>(reinterpret_cast<uint8_t*>(A.h16) +
+                                                   perm_piece(U.r0, d.I, U.N, row >> 3, nn) + (row & 7) * 2) =
+                            __float2half_rn(hs);
+                    }
+                }
+            }
+            if (over) atomicOr(A.err, kErrRange);
+            // the accumulators are read: the next unit's MMAs wait for this
+            // thread's arrival on their operand slot
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(ue + 8 * us);
+        }
+    }
+    __syncthreads();
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(kCols) : "memory");
+    }
+}
+
 void prefill_setup() {
     const int smem = kPSlots * kSlotBytes;
     cudaFuncSetAttribute(prefill_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(prefill_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(prefill_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(prefill_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(gemm_ws_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
+    cudaFuncSetAttribute(gemm_ws_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
 }
 
 }  // namespace
@@ -804,16 +1493,24 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     bool rare = false;   // a Q6_K or BF16 tensor anywhere in the layer
     for (int e = 0; e < d.E + d.has_shared; ++e)
         for (int j = 0; j < 3; ++j) rare |= tab.fmt[e][j] == kQ6K || tab.fmt[e][j] == kBF16;
+    A.xp = reinterpret_cast<uint8_t*>(w.pdn);   // dead until the down GEMM writes its partial rows
+    if (!rare) {
+        prof_begin("xperm", s);
+        const cudaError_t ex = launch_pdl(xperm_kernel, dim3(2 * g_psms), dim3(256), 0, s,
+                                          static_cast<const __half*>(w.x16), static_cast<const int32_t*>(w.offsets),
+                                          static_cast<const int32_t*>(w.perm), d, A.xp);
+        prof_end(s);
+        if (ex != cudaSuccess) return ex;
+    }
     prof_begin("gateup_tc", s);
     cudaError_t err = rare ? launch_pdl(prefill_kernel<false, true>, dim3(g_psms), dim3(prefill_threads(false)), smem,
                                         s, tab, A)
-                           : launch_pdl(prefill_kernel<false, false>, dim3(g_psms), dim3(prefill_threads(false)), smem,
-                                        s, tab, A);
+                           : launch_pdl(gemm_ws_kernel<false>, dim3(g_psms), dim3(g_threads(false)), kGSmem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     prof_begin("down_tc", s);
     err = rare ? launch_pdl(prefill_kernel<true, true>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A)
-               : launch_pdl(prefill_kernel<true, false>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A);
+               : launch_pdl(gemm_ws_kernel<true>, dim3(g_psms), dim3(g_threads(true)), kGSmem, s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);
