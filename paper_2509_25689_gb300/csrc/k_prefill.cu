@@ -828,35 +828,61 @@ __device__ __forceinline__ size_t perm_piece(int r0, int K, int N, int p, int n)
     return (size_t)r0 * K * 2 + ((size_t)p * N + n) * 16;
 }
 
-// The tokens (fp16, as the logits kernel scaled them) in that layout.
-__global__ void __launch_bounds__(256) xperm_kernel(const __half* __restrict__ x16,
-                                                    const int32_t* __restrict__ offsets,
-                                                    const int32_t* __restrict__ perm, const Dims d,
-                                                    uint8_t* __restrict__ xp) {
+// The tokens (fp16, as the logits kernel scaled them) in that layout.  Work
+// items are (tile, 64 pieces) of the call's tiles (the slots' tiles in slot
+// order); warp w writes the runs of pieces w, w + 8, ... of its item: lane l
+// the rows l, l + 32, ... of a run, so every store of a warp is 512
+// contiguous bytes.
+constexpr int kXpWarps = 8, kXpPieces = 64;
+__global__ void __launch_bounds__(kXpWarps * 32) xperm_kernel(const __half* __restrict__ x16,
+                                                              const int32_t* __restrict__ offsets,
+                                                              const int32_t* __restrict__ perm,
+                                                              const int32_t* __restrict__ active, const Dims d,
+                                                              uint8_t* __restrict__ xp) {
     pdl_wait();
-    __shared__ int32_t s_off[kMaxExperts + 1];
-    const int E = d.E, TK = d.T * d.K, A = TK + (d.has_shared ? d.T : 0);
-    for (int i = threadIdx.x; i <= E; i += blockDim.x) s_off[i] = offsets[i];
-    __syncthreads();
-    const int lane = threadIdx.x & 31, np = d.H / 8;
-    for (int r = blockIdx.x * 8 + (threadIdx.x >> 5); r < A; r += gridDim.x * 8) {
-        int pos0, ntot, t;
-        if (r < TK) {
-            // the expert of position r: the last e with offsets[e] <= r
-            int lo = 0, hi = E - 1;
-            while (lo < hi) {
-                const int mid = (lo + hi + 1) >> 1;
-                if (s_off[mid] <= r) lo = mid; else hi = mid - 1;
-            }
-            pos0 = s_off[lo]; ntot = s_off[lo + 1] - pos0; t = perm[r] / d.K;
-        } else {
-            pos0 = TK; ntot = d.T; t = r - TK;
+    __shared__ int32_t s_first[kMaxExperts + 1], s_ntot[kMaxExperts + 1], s_pre[kMaxExperts + 2];
+    __shared__ int32_t s_tok[kGNT];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n_slots = active[0] + d.has_shared, TK = d.T * d.K, np = d.H / 8;
+    for (int i = tid; i < n_slots; i += blockDim.x) {
+        if (i < d.has_shared) { s_first[i] = TK; s_ntot[i] = d.T; }
+        else {
+            const int e = active[1 + i - d.has_shared];
+            s_first[i] = offsets[e]; s_ntot[i] = offsets[e + 1] - offsets[e];
         }
-        const int q = r - pos0, tt = q / kGNT, n = q - tt * kGNT, N = min(kGNT, ntot - tt * kGNT);
-        const int r0 = pos0 + tt * kGNT;
-        const uint4* src = reinterpret_cast<const uint4*>(x16 + (size_t)t * d.H);
-        for (int p = lane; p < np; p += 32)
-            *reinterpret_cast<uint4*>(xp + perm_piece(r0, d.H, N, p, n)) = __ldg(src + p);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int run = 0;
+        for (int i = 0; i < n_slots; ++i) { s_pre[i] = run; run += (s_ntot[i] + kGNT - 1) / kGNT; }
+        s_pre[n_slots] = run;
+    }
+    __syncthreads();
+    // work items: (tile, block of kXpPieces pieces), so that large tiles spread over CTAs
+    const int n_pb = (np + kXpPieces - 1) / kXpPieces, n_items = s_pre[n_slots] * n_pb;
+    int p = 0;
+    for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+        const int ti = it / n_pb, pb = it - ti * n_pb;
+        while (p + 1 < n_slots && s_pre[p + 1] <= ti) ++p;
+        const int tt = ti - s_pre[p], r0 = s_first[p] + tt * kGNT, N = min(kGNT, s_ntot[p] - tt * kGNT);
+        __syncthreads();   // the previous item's token ids are read
+        for (int n = tid; n < N; n += blockDim.x) s_tok[n] = p < d.has_shared ? tt * kGNT + n : perm[r0 + n] / d.K;
+        __syncthreads();
+        uint8_t* dst = xp + (size_t)r0 * d.H * 2;
+        const int pe = min(np, (pb + 1) * kXpPieces);
+        for (int pc = pb * kXpPieces + warp; pc < pe; pc += kXpWarps) {
+            uint4 v[kGNT / 32];   // all loads of the run first, then the stores
+#pragma unroll
+            for (int j = 0; j < kGNT / 32; ++j) {
+                const int n = lane + 32 * j;
+                if (n < N) v[j] = __ldg(reinterpret_cast<const uint4*>(x16 + (size_t)s_tok[n] * d.H) + pc);
+            }
+#pragma unroll
+            for (int j = 0; j < kGNT / 32; ++j) {
+                const int n = lane + 32 * j;
+                if (n < N) *reinterpret_cast<uint4*>(dst + ((size_t)pc * N + n) * 16) = v[j];
+            }
+        }
     }
     pdl_launch();
 }
@@ -1496,9 +1522,10 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     A.xp = reinterpret_cast<uint8_t*>(w.pdn);   // dead until the down GEMM writes its partial rows
     if (!rare) {
         prof_begin("xperm", s);
-        const cudaError_t ex = launch_pdl(xperm_kernel, dim3(2 * g_psms), dim3(256), 0, s,
+        const cudaError_t ex = launch_pdl(xperm_kernel, dim3(4 * g_psms), dim3(kXpWarps * 32), 0, s,
                                           static_cast<const __half*>(w.x16), static_cast<const int32_t*>(w.offsets),
-                                          static_cast<const int32_t*>(w.perm), d, A.xp);
+                                          static_cast<const int32_t*>(w.perm), static_cast<const int32_t*>(w.active),
+                                          d, A.xp);
         prof_end(s);
         if (ex != cudaSuccess) return ex;
     }
