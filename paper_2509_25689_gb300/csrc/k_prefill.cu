@@ -1395,43 +1395,60 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
             bool bad = false;
             SBlk B;
             uint32_t so = 0;
-            int ps = 0, cur = -1;
-            for (int c = gsel; c < nC; c += nG) {
-                const int g = gbase + c, s = g % kGOps, st = c / cps, cl = c - st * cps;
-                if (st != cur) {
-                    cur = st;
-                    const int q = pbase + st;
-                    ps = q % kGPk;
-                    if (!mbar_wait(pkf + 8 * ps, (q / kGPk) & 1)) { bad = true; break; }
-                    so = (uint32_t)(ps * kGPkBytes);
-                    if (fz != kQ80) {
-                        const uint32_t r[4] = {rec[0] + so, rec[1] + so, rec[2] + so, rec[3] + so};
-                        load_sblk_s(fz, r, hf, B);
-                    }
-                }
-                if (g >= kGOps && !mbar_wait(ope + 8 * s, ((g - kGOps) / kGOps) & 1)) { bad = true; break; }
-                if (failed()) { bad = true; break; }
+            // one chunk: c its index in the unit, cc its 64-column quarter of the
+            // superblock, lb its first Q8_0 block in the stage
+            auto chunk = [&](int c, int cc, int lb, uint32_t so) -> bool {
+                const int g = gbase + c, s = g % kGOps;
+                if (g >= kGOps && !mbar_wait(ope + 8 * s, ((g - kGOps) / kGOps) & 1)) return false;
+                if (failed()) return false;
                 uint4* const dst = sv4 + (s * kGSlotBytes + z * kABytes) / 16 + rr;
                 if (fz == kQ2K) {
-                    dq_q2k(B, c & 3, hf, dst);
+                    dq_q2k(B, cc, hf, dst);
                 } else if (fz == kQ3K) {
-                    dq_q3k(B, c & 3, hf, dst);
+                    dq_q3k(B, cc, hf, dst);
                 } else if (fz == kQ4K) {
-                    dq_q4k(B, c & 3, hf, dst);
-                } else {   // Q8_0: block 2 cl + hf of the stage
-                    const int lb = 2 * cl + hf;
-                    const uint32_t cp = rec[1] + so + lb * (32 * 32);
+                    dq_q4k(B, cc, hf, dst);
+                } else {   // Q8_0: block lb + hf of the stage
+                    const uint32_t cp = rec[1] + so + (lb + hf) * (32 * 32);
                     const uint4 w0 = g_lds128(cp), w1 = g_lds128(cp + 16);
                     const uint32_t w[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-                    dq_q80(w, g_lds16(rec[0] + so + lb * (32 * 2)), hf, dst);
+                    dq_q80(w, g_lds16(rec[0] + so + (lb + hf) * (32 * 2)), hf, dst);
                 }
                 // this thread's operand stores before the tensor cores read them
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 mbar_arrive(opf + 8 * s);
-                if (c + nG >= nC || (c + nG) / cps != st) {   // this warp's last chunk of the stage
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(pke + 8 * ps);
+                return true;
+            };
+            const int nst = (nC + cps - 1) / cps;
+            for (int st = 0; st < nst && !bad; ++st) {
+                const int q = pbase + st, ps = q % kGPk;
+                if (!mbar_wait(pkf + 8 * ps, (q / kGPk) & 1)) { bad = true; break; }
+                const uint32_t so = (uint32_t)(ps * kGPkBytes);
+                if (fz != kQ80) {
+                    const uint32_t r[4] = {rec[0] + so, rec[1] + so, rec[2] + so, rec[3] + so};
+                    load_sblk_s(fz, r, hf, B);
                 }
+                if (cps == 4) {
+                    // a whole superblock: the quarter index is a constant in each copy
+#pragma unroll
+                    for (int cl = 0; cl < 4; ++cl) {
+                        const int c = 4 * st + cl;
+                        if (c >= nC) break;
+                        if (kDown && (cl & 1) != gsel) continue;
+                        if (!chunk(c, cl, 0, so)) { bad = true; break; }
+                    }
+                } else {
+                    // 128 columns (a Q8_0 tensor in the unit): one chunk per group
+                    for (int cl = gsel; cl < 2; cl += nG) {
+                        const int c = 2 * st + cl;
+                        if (c >= nC) break;
+                        if (!chunk(c, c & 3, 2 * cl, so)) { bad = true; break; }
+                    }
+                }
+                if (bad) break;
+                // every worker warp takes part in every stage: release it
+                __syncwarp();
+                if (lane == 0) mbar_arrive(pke + 8 * ps);
             }
             gbase += nC;
             pbase += (nC + cps - 1) / cps;
