@@ -1330,7 +1330,19 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
             if (lane == 0) mbar_arrive(ue + 8 * us);
         }
     } else if (warp == kWarpM) {
-        // ---- MMA issue
+        // ---- MMA issue.  The operand descriptors of both slots are built once:
+        // a 16-column step of K moves an A operand by 2 * kMT * 16 bytes and B
+        // by 2 * kGNT * 16 bytes, i.e. the descriptors' start-address field
+        // (bytes / 16) by 256 and 512.
+        static_assert(kGOps == 2, "the issue loop picks a slot's descriptors with a select");
+        uint64_t dA[kGOps][2], dB[kGOps];
+#pragma unroll
+        for (int sl2 = 0; sl2 < kGOps; ++sl2) {
+            const uint32_t sbase = ring + sl2 * kGSlotBytes;
+            dA[sl2][0] = sdesc(sbase, kMT * 16, 128);
+            dA[sl2][1] = sdesc(sbase + kABytes, kMT * 16, 128);
+            dB[sl2] = sdesc(sbase + 2 * kABytes, kGNT * 16, 128);
+        }
         int mq = 0, last = -1;
         for (int ui = 0;; ++ui) {
             const int us = ui & 1;
@@ -1345,14 +1357,12 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
                     // (the workers fenced their operand stores; the activations came by bulk copy)
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint32_t idesc = idesc_f16(kMT, U.Npad);
-                    const uint32_t sbase = ring + s * kGSlotBytes, bsm = sbase + 2 * kABytes;
+                    const uint64_t a0 = s ? dA[1][0] : dA[0][0], a1 = s ? dA[1][1] : dA[0][1], b0 = s ? dB[1] : dB[0];
 #pragma unroll
                     for (int kk = 0; kk < kKC / 16; ++kk) {
                         const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;
-                        const uint64_t db = sdesc(bsm + 2 * kk * kGNT * 16, kGNT * 16, 128);
-                        mma_f16(tbase, sdesc(sbase + 2 * kk * kMT * 16, kMT * 16, 128), db, idesc, acc);
-                        if (!kDown)
-                            mma_f16(tbase + kGNT, sdesc(sbase + kABytes + 2 * kk * kMT * 16, kMT * 16, 128), db, idesc, acc);
+                        mma_f16(tbase, a0 + 256u * kk, b0 + 512u * kk, idesc, acc);
+                        if (!kDown) mma_f16(tbase + kGNT, a1 + 256u * kk, b0 + 512u * kk, idesc, acc);
                     }
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
                                  ::"r"(ope + 8 * s) : "memory");
