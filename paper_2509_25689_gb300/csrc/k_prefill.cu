@@ -810,12 +810,16 @@ __global__ void __launch_bounds__(prefill_threads(kDown), 1) prefill_kernel(cons
 __host__ __device__ constexpr int g_workers(bool down) { return 16; }
 __host__ __device__ constexpr int g_threads(bool down) { return (g_workers(down) + 3) * 32; }
 constexpr int kGNT = 256;                      // tokens per unit (MMA N up to 256)
-constexpr int kGSlotBytes = 2 * kABytes + kGNT * kKC * 2;   // operand slot: A gate | A up | B, 64 KB
-constexpr int kGOps = 2;                       // operand slots (a third one fits only with 128-token
-                                               // units, measured slower on the Zipf prefill)
+// operand slots: gate/up two of A gate | A up | B (64 KB), down three of
+// A | B (48 KB); a third gate/up slot fits only with 128-token units,
+// measured slower on the Zipf prefill
+__host__ __device__ constexpr int g_ops(bool down) { return down ? 3 : 2; }
+__host__ __device__ constexpr int g_bofs(bool down) { return down ? kABytes : 2 * kABytes; }
+__host__ __device__ constexpr int g_slot(bool down) { return g_bofs(down) + kGNT * kKC * 2; }
+constexpr int kGOpsMax = 3;
 constexpr int kGPk = 2;                        // packed-record stages
 constexpr int kGPkBytes = 36 * 1024;           // Q4_K + Q4_K superblock of 128 rows: 2 x 18,432
-constexpr int kGSmem = kGOps * kGSlotBytes + kGPk * kGPkBytes;
+__host__ __device__ constexpr int g_smem(bool down) { return g_ops(down) * g_slot(down) + kGPk * kGPkBytes; }
 
 // Activation rows of the warp-specialised GEMM in the order its units read
 // them: slot positions r (the permutation's order for the routed experts,
@@ -1152,6 +1156,7 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
     constexpr int kW = g_workers(kDown);            // worker warps
     constexpr int kThr = g_threads(kDown);
     constexpr int kWarpP = kW, kWarpB = kW + 1, kWarpM = kW + 2;
+    constexpr int kGOps = g_ops(kDown), kGSlotBytes = g_slot(kDown), kBOfs = g_bofs(kDown);
     pdl_wait();
     pdl_launch();
     extern __shared__ __align__(1024) uint8_t smem[];
@@ -1159,7 +1164,7 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
     __shared__ GUnit s_unit[2];
     __shared__ int32_t s_row[2][kGNT], s_asg[2][kGNT], s_ex[2][kGNT];
     __shared__ float s_w[2][kGNT];
-    __shared__ __align__(8) uint64_t op_full[kGOps], op_empty[kGOps], pk_full[kGPk], pk_empty[kGPk];
+    __shared__ __align__(8) uint64_t op_full[kGOpsMax], op_empty[kGOpsMax], pk_full[kGPk], pk_empty[kGPk];
     __shared__ __align__(8) uint64_t u_full[2], u_empty[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
@@ -1321,7 +1326,7 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
                 __syncwarp();
                 if (lane < 8)
                     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                                 ::"r"(ring + s * kGSlotBytes + 2 * kABytes + lane * kGNT * 16),
+                                 ::"r"(ring + s * kGSlotBytes + kBOfs + lane * kGNT * 16),
                                    "l"(src + perm_piece(U.r0, K, U.N, c * 8 + lane, 0)), "r"((uint32_t)(U.N * 16)),
                                    "r"(opf + 8 * s) : "memory");
             }
@@ -1334,14 +1339,13 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
         // a 16-column step of K moves an A operand by 2 * kMT * 16 bytes and B
         // by 2 * kGNT * 16 bytes, i.e. the descriptors' start-address field
         // (bytes / 16) by 256 and 512.
-        static_assert(kGOps == 2, "the issue loop picks a slot's descriptors with a select");
-        uint64_t dA[kGOps][2], dB[kGOps];
+        uint64_t dA[kGOpsMax][2], dB[kGOpsMax];
 #pragma unroll
-        for (int sl2 = 0; sl2 < kGOps; ++sl2) {
+        for (int sl2 = 0; sl2 < kGOpsMax; ++sl2) {
             const uint32_t sbase = ring + sl2 * kGSlotBytes;
             dA[sl2][0] = sdesc(sbase, kMT * 16, 128);
             dA[sl2][1] = sdesc(sbase + kABytes, kMT * 16, 128);
-            dB[sl2] = sdesc(sbase + 2 * kABytes, kGNT * 16, 128);
+            dB[sl2] = sdesc(sbase + kBOfs, kGNT * 16, 128);
         }
         int mq = 0, last = -1;
         for (int ui = 0;; ++ui) {
@@ -1357,7 +1361,9 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
                     // (the workers fenced their operand stores; the activations came by bulk copy)
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint32_t idesc = idesc_f16(kMT, U.Npad);
-                    const uint64_t a0 = s ? dA[1][0] : dA[0][0], a1 = s ? dA[1][1] : dA[0][1], b0 = s ? dB[1] : dB[0];
+                    const uint64_t a0 = s == 0 ? dA[0][0] : s == 1 ? dA[1][0] : dA[2][0];
+                    const uint64_t a1 = s == 0 ? dA[0][1] : s == 1 ? dA[1][1] : dA[2][1];
+                    const uint64_t b0 = s == 0 ? dB[0] : s == 1 ? dB[1] : dB[2];
 #pragma unroll
                     for (int kk = 0; kk < kKC / 16; ++kk) {
                         const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;
@@ -1527,8 +1533,8 @@ void prefill_setup() {
     cudaFuncSetAttribute(prefill_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(prefill_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(prefill_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    cudaFuncSetAttribute(gemm_ws_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
-    cudaFuncSetAttribute(gemm_ws_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
+    cudaFuncSetAttribute(gemm_ws_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, g_smem(false));
+    cudaFuncSetAttribute(gemm_ws_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, g_smem(true));
 }
 
 }  // namespace
@@ -1559,12 +1565,12 @@ cudaError_t launch_prefill(const Dims& d, const ExpertTab& tab, const Work& w, f
     prof_begin("gateup_tc", s);
     cudaError_t err = rare ? launch_pdl(prefill_kernel<false, true>, dim3(g_psms), dim3(prefill_threads(false)), smem,
                                         s, tab, A)
-                           : launch_pdl(gemm_ws_kernel<false>, dim3(g_psms), dim3(g_threads(false)), kGSmem, s, tab, A);
+                           : launch_pdl(gemm_ws_kernel<false>, dim3(g_psms), dim3(g_threads(false)), g_smem(false), s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     prof_begin("down_tc", s);
     err = rare ? launch_pdl(prefill_kernel<true, true>, dim3(g_psms), dim3(prefill_threads(true)), smem, s, tab, A)
-               : launch_pdl(gemm_ws_kernel<true>, dim3(g_psms), dim3(g_threads(true)), kGSmem, s, tab, A);
+               : launch_pdl(gemm_ws_kernel<true>, dim3(g_psms), dim3(g_threads(true)), g_smem(true), s, tab, A);
     prof_end(s);
     if (err != cudaSuccess) return err;
     return launch_combine(d, w.pdn, out, s);
