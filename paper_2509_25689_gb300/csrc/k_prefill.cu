@@ -312,16 +312,15 @@ __device__ __forceinline__ uint4 pick4(const uint4 (&v)[4], int i) {
     return (i & 2) ? b : a;
 }
 
-// ---- chunk decode for the warp-specialised GEMM: the values dequant_store
-// produces (the same fp16 roundings: d * sc and dmin * m are exact products
-// rounded once, then one fused multiply-add per weight pair), with fewer
-// instructions: a code field at bit s <= 8 of each 16-bit half, OR-ed into
-// the fp16 pair 2^(10 - s), reads as 2^(10 - s) + code exactly (the field
-// lands in the mantissa at unit weight), so one AND-OR and one subtraction
-// give the code without a shift; the scale fields of two sub-blocks are
-// widened as one fp16 pair.  Stores are plain shared-memory stores the
-// compiler may schedule (the proxy fence after them orders them for the
-// tensor cores).
+// ---- chunk decode: each thread turns 32 weights of its row into fp16 in
+// the A operand.  Roundings: d * sc and dmin * m (exact products) are rounded
+// to fp16 once, then one fused multiply-add per weight pair.  A code field at
+// bit s <= 8 of each 16-bit half, OR-ed into the fp16 pair 2^(10 - s), reads
+// as 2^(10 - s) + code exactly (the field lands in the mantissa at unit
+// weight), so one AND-OR and one subtraction give the code without a shift;
+// the scale fields of two sub-blocks are widened as one fp16 pair.  Stores
+// are plain shared-memory stores the compiler may schedule (the proxy fence
+// after them orders them for the tensor cores).
 __device__ __forceinline__ constexpr uint32_t magic_bits(int s) {
     return ((uint32_t)(25 - s) << 10) | ((uint32_t)(25 - s) << 26);
 }
