@@ -743,6 +743,302 @@ __device__ __forceinline__ void tile_epi(const Geo& h, uint32_t st, int jj, int 
     }
 }
 
+// Two tokens of a multi-token item through one 16-row tile (rows 16 rt + g,
+// + 8) of a Q2_K superblock.  The masked code operands do not depend on the
+// token, so each is built once for both tokens' MMAs, and the epilogue's
+// scale conversions are shared; per token the arithmetic is that of
+// tile_mma<kQ2K, 1> and tile_epi<kQ2K, 1> in the same order, so the sums are
+// the ones the per-token passes give.  acc[k][hl]: token tk0 + k's sum of
+// row 16 rt + g + 8 hl, updated in place.
+__device__ __forceinline__ void tile_pair_q2k(const Geo& h, uint32_t st, int jj, int rt, int tk0, uint32_t zaddr,
+                                              float (&acc)[2][2]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const bool own0 = g == t, own1 = g == t + 4;
+    const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
+    const uint32_t tbA = st + h.tok0 + tk0 * h.tstride, tbB = tbA + h.tstride;
+    const uint32_t xbA = tbA + h.tx + jj * 512, xbB = tbB + h.tx + jj * 512;
+    const int rbase = jj * 32 + 16 * rt + g;
+    const uint4 c0 = lds128(st + w3 + rbase * 64 + 16 * t), c1 = lds128(st + w3 + (rbase + 8) * 64 + 16 * t);
+    float D[2][2][2][4];   // [token][sub-block group][pair parity][D fragment]
+#pragma unroll
+    for (int i = 0; i < 32; ++i) (&D[0][0][0][0])[i] = 0.0f;
+#pragma unroll
+    for (int gm = 0; gm < 2; ++gm) {
+        uint32_t XA0[8], XB0[8], XA1[8], XB1[8];
+        ld_frag8(own0 ? xbA + 32 * (8 * gm + t) : zaddr, XA0);
+        ld_frag8(own1 ? xbA + 32 * (8 * gm + 4 + t) : zaddr, XB0);
+        ld_frag8(own0 ? xbB + 32 * (8 * gm + t) : zaddr, XA1);
+        ld_frag8(own1 ? xbB + 32 * (8 * gm + 4 + t) : zaddr, XB1);
+        const uint32_t qa0 = sub4(c0, 2 * gm), qa1 = sub4(c1, 2 * gm);
+        const uint32_t qb0 = sub4(c0, 2 * gm + 1), qb1 = sub4(c1, 2 * gm + 1);
+        const uint32_t sa0 = qa0 >> 10, sa1 = qa1 >> 10, sb0 = qb0 >> 10, sb1 = qb1 >> 10;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
+            const bool sh = m > 4;
+            const uint32_t a0 = (sh ? sa0 : qa0) & mk, a1 = (sh ? sa1 : qa1) & mk;
+            const uint32_t a2 = (sh ? sb0 : qb0) & mk, a3 = (sh ? sb1 : qb1) & mk;
+            mma16816(D[0][gm][m & 1], a0, a1, a2, a3, XA0[m], XB0[m]);
+            mma16816(D[1][gm][m & 1], a0, a1, a2, a3, XA1[m], XB1[m]);
+        }
+    }
+    auto h2pair = [](uint32_t bits) { return __half22float2(*reinterpret_cast<const __half2*>(&bits)); };
+    float cf0[2], cf1[2], S[2][4];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t sb = (k ? tbB : tbA) + h.ts + jj * (kStatFloats * 4);
+        cf0[k] = ldsf(sb + 4 * (kStatC + t)); cf1[k] = ldsf(sb + 4 * (kStatC + 4 + t));
+        const uint4 Su = lds128(sb + 4 * (kStatS16 + 4 * t));
+        S[k][0] = __uint_as_float(Su.x); S[k][1] = __uint_as_float(Su.y);
+        S[k][2] = __uint_as_float(Su.z); S[k][3] = __uint_as_float(Su.w);
+    }
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) {
+        const int rec = rbase + 8 * hl;
+        const float d = h2f(lds16(st + w0 + rec * 2)) * 16777216.0f;
+        const float dm = h2f(lds16(st + w1 + rec * 2)) * 1048576.0f;   // m sits 4 bits up: 2^-20
+        const uint32_t f = lds32(st + w2 + rec * 16 + 4 * t);
+        const uint32_t fo = __byte_perm(f, 0u, 0x7371u);
+        const float2 s02 = h2pair(f & 0x000F000Fu), s13 = h2pair(fo & 0x000F000Fu);
+        const float2 m02 = h2pair(f & 0x00F000F0u), m13 = h2pair(fo & 0x00F000F0u);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            float Dk[2][2];
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm)
+#pragma unroll
+                for (int cc = 0; cc < 2; ++cc) Dk[gm][cc] = D[k][gm][0][2 * hl + cc] + D[k][gm][1][2 * hl + cc];
+            const float a0 = fmaf(s13.x, Dk[0][1], s02.x * Dk[0][0]);
+            const float a1 = fmaf(s13.y, Dk[1][1], s02.y * Dk[1][0]);
+            const float am = fmaf(m13.y, S[k][3], fmaf(m02.y, S[k][2], fmaf(m13.x, S[k][1], m02.x * S[k][0])));
+            const float v = fmaf(d, fmaf(cf1[k], a1, cf0[k] * a0), -dm * am);
+            acc[k][hl] += v;
+        }
+    }
+}
+
+// Q3_K, as tile_pair_q2k: code q = low2 + 4 hbit, the low bits through the
+// Q2_K MMAs, the high bits through MMAs of their own against the token's
+// operand scaled by 4 * 2^(pos(m) - m) (as tile_mma<kQ3K, 1>); the 6-bit
+// scales (stored + 32) are widened once for both tokens (as tile_epi).
+__device__ __forceinline__ void tile_pair_q3k(const Geo& h, uint32_t st, int jj, int rt, int tk0, uint32_t zaddr,
+                                              float (&acc)[2][2]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const bool own0 = g == t, own1 = g == t + 4;
+    const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
+    const uint32_t tbA = st + h.tok0 + tk0 * h.tstride, tbB = tbA + h.tstride;
+    const uint32_t xbA = tbA + h.tx + jj * 512, xbB = tbB + h.tx + jj * 512;
+    const int rbase = jj * 32 + 16 * rt + g;
+    const uint4 c0 = lds128(st + w2 + rbase * 64 + 16 * t), c1 = lds128(st + w2 + (rbase + 8) * 64 + 16 * t);
+    const uint2 hv0 = lds64(st + w3 + rbase * 32 + 8 * t), hv1 = lds64(st + w3 + (rbase + 8) * 32 + 8 * t);
+    float D[2][2][2][4];   // [token][sub-block group][pair parity][D fragment]
+#pragma unroll
+    for (int i = 0; i < 32; ++i) (&D[0][0][0][0])[i] = 0.0f;
+    // one sub-block group at a time (each accumulator sees its MMAs in the
+    // order of tile_mma<kQ3K, 1>: the low-bit pairs, then the high bits)
+#pragma unroll
+    for (int gm = 0; gm < 2; ++gm) {
+        uint32_t XA[2][8], XB[2][8];   // [token][pair]
+        ld_frag8(own0 ? xbA + 32 * (8 * gm + t) : zaddr, XA[0]);
+        ld_frag8(own1 ? xbA + 32 * (8 * gm + 4 + t) : zaddr, XB[0]);
+        ld_frag8(own0 ? xbB + 32 * (8 * gm + t) : zaddr, XA[1]);
+        ld_frag8(own1 ? xbB + 32 * (8 * gm + 4 + t) : zaddr, XB[1]);
+        const uint32_t qa0 = sub4(c0, 2 * gm), qa1 = sub4(c1, 2 * gm);
+        const uint32_t qb0 = sub4(c0, 2 * gm + 1), qb1 = sub4(c1, 2 * gm + 1);
+        const uint32_t sa0 = qa0 >> 10, sa1 = qa1 >> 10, sb0 = qb0 >> 10, sb1 = qb1 >> 10;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const uint32_t mk = 0x00030003u << (m <= 4 ? 2 * m : 2 * (m - 5));
+            const bool sh = m > 4;
+            const uint32_t a0 = (sh ? sa0 : qa0) & mk, a1 = (sh ? sa1 : qa1) & mk;
+            const uint32_t a2 = (sh ? sb0 : qb0) & mk, a3 = (sh ? sb1 : qb1) & mk;
+            mma16816(D[0][gm][m & 1], a0, a1, a2, a3, XA[0][m], XB[0][m]);
+            mma16816(D[1][gm][m & 1], a0, a1, a2, a3, XA[1][m], XB[1][m]);
+        }
+        const uint32_t ha0 = gm ? hv0.y : hv0.x, ha1 = gm ? hv1.y : hv1.x;
+        const uint32_t hb0 = ha0 >> 8, hb1 = ha1 >> 8;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const uint32_t mh = 0x00010001u << m;
+            const int e = m <= 4 ? m + 2 : m - 8;
+            const uint32_t sc16 = (uint32_t)(15 + e) << 10;
+            const __half2 scl = __halves2half2(__ushort_as_half((unsigned short)sc16), __ushort_as_half((unsigned short)sc16));
+            const uint32_t a0 = ha0 & mh, a1 = ha1 & mh, a2 = hb0 & mh, a3 = hb1 & mh;
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const __half2 xa = __hmul2(*reinterpret_cast<const __half2*>(&XA[k][m]), scl);
+                const __half2 xb2 = __hmul2(*reinterpret_cast<const __half2*>(&XB[k][m]), scl);
+                mma16816(D[k][gm][(m + 1) & 1], a0, a1, a2, a3, *reinterpret_cast<const uint32_t*>(&xa),
+                         *reinterpret_cast<const uint32_t*>(&xb2));
+            }
+        }
+    }
+    float cf0[2], cf1[2], S[2][4];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t sb = (k ? tbB : tbA) + h.ts + jj * (kStatFloats * 4);
+        cf0[k] = ldsf(sb + 4 * (kStatC + t)); cf1[k] = ldsf(sb + 4 * (kStatC + 4 + t));
+        const uint4 Su = lds128(sb + 4 * (kStatS16 + 4 * t));
+        S[k][0] = __uint_as_float(Su.x); S[k][1] = __uint_as_float(Su.y);
+        S[k][2] = __uint_as_float(Su.z); S[k][3] = __uint_as_float(Su.w);
+    }
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) {
+        const int rec = rbase + 8 * hl;
+        const float d = h2f(lds16(st + w0 + rec * 2)) * 16777216.0f;
+        const uint32_t sp = st + w1 + rec * 12;
+        const uint32_t lo = lds16(sp + 2 * t), hi = lds8(sp + 8 + t);
+        const uint32_t u = __byte_perm(lo, 0u, 0x7170u);
+        const uint32_t v = __byte_perm(hi, 0u, 0x7070u);
+        const __half2 c32 = __halves2half2(__ushort_as_half((unsigned short)32), __ushort_as_half((unsigned short)32));
+        const uint32_t uA = u & 0x000F000Fu, uB = (u >> 4) & 0x000F000Fu;
+        const __half2 lA = *reinterpret_cast<const __half2*>(&uA);
+        const __half2 lB = *reinterpret_cast<const __half2*>(&uB);
+        const uint32_t hA = v & 0x00300003u, hB = v & 0x00C0000Cu;
+        const __half2 mA = __halves2half2(__float2half(16.0f), __float2half(1.0f));
+        const __half2 mB = __halves2half2(__float2half(4.0f), __float2half(0.25f));
+        const __half2 sA = __hsub2(__hfma2(*reinterpret_cast<const __half2*>(&hA), mA, lA), c32);
+        const __half2 sB = __hsub2(__hfma2(*reinterpret_cast<const __half2*>(&hB), mB, lB), c32);
+        const float2 vA = __half22float2(sA), vB = __half22float2(sB);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            float Dk[2][2];
+#pragma unroll
+            for (int gm = 0; gm < 2; ++gm)
+#pragma unroll
+                for (int cc = 0; cc < 2; ++cc) Dk[gm][cc] = D[k][gm][0][2 * hl + cc] + D[k][gm][1][2 * hl + cc];
+            const float P0 = fmaf(Dk[0][0], cf0[k], -4.0f * S[k][0]), P1 = fmaf(Dk[0][1], cf0[k], -4.0f * S[k][1]);
+            const float P2 = fmaf(Dk[1][0], cf1[k], -4.0f * S[k][2]), P3 = fmaf(Dk[1][1], cf1[k], -4.0f * S[k][3]);
+            const float a = fmaf(vB.y, P3, fmaf(vA.y, P2, fmaf(vB.x, P1, vA.x * P0)));
+            acc[k][hl] = fmaf(d, a, acc[k][hl]);
+        }
+    }
+}
+
+// Q4_K, as tile_pair_q2k (tile_mma<kQ4K, 1> and tile_epi<kQ4K, 1> per token).
+__device__ __forceinline__ void tile_pair_q4k(const Geo& h, uint32_t st, int jj, int rt, int tk0, uint32_t zaddr,
+                                              float (&acc)[2][2]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const bool own0 = g == t, own1 = g == t + 4;
+    const int w0 = h.woff[0], w1 = h.woff[1], w2 = h.woff[2], w3 = h.woff[3];
+    const uint32_t tbA = st + h.tok0 + tk0 * h.tstride, tbB = tbA + h.tstride;
+    const uint32_t xbA = tbA + h.tx + jj * 512, xbB = tbB + h.tx + jj * 512;
+    const int rbase = jj * 32 + 16 * rt + g;
+    const int r0 = rbase - jj * 32, r1 = r0 + 8;
+    const uint4 cA0 = lds128(st + w3 + ((jj * 2 + 0) * 32 + r0) * 64 + 16 * t);
+    const uint4 cA1 = lds128(st + w3 + ((jj * 2 + 0) * 32 + r1) * 64 + 16 * t);
+    const uint4 cB0 = lds128(st + w3 + ((jj * 2 + 1) * 32 + r0) * 64 + 16 * t);
+    const uint4 cB1 = lds128(st + w3 + ((jj * 2 + 1) * 32 + r1) * 64 + 16 * t);
+    float D[2][2][2][4];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) (&D[0][0][0][0])[i] = 0.0f;
+    // one half of the pairs at a time (accumulator D[.][hm][.] takes only hm's)
+#pragma unroll
+    for (int hm = 0; hm < 2; ++hm) {
+        uint32_t XA[2][8], XB[2][8];   // [token][pair]
+        ld_frag8(own0 ? xbA + 64 * t + 32 * hm : zaddr, XA[0]);
+        ld_frag8(own1 ? xbA + 64 * (t + 4) + 32 * hm : zaddr, XB[0]);
+        ld_frag8(own0 ? xbB + 64 * t + 32 * hm : zaddr, XA[1]);
+        ld_frag8(own1 ? xbB + 64 * (t + 4) + 32 * hm : zaddr, XB[1]);
+#pragma unroll
+        for (int mm = 0; mm < 8; ++mm) {
+            const int m = 8 * hm + mm, wi = m >> 2, j = m & 3;
+            const uint32_t mk = (j & 1) ? 0x00F000F0u : 0x000F000Fu;
+            const int sh = j < 2 ? 0 : 8;
+            const uint32_t a0 = (sub4(cA0, wi) >> sh) & mk, a1 = (sub4(cA1, wi) >> sh) & mk;
+            const uint32_t a2 = (sub4(cB0, wi) >> sh) & mk, a3 = (sub4(cB1, wi) >> sh) & mk;
+            mma16816(D[0][hm][mm & 1], a0, a1, a2, a3, XA[0][mm], XB[0][mm]);
+            mma16816(D[1][hm][mm & 1], a0, a1, a2, a3, XA[1][mm], XB[1][mm]);
+        }
+    }
+    float cf0[2], cf1[2], S0[2], S1[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t sb = (k ? tbB : tbA) + h.ts + jj * (kStatFloats * 4);
+        const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
+        cf0[k] = __uint_as_float(Cu.x); cf1[k] = __uint_as_float(Cu.y);
+        S0[k] = __uint_as_float(Su.x); S1[k] = __uint_as_float(Su.y);
+    }
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) {
+        const int rec = rbase + 8 * hl;
+        const float d = h2f(lds16(st + w0 + rec * 2));
+        const float dm = h2f(lds16(st + w1 + rec * 2));
+        const uint32_t sp = st + w2 + rec * 12;
+        const uint32_t f = lds16(sp + 2 * t), hi = lds8(sp + 8 + t);
+        const float sc0 = (float)((f & 15u) | ((hi & 3u) << 4));
+        const float m0 = (float)(((f >> 4) & 15u) | (((hi >> 2) & 3u) << 4));
+        const float sc1 = (float)(((f >> 8) & 15u) | (((hi >> 4) & 3u) << 4));
+        const float m1 = (float)(((f >> 12) & 15u) | (((hi >> 6) & 3u) << 4));
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const float D0 = (D[k][0][0][2 * hl] + D[k][0][1][2 * hl]) + (D[k][1][0][2 * hl] + D[k][1][1][2 * hl]);
+            const float D1 = (D[k][0][0][2 * hl + 1] + D[k][0][1][2 * hl + 1]) +
+                             (D[k][1][0][2 * hl + 1] + D[k][1][1][2 * hl + 1]);
+            const float a_sc = fmaf(sc1 * cf1[k], D1, sc0 * cf0[k] * D0);
+            const float a_m = fmaf(m1, S1[k], m0 * S0[k]);
+            const float v = fmaf(d, a_sc, -dm * a_m);
+            acc[k][hl] += v;
+        }
+    }
+}
+
+// Q8_0, as tile_pair_q2k: one half of each superblock's code pairs
+// (tile_mma<kQ80, 1> and tile_epi<kQ80, 1> per token).
+__device__ __forceinline__ void tile_pair_q80(const Geo& h, uint32_t st, int jj, int half, int rt, int tk0,
+                                              uint32_t zaddr, float (&acc)[2][2]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const bool own0 = g == t, own1 = g == t + 4;
+    const int w0 = h.woff[0], w1 = h.woff[1];
+    const uint32_t tbA = st + h.tok0 + tk0 * h.tstride, tbB = tbA + h.tstride;
+    const uint32_t xbA = tbA + h.tx + jj * 512, xbB = tbB + h.tx + jj * 512;
+    const int rbase = jj * 32 + 16 * rt + g;
+    const int r0 = rbase - jj * 32, r1 = r0 + 8;
+    const uint4 cA0 = lds128(st + w1 + ((8 * jj + t) * 32 + r0) * 32 + 16 * half);
+    const uint4 cA1 = lds128(st + w1 + ((8 * jj + t) * 32 + r1) * 32 + 16 * half);
+    const uint4 cB0 = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r0) * 32 + 16 * half);
+    const uint4 cB1 = lds128(st + w1 + ((8 * jj + t + 4) * 32 + r1) * 32 + 16 * half);
+    float D[2][2][2][4];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) (&D[0][0][0][0])[i] = 0.0f;
+    uint32_t XA[2][8], XB[2][8];   // [token][pair]
+    ld_frag8(own0 ? xbA + 64 * t + 32 * half : zaddr, XA[0]);
+    ld_frag8(own1 ? xbA + 64 * (t + 4) + 32 * half : zaddr, XB[0]);
+    ld_frag8(own0 ? xbB + 64 * t + 32 * half : zaddr, XA[1]);
+    ld_frag8(own1 ? xbB + 64 * (t + 4) + 32 * half : zaddr, XB[1]);
+#pragma unroll
+    for (int mm = 0; mm < 8; ++mm) {
+        const int wi = mm >> 1, sh = (mm & 1) ? 8 : 0, a = mm & 3;
+        const uint32_t a0 = (sub4(cA0, wi) >> sh) & 0x00FF00FFu, a1 = (sub4(cA1, wi) >> sh) & 0x00FF00FFu;
+        const uint32_t a2 = (sub4(cB0, wi) >> sh) & 0x00FF00FFu, a3 = (sub4(cB1, wi) >> sh) & 0x00FF00FFu;
+        mma16816(D[0][a >> 1][a & 1], a0, a1, a2, a3, XA[0][mm], XB[0][mm]);
+        mma16816(D[1][a >> 1][a & 1], a0, a1, a2, a3, XA[1][mm], XB[1][mm]);
+    }
+    float cf0[2], cf1[2], o0[2], o1[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t sb = (k ? tbB : tbA) + h.ts + jj * (kStatFloats * 4);
+        const uint2 Cu = lds64(sb + 4 * (kStatC + 2 * t)), Su = lds64(sb + 4 * (kStatS32 + 2 * t));
+        cf0[k] = __uint_as_float(Cu.x); cf1[k] = __uint_as_float(Cu.y);
+        o0[k] = half ? 0.0f : 128.0f * __uint_as_float(Su.x);
+        o1[k] = half ? 0.0f : 128.0f * __uint_as_float(Su.y);
+    }
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) {
+        const int r = (rbase + 8 * hl) - jj * 32;
+        const float d0 = h2f(lds16(st + w0 + ((8 * jj + 2 * t) * 32 + r) * 2));
+        const float d1 = h2f(lds16(st + w0 + ((8 * jj + 2 * t + 1) * 32 + r) * 2));
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const float D0 = (D[k][0][0][2 * hl] + D[k][0][1][2 * hl]) + (D[k][1][0][2 * hl] + D[k][1][1][2 * hl]);
+            const float D1 = (D[k][0][0][2 * hl + 1] + D[k][0][1][2 * hl + 1]) +
+                             (D[k][1][0][2 * hl + 1] + D[k][1][1][2 * hl + 1]);
+            const float v = fmaf(d1, fmaf(D1, cf1[k], -o1[k]), d0 * fmaf(D0, cf0[k], -o0[k]));
+            acc[k][hl] += v;
+        }
+    }
+}
+
 // The warp's superblocks col, col + kCols, ... of a stage, one tile at a time.
 template <int FMT>
 __device__ __forceinline__ void tile_cols(const Geo& h, uint32_t st, int col, int ks, int rt0, int tk,
@@ -1109,9 +1405,48 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 #pragma unroll
                     for (int i = 0; i < 4; ++i) { acc[0][tk][i] += cur[tk][i]; cur[tk][i] = 0.0f; }
             }
+            // Items of several tokens: Q2_K / Q3_K / Q4_K / Q8_0 tiles take the
+            // tokens two at a time (the code operands built once for both, per
+            // 16-row tile); sums equal to the per-token passes
+            constexpr bool kPairs = MT > 1 && kNT == 2;
+            const bool pairs = kPairs && (fmt == kQ2K || fmt == kQ3K || fmt == kQ4K || fmt == kQ80);
 #pragma unroll
             for (int tk = 0; tk < MT; ++tk) {
                 if (tk >= ntok) break;
+                if constexpr (kPairs) {
+                    if (pairs && (tk & 1)) continue;   // done with tk - 1
+                    if (pairs && tk + 1 < ntok) {
+                        for (int jj = wcol; jj < ks; jj += kCols) {
+#pragma unroll 1
+                            for (int rt = 0; rt < 2; ++rt) {
+                                // this row tile's sums of the two tokens (indices fixed at compile
+                                // time on this side, so the sums stay in registers)
+                                float a[2][2];
+#pragma unroll
+                                for (int hl = 0; hl < 2; ++hl) {
+                                    a[0][hl] = rt ? cur[tk][2 + hl] : cur[tk][hl];
+                                    a[1][hl] = rt ? cur[(tk + 1) % MT][2 + hl] : cur[(tk + 1) % MT][hl];
+                                }
+                                if (fmt == kQ80) {
+                                    tile_pair_q80(GS, stage, jj, 0, rt, tk, zaddr, a);
+                                    tile_pair_q80(GS, stage, jj, 1, rt, tk, zaddr, a);
+                                } else if (fmt == kQ2K) {
+                                    tile_pair_q2k(GS, stage, jj, rt, tk, zaddr, a);
+                                } else if (fmt == kQ3K) {
+                                    tile_pair_q3k(GS, stage, jj, rt, tk, zaddr, a);
+                                } else {
+                                    tile_pair_q4k(GS, stage, jj, rt, tk, zaddr, a);
+                                }
+#pragma unroll
+                                for (int hl = 0; hl < 2; ++hl) {
+                                    if (rt) { cur[tk][2 + hl] = a[0][hl]; cur[(tk + 1) % MT][2 + hl] = a[1][hl]; }
+                                    else { cur[tk][hl] = a[0][hl]; cur[(tk + 1) % MT][hl] = a[1][hl]; }
+                                }
+                            }
+                        }
+                        continue;
+                    }
+                }
                 if (fmt == kQ80) {
                     for (int jj = wcol; jj < ks; jj += kCols) {   // both halves of each superblock's code pairs
                         TileAcc<kNT> T0, T1;
