@@ -257,7 +257,7 @@ const char* mq_strerror(int status);
  * mma.sync kernels stream whole 256-element superblocks).  Process wide;
  * the MQ_FORCE_PATH environment variable ("decode"/"prefill"/"decode_tc")
  * sets the initial value.  threshold <= 0 keeps the current one (default
- * 40).  Returns MQ_EINVAL for another mode. */
+ * 50).  Returns MQ_EINVAL for another mode. */
 int mq_set_path(int mode, int32_t prefill_threshold);
 
 /* Test hook for the bounded waits (no counterpart in the paper).  Arms a

@@ -22,9 +22,9 @@ constexpr int32_t kFusedRouteTokens = 256;   // up to this many tokens: one rout
 
 int g_path_mode = -1;        // -1: not yet read from the environment
 // automatic path choice: the grouped GEMM from this many tokens on (on the
-// V3 layer with mixed formats it is the faster path from about 40 tokens:
-// 32 tokens 1.89 ms decode / 2.04 ms GEMM, 48 tokens 2.86 / 2.48 ms)
-int32_t g_prefill_threshold = 40;
+// V3 layer with mixed formats it is the faster path from about 50 tokens:
+// 48 tokens 2.46 ms decode / 2.50 ms GEMM, 56 tokens 2.83 / 2.64 ms)
+int32_t g_prefill_threshold = 50;
 
 int path_mode() {
     if (g_path_mode < 0) {
