@@ -164,6 +164,9 @@ constexpr int kRingBytes = 192 * 1024;
 constexpr int kSlotBytes = kRingBytes / kNST;
 constexpr int kStageSb = 16;                        // superblocks per stage (Q8_0: 8), fewer if over budget
 constexpr int kMaxCachedAssign = 1024;              // routed assignments cached in smem
+#ifndef MQ_SPLIT_SHARED
+#define MQ_SPLIT_SHARED 1
+#endif
 #ifndef MQ_PREROUTE_DEPTH
 #define MQ_PREROUTE_DEPTH 3
 #endif
@@ -1059,6 +1062,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     constexpr int kRedBufs = MT == 1 ? 2 : 1;          // item-end reduction buffers (smem budget)
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
+    __shared__ float s_wts[kMaxCachedAssign];   // routing weights by assignment (the first kMaxCachedAssign)
     __shared__ __align__(8) uint64_t bars[2 * kNST];
     __shared__ Hdr hdr[kNST];
     __shared__ float red[kRedBufs][kConsumers][2][MT][32];
@@ -1164,10 +1168,12 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             int e0 = __ldcg(&A.plan->slot_e[lane]), f0 = __ldcg(&A.plan->slot_first[lane]);
             int nt0 = __ldcg(&A.plan->slot_ntot[lane]);
             int pv0[4];
+            float wv0[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int i = 32 * u + lane;
                 pv0[u] = i < n_routed ? __ldcg(A.perm + i) : 0;
+                wv0[u] = i < n_routed ? __ldcg(A.wts + i) : 0.0f;
             }
             n_slots = ns0;
             for (int i = lane; i <= n_slots; i += 32) {
@@ -1193,19 +1199,21 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int i = 32 * u + lane;
-                if (i < n_routed) s_perm[i] = pv0[u];
+                if (i < n_routed) { s_perm[i] = pv0[u]; s_wts[i] = wv0[u]; }
             }
             for (int i0 = 128; i0 < n_routed; i0 += 128) {
                 int v[4];
+                float wv[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int i = i0 + 32 * u + lane;
                     v[u] = i < n_routed ? __ldcg(A.perm + i) : 0;
+                    wv[u] = i < n_routed ? __ldcg(A.wts + i) : 0.0f;
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int i = i0 + 32 * u + lane;
-                    if (i < n_routed) s_perm[i] = v[u];
+                    if (i < n_routed) { s_perm[i] = v[u]; s_wts[i] = wv[u]; }
                 }
             }
             __syncwarp();
@@ -1218,12 +1226,16 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
         // items are handed out by one counter (zeroed per call) in the order
         // above: the shared expert's gate/up items (Q8_0, the heaviest) first,
         // so the CTAs even out on the lighter routed items that follow
-        auto claim = [&]() -> int {
-            int v = 0;
-            if (lane == 0) v = (int)atomicAdd(A.next, 1u);
-            return __shfl_sync(kFull, v, 0);
+        // A claim is the atomic (lane 0) and, later, the broadcast of its
+        // result: nothing reads the result register before the broadcast, so
+        // the atomic's round trip runs while the stages are posted.
+        auto claim_issue = [&]() -> uint32_t {
+            uint32_t v = 0;
+            if (lane == 0) v = atomicAdd(A.next, 1u);
+            return v;
         };
-        int id_next = claim();
+        auto claim_take = [&](uint32_t v) -> int { return __shfl_sync(kFull, (int)v, 0); };
+        int id_next = claim_take(claim_issue());
         for (;;) {
             const int id = id_next;
             if (!routed && id >= n_sh_items) wait_routing();
@@ -1233,7 +1245,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             // after this item's stages are posted, so that the shared expert's
             // items spread over the CTAs instead of going two to a CTA
             const bool claim_early = routed || !A.split_shared;
-            if (item >= 0 && claim_early) id_next = claim();
+            const bool pending = item >= 0 && claim_early;
+            const uint32_t pend = pending ? claim_issue() : 0u;
             if (item >= 0) {
                 decode_item(A, sc, s_perm, n_slots, n_gu, item, cur_gu, cur_dn, P);
                 fmt0 = tab.fmt[P.e][P.down ? 2 : 0];
@@ -1365,7 +1378,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             if (failed) { if (lane == 0) { atomicOr(A.err, kErrEmpty); s_fail = 1; } break; }
             if (item < 0) break;
-            if (!claim_early) id_next = claim();
+            id_next = claim_take(pending ? pend : claim_issue());
         }
     } else {
         // ============================ consumer warps =============================
@@ -1544,9 +1557,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     A.pdn[(size_t)a * d.H + 32 * (e_rb + 1) + lane] = v1;
                 } else {
                     // SwiGLU (routing weight folded in), then prepare h for the down projection
-                    // routing weights: written by the logits kernel's routing CTA and
-                    // acquired by this CTA's producer before it posted the item
-                    const float w = e_shared ? 1.0f : __ldcg(A.wts + a);
+                    // routing weights: written by the logits kernel's routing CTA,
+                    // acquired by this CTA's producer before it posted the item and
+                    // cached in shared memory (the first kMaxCachedAssign entries)
+                    const float w = e_shared ? 1.0f : a < kMaxCachedAssign ? s_wts[a] : __ldcg(A.wts + a);
                     const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
                     const int fam = families_of(tab.fmt[e_e][2]);
                     __half* hq = A.hq + (size_t)a * kFamSlots * A.nsbi * 256;
@@ -1623,10 +1637,10 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.hready = w.counters + 1;
     A.scount = w.counters + 1 + (kMaxExperts + 1);
     A.spart = w.spart;
-    A.split_shared = d.T == 1 && d.has_shared && A.nsbx >= 2 ? 1 : 0;   // one token: the routing front
+    A.split_shared = MQ_SPLIT_SHARED && d.T == 1 && d.has_shared && A.nsbx >= 2 ? 1 : 0;   // one token: the routing front
     A.logits_done = w.logits_done;
     A.route_ready = w.route_ready;
-    A.n_logit_ctas = (uint32_t)(d.E * ((d.T + 7) / 8));   // the logits kernel's grid (experts x 8-token groups)
+    A.n_logit_ctas = router_logits_ctas(d);   // the logits kernel's grid
     A.err = w.err;
     A.wait_ns = 1000000000ull;
     A.fail_first_stage = 0;

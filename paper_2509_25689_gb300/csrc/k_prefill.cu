@@ -116,8 +116,8 @@ __device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
 //     eight per chunk parity) and, at the unit's end, run the epilogue out
 //     of tensor memory; the gate/up epilogue writes h straight into the down
 //     GEMM's activation layout;
-//   - an activation warp moves the chunk's activation rows with eight bulk
-//     copies from the tile-ordered copy of the tokens (xperm_kernel) or of h;
+//   - an activation warp moves the chunk's activation rows with one bulk
+//     copy from the tile-ordered copy of the tokens (xperm_kernel) or of h;
 //   - an MMA warp issues a chunk's MMAs once the workers and the activation
 //     warp have filled its operand slot (a two-slot ring) and commits them
 //     to the slot's empty barrier.
@@ -143,8 +143,9 @@ __host__ __device__ constexpr int g_smem(bool down) { return g_ops(down) * g_slo
 // T*K + t for the shared expert), cut into tiles of up to kGNT rows of one
 // slot.  In a tile of N rows starting at position r0, the 16-byte piece p
 // (columns 8p .. 8p+7) of row n sits (p * N + n) * 16 bytes after r0 * K * 2,
-// so a 64-column chunk of a tile is eight contiguous runs of N x 16 bytes:
-// one bulk copy each into the canonical operand layout.
+// so a 64-column chunk of a tile is one contiguous run of 8 x N x 16 bytes:
+// one bulk copy into the canonical operand layout whose core matrices are
+// N x 16 bytes apart along K.
 __device__ __forceinline__ size_t perm_piece(int r0, int K, int N, int p, int n) {
     return (size_t)r0 * K * 2 + ((size_t)p * N + n) * 16;
 }
@@ -657,10 +658,11 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
         // the stages still in flight land before the CTA exits
         for (int q = max(0, pq - kGPk); q < pq; ++q) (void)mbar_wait(pkf + 8 * (q % kGPk), (q / kGPk) & 1);
     } else if (warp == kWarpB) {
-        // ---- activations: the chunk's rows of the unit's tile, eight bulk copies
-        // (one per 8-column piece) into the operand slot; the MMA may read rows
-        // N .. Npad - 1 of an earlier chunk: they only reach accumulator
-        // columns the epilogue never reads
+        // ---- activations: the chunk's rows of the unit's tile, one bulk copy
+        // (its eight 8-column pieces are contiguous in the tile-ordered copy)
+        // into the operand slot; the MMA reads rows N .. Npad - 1 of a piece
+        // from the next piece or past the copied run: they only reach
+        // accumulator columns the epilogue never reads
         const uint8_t* src = kDown ? reinterpret_cast<const uint8_t*>(A.h16) : A.xp;
         int gq = 0;
         for (int ui = 0;; ++ui) {
@@ -673,30 +675,32 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
                 const int s = gq % kGOps;
                 if (gq >= kGOps && !mbar_wait(ope + 8 * s, ((gq - kGOps) / kGOps) & 1)) { bad = true; break; }
                 if (failed()) { bad = true; break; }
-                if (lane == 0) g_arrive_tx(opf + 8 * s, (uint32_t)(U.N * 128));
-                __syncwarp();
-                if (lane < 8)
+                // the chunk's eight pieces are one contiguous run of 8 N x 16
+                // bytes; the MMA's B descriptor steps N x 16 bytes per piece
+                if (lane == 0) {
+                    g_arrive_tx(opf + 8 * s, (uint32_t)(U.N * 128));
                     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                                 ::"r"(ring + s * kGSlotBytes + kBOfs + lane * kGNT * 16),
-                                   "l"(src + perm_piece(U.r0, K, U.N, c * 8 + lane, 0)), "r"((uint32_t)(U.N * 16)),
-                                   "r"(opf + 8 * s) : "memory");
+                                 ::"r"(ring + s * kGSlotBytes + kBOfs), "l"(src + perm_piece(U.r0, K, U.N, c * 8, 0)),
+                                   "r"((uint32_t)(U.N * 128)), "r"(opf + 8 * s) : "memory");
+                }
+                __syncwarp();
             }
             if (bad) { if (lane == 0) fail(); break; }
             __syncwarp();
             if (lane == 0) mbar_arrive(ue + 8 * us);
         }
     } else if (warp == kWarpM) {
-        // ---- MMA issue.  The operand descriptors of both slots are built once:
-        // a 16-column step of K moves an A operand by 2 * kMT * 16 bytes and B
-        // by 2 * kGNT * 16 bytes, i.e. the descriptors' start-address field
-        // (bytes / 16) by 256 and 512.
+        // ---- MMA issue.  The A descriptors of the slots are built once, B's
+        // per unit: B holds the chunk's eight pieces of N rows x 16 bytes one
+        // after the other (leading byte offset N x 16).  A 16-column step of K
+        // moves A by 2 * kMT * 16 bytes and B by 2 * N * 16 bytes, i.e. the
+        // descriptors' start-address field (bytes / 16) by 256 and 2 N.
         uint64_t dA[kGOpsMax][2], dB[kGOpsMax];
 #pragma unroll
         for (int sl2 = 0; sl2 < kGOpsMax; ++sl2) {
             const uint32_t sbase = ring + sl2 * kGSlotBytes;
             dA[sl2][0] = sdesc(sbase, kMT * 16, 128);
             dA[sl2][1] = sdesc(sbase + kABytes, kMT * 16, 128);
-            dB[sl2] = sdesc(sbase + kBOfs, kGNT * 16, 128);
         }
         int mq = 0, last = -1;
         for (int ui = 0;; ++ui) {
@@ -704,6 +708,10 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
             if (!mbar_wait(uf + 8 * us, (ui >> 1) & 1)) { if (lane == 0) fail(); break; }
             const GUnit U = s_unit[us];
             if (U.u < 0) break;
+#pragma unroll
+            for (int sl2 = 0; sl2 < kGOpsMax; ++sl2)
+                dB[sl2] = sdesc(ring + sl2 * kGSlotBytes + kBOfs, (uint32_t)U.N * 16u, 128);
+            const uint32_t bstep = 2u * (uint32_t)U.N;
             bool bad = false;
             for (int c = 0; c < nC; ++c, ++mq) {
                 const int s = mq % kGOps;
@@ -718,8 +726,8 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
 #pragma unroll
                     for (int kk = 0; kk < kKC / 16; ++kk) {
                         const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;
-                        mma_f16(tbase, a0 + 256u * kk, b0 + 512u * kk, idesc, acc);
-                        if (!kDown) mma_f16(tbase + kGNT, a1 + 256u * kk, b0 + 512u * kk, idesc, acc);
+                        mma_f16(tbase, a0 + 256u * kk, b0 + bstep * kk, idesc, acc);
+                        if (!kDown) mma_f16(tbase + kGNT, a1 + 256u * kk, b0 + bstep * kk, idesc, acc);
                     }
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
                                  ::"r"(ope + 8 * s) : "memory");

@@ -443,24 +443,44 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(int32_t* __restri
 }
 
 // ---------------------------------------------------------------------------
-// logits: grid (E, ceil(T / kTok)), one warp per 1024-element segment
+// logits: grid (ceil(E / epc), ceil(T / kTok)); a CTA holds epc experts, one
+// warp per (expert, 1024-element segment), so that at decode most SMs hold
+// no logits CTA and take the expert-FFN grid (which needs a whole SM's shared
+// memory) as soon as it launches.  Every expert's sum is formed in the same
+// canonical order whatever epc is.
 // ---------------------------------------------------------------------------
 constexpr int kTok = 8;
+#ifndef MQ_LOGITS_EPC
+#define MQ_LOGITS_EPC 1
+#endif
+constexpr int kLogitsEpc = MQ_LOGITS_EPC;   // experts per logits CTA (fewer if the warps would exceed 32)
+
+__host__ __device__ __forceinline__ int logits_nseg(int H) { return (H / 128 + 7) / 8; }
+__host__ __device__ __forceinline__ int logits_epc(int H) {
+    const int nseg = logits_nseg(H);
+    const int e = 32 / (nseg > 0 ? nseg : 1);
+    return e < 1 ? 1 : (e > kLogitsEpc ? kLogitsEpc : e);
+}
 
 __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __restrict__ x,
                                                              const float* __restrict__ W, int H, int T,
                                                              int E, float* __restrict__ z,
                                                              __half* __restrict__ xq, float* __restrict__ xs,
                                                              __half* __restrict__ x16, int32_t* __restrict__ xe,
-                                                             int x_fams, const FusedRoute fr) {
+                                                             int x_fams, int epc, const FusedRoute fr) {
     __shared__ float part[32][kTok];
-    __shared__ float pmax[32][kTok];   // per segment: largest |x| of each token (prefill copy only)
+    __shared__ float pmax[32][kTok];   // per warp: largest |x| of each token (prefill copy only)
     __shared__ int s_last;
-    const int e = blockIdx.x, t0 = blockIdx.y * kTok;
-    const int seg = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t0 = blockIdx.y * kTok;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nchunk = H >> 7, nseg = (nchunk + 7) >> 3;
-    const int c0 = seg * 8, nc = min(8, nchunk - c0);
-    const float* wrow = W + (size_t)e * H;
+    // warp -> (local expert le, segment seg); warps past epc experts (the
+    // routing CTA's extra warps) and experts past E take no segment
+    const int le = warp / nseg, seg = warp - le * nseg;
+    const int e = blockIdx.x * epc + le;
+    const bool work = le < epc && e < E;
+    const int c0 = seg * 8, nc = work ? min(8, nchunk - c0) : 0;
+    const float* wrow = W + (size_t)(work ? e : 0) * H;
     // The router weights are an input no kernel of this library writes, so
     // their loads go out before the wait for the previous kernel (which may
     // be the previous layer's combine, writing this call's x).
@@ -508,15 +528,17 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     }
     if (lane == 0) {
 #pragma unroll
-        for (int j = 0; j < kTok; ++j) { part[seg][j] = acc[j]; pmax[seg][j] = amx[j]; }
+        for (int j = 0; j < kTok; ++j) { part[warp][j] = acc[j]; pmax[warp][j] = amx[j]; }
     }
     __syncthreads();
-    if (threadIdx.x < kTok) {
-        const int t = t0 + threadIdx.x;
-        if (t < T) {
-            float r = part[0][threadIdx.x];
-            for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[s][threadIdx.x]);
-            z[(size_t)t * E + e] = r;
+    // z: per (local expert, token), the expert's segments left to right
+    if (threadIdx.x < epc * kTok) {
+        const int l2 = threadIdx.x / kTok, j = threadIdx.x - l2 * kTok;
+        const int e2 = blockIdx.x * epc + l2, t = t0 + j;
+        if (e2 < E && t < T) {
+            float r = part[l2 * nseg][j];
+            for (int s = 1; s < nseg; ++s) r = __fadd_rn(r, part[l2 * nseg + s][j]);
+            z[(size_t)t * E + e2] = r;
         }
     }
     // fp16 copy of the tokens for the prefill GEMM (each token scaled by its
@@ -525,11 +547,12 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
         for (int j = 0; j < kTok; ++j) {
             const int t = t0 + j;
             if (t >= T) break;
+            // the CTA's first expert's warps saw the whole token
             float m = pmax[0][j];
             for (int s = 1; s < nseg; ++s) m = fmaxf(m, pmax[s][j]);
             const int ex = token_exp(m);
-            if (e == 0 && threadIdx.x == 0) xe[t] = ex;
-            for (int k = e * blockDim.x + threadIdx.x; k < H; k += E * blockDim.x)
+            if (blockIdx.x == 0 && threadIdx.x == 0) xe[t] = ex;
+            for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < H; k += gridDim.x * blockDim.x)
                 x16[(size_t)t * H + k] = __float2half_rn(ldexpf(bf16_lo(x[(size_t)t * H + k]), -ex));
         }
     }
@@ -537,7 +560,7 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     // kernels, spread over all of them: warp `seg` of the CTA of expert e
     // takes the 32-element blocks 32*seg + e, 32*seg + e + E, ... of its
     // segment (blocks past the hidden size, up to the 256 padding, are zero).
-    if (xq != nullptr) {
+    if (xq != nullptr && work) {
         const int nsb = (H + 255) / 256;
         const size_t qstride = (size_t)kFamSlots * nsb * 256, sstride = (size_t)nsb * kStatFloats;
         for (int j = 0; j < kTok; ++j) {
@@ -587,6 +610,11 @@ cudaError_t launch_zero(uint32_t* words, int n, cudaStream_t s) {
     return e;
 }
 
+uint32_t router_logits_ctas(const Dims& d) {
+    const int epc = logits_epc(d.H);
+    return (uint32_t)(((d.E + epc - 1) / epc) * ((d.T + kTok - 1) / kTok));
+}
+
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
                                  __half* x16, int32_t* xe, const FusedRoute* fused, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
@@ -599,19 +627,20 @@ cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* 
         dim3 grid((d.E + kEB - 1) / kEB, (d.T + kTokT - 1) / kTokT);
         e = launch_pdl(router_logits_tile_kernel, grid, dim3(nseg * 32), 0, s, x, W, d.H, d.T, d.E, z, x16, xe);
     } else {
-        dim3 grid(d.E, (d.T + kTok - 1) / kTok);
+        const int epc = logits_epc(d.H);
+        dim3 grid((d.E + epc - 1) / epc, (d.T + kTok - 1) / kTok);
         FusedRoute fr{};
-        int threads = nseg * 32;
+        int warps = epc * nseg;
         size_t smem = 0;
         if (fused != nullptr) {
             fr = *fused;
             fr.on = 1;
             fr.n_ctas = grid.x * grid.y;
-            threads = (nseg > kPermWarps ? nseg : kPermWarps) * 32;   // the last CTA routes with kPermWarps warps
+            if (warps < kPermWarps) warps = kPermWarps;   // the last CTA routes with kPermWarps warps
             smem = sizeof(PermSmem);
         }
-        e = launch_pdl(router_logits_kernel, grid, dim3(threads), smem, s, x, W, d.H, d.T, d.E, z, xq, xs, x16, xe,
-                       d.x_fams, fr);
+        e = launch_pdl(router_logits_kernel, grid, dim3(warps * 32), smem, s, x, W, d.H, d.T, d.E, z, xq, xs, x16,
+                       xe, d.x_fams, epc, fr);
     }
     prof_end(s);
     return e;

@@ -143,9 +143,11 @@ struct FusedRoute {
 // stream is done; the first kernel of every forward call.
 cudaError_t launch_zero(uint32_t* words, int n, cudaStream_t s);
 // fused: nullptr, or the routing outputs for the fused last-CTA routing
-// (one CTA per expert x 8 tokens; the logits kernel with activation prep)
+// (the logits kernel with activation prep; router_logits_ctas(d) CTAs, each
+// up to 4 experts x 8 tokens)
 cudaError_t launch_router_logits(const Dims& d, const uint16_t* x, const float* W, float* z, __half* xq, float* xs,
                                  __half* x16, int32_t* xe, const FusedRoute* fused, cudaStream_t s);
+uint32_t router_logits_ctas(const Dims& d);
 cudaError_t launch_topk(const Dims& d, const float* z, const float* bias, int32_t* idx, float* wts, cudaStream_t s);
 cudaError_t launch_permute(const Dims& d, const int32_t* idx, int32_t* offsets, int32_t* perm, int32_t* inv,
                            int32_t* active, Plan* plan, cudaStream_t s);

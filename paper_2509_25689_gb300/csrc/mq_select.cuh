@@ -198,11 +198,25 @@ __device__ __forceinline__ void route_token_compact(const float* __restrict__ z,
     const int gs = E / G;
     float* u_sh = sc;
     float* s_sh = sc + 256;
+    // the token's logits (E <= 256: at most 8 per lane) as one batch of
+    // independent loads, then the scores in a rolled loop (small code)
+    float zv[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        const int e = lane + 32 * m;
+        zv[m] = e < E ? __ldcg(z + (size_t)t * E + e) : 0.0f;
+    }
 #pragma unroll 1
-    for (int e = lane; e < E; e += 32) {
-        const float sv = canonical_sigmoid(__ldcg(z + (size_t)t * E + e));
-        s_sh[e] = sv;
-        u_sh[e] = __fadd_rn(sv, bias ? bias[e] : 0.0f);
+    for (int m = 0; 32 * m < E; ++m) {
+        const int e = lane + 32 * m;
+        float zm = zv[0];
+#pragma unroll
+        for (int q = 1; q < 8; ++q) zm = q == m ? zv[q] : zm;
+        if (e < E) {
+            const float sv = canonical_sigmoid(zm);
+            s_sh[e] = sv;
+            u_sh[e] = __fadd_rn(sv, bias ? bias[e] : 0.0f);
+        }
     }
     __syncwarp();
     // group score = sum of the two largest u of the group (as route_token)
