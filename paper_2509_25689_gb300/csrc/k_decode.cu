@@ -183,6 +183,11 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
 __device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+__device__ __forceinline__ uint32_t atom_acq_rel_add(uint32_t* p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
 
 // stage header written by the producer (one per ring slot); the stage's
 // byte layout is geo[down][fmt - 1][ntok - 1]
@@ -1538,14 +1543,17 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     float* sp = A.spart + (size_t)t * 4 * d.I;
                     sp[(2 * e_half + 0) * d.I + 32 * e_rb + lane] = v0;
                     sp[(2 * e_half + 1) * d.I + 32 * e_rb + lane] = v1;
-                    __threadfence();
+                    // the warp barrier orders every lane's stores before lane 0's
+                    // acquire-release count, which publishes them and, in the
+                    // half that counts second, acquires the other half's; the
+                    // second barrier orders that acquire before every lane's loads
                     __syncwarp();
                     uint32_t before = 0;
-                    if (lane == 0) before = atomicAdd(A.scount + (size_t)t * (d.I / 32) + e_rb, 1u);
+                    if (lane == 0) before = atom_acq_rel_add(A.scount + (size_t)t * (d.I / 32) + e_rb, 1u);
                     before = __shfl_sync(kFull, before, 0);
+                    __syncwarp();
                     finish = before == 1u;
                     if (finish) {
-                        __threadfence();
                         const int o = 1 - e_half;
                         v0 += __ldcg(sp + (2 * o + 0) * d.I + 32 * e_rb + lane);
                         v1 += __ldcg(sp + (2 * o + 1) * d.I + 32 * e_rb + lane);
@@ -1569,9 +1577,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     const int n_rb = d.I / 32;
                     if (e_rb == n_rb - 1)
                         for (int jb = n_rb; jb < 8 * A.nsbi; ++jb) prep_block32(0.0f, jb, fam, hq, hs, A.nsbi);
-                    // publish the block: every lane's writes, then one release add
-                    // on the slot's counter (down items of the slot wait for it)
-                    __threadfence();
+                    // publish the block: the warp barrier orders every lane's
+                    // writes before lane 0's release add on the slot's counter
+                    // (down items of the slot acquire it)
                     __syncwarp();
                     if (lane == 0) red_release_add(A.hready + e_slot, 1u);
                 }

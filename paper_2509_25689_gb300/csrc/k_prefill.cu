@@ -126,15 +126,27 @@ __device__ __forceinline__ float silu(float v) { return v / (1.0f + expf(-v)); }
 // the producer, activation and MMA warps
 __host__ __device__ constexpr int g_workers(bool down) { return 16; }
 __host__ __device__ constexpr int g_threads(bool down) { return (g_workers(down) + 3) * 32; }
-constexpr int kGNT = 256;                      // tokens per unit (MMA N up to 256)
+#ifndef MQ_GNT
+#define MQ_GNT 256
+#endif
+#ifndef MQ_GOPS_GU
+#define MQ_GOPS_GU 2
+#endif
+#ifndef MQ_GOPS_DN
+#define MQ_GOPS_DN 3
+#endif
+#ifndef MQ_GPK
+#define MQ_GPK 2
+#endif
+constexpr int kGNT = MQ_GNT;                   // tokens per unit (MMA N up to 256)
 // operand slots: gate/up two of A gate | A up | B (64 KB), down three of
 // A | B (48 KB); a third gate/up slot fits only with 128-token units,
 // measured slower on the Zipf prefill
-__host__ __device__ constexpr int g_ops(bool down) { return down ? 3 : 2; }
+__host__ __device__ constexpr int g_ops(bool down) { return down ? MQ_GOPS_DN : MQ_GOPS_GU; }
 __host__ __device__ constexpr int g_bofs(bool down) { return down ? kABytes : 2 * kABytes; }
 __host__ __device__ constexpr int g_slot(bool down) { return g_bofs(down) + kGNT * kKC * 2; }
-constexpr int kGOpsMax = 3;
-constexpr int kGPk = 2;                        // packed-record stages
+constexpr int kGOpsMax = MQ_GOPS_GU > MQ_GOPS_DN ? MQ_GOPS_GU : MQ_GOPS_DN;
+constexpr int kGPk = MQ_GPK;                   // packed-record stages
 constexpr int kGPkBytes = 37376;               // Q6_K + Q6_K half superblock of 128 rows: 2 x 18,688
 __host__ __device__ constexpr int g_smem(bool down) { return g_ops(down) * g_slot(down) + kGPk * kGPkBytes; }
 
@@ -720,9 +732,10 @@ __global__ void __launch_bounds__(g_threads(kDown), 1) gemm_ws_kernel(const __gr
                     // (the workers fenced their operand stores; the activations came by bulk copy)
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint32_t idesc = idesc_f16(kMT, U.Npad);
-                    const uint64_t a0 = s == 0 ? dA[0][0] : s == 1 ? dA[1][0] : dA[2][0];
-                    const uint64_t a1 = s == 0 ? dA[0][1] : s == 1 ? dA[1][1] : dA[2][1];
-                    const uint64_t b0 = s == 0 ? dB[0] : s == 1 ? dB[1] : dB[2];
+                    uint64_t a0 = dA[0][0], a1 = dA[0][1], b0 = dB[0];
+#pragma unroll
+                    for (int q = 1; q < kGOpsMax; ++q)
+                        if (s == q) { a0 = dA[q][0]; a1 = dA[q][1]; b0 = dB[q]; }
 #pragma unroll
                     for (int kk = 0; kk < kKC / 16; ++kk) {
                         const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;

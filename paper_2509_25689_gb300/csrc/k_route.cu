@@ -576,19 +576,21 @@ __global__ void __launch_bounds__(1024) router_logits_kernel(const uint16_t* __r
     }
     if (!fr.on) return;
     // Routing fused in: every CTA publishes its logits and prepared tokens
-    // (each thread fences its own writes, then one count per CTA); the CTA
-    // that counts last routes every token and permutes, reading the others'
-    // logits after a fence, then publishes the result with a release store.
-    // The expert-FFN kernel, launched as this grid's dependent, waits on the
+    // with one acquire-release count (the block barrier orders every
+    // thread's stores before thread 0's count); the CTA that counts last has
+    // acquired every other CTA's stores with it, routes every token and
+    // permutes, then publishes the result with a release store.  The
+    // expert-FFN kernel, launched as this grid's dependent, waits on the
     // count (prepared tokens) and on the release flag (routing result).
-    __threadfence();
     __syncthreads();
-    if (threadIdx.x == 0) s_last = atomicAdd(fr.logits_done, 1u) == fr.n_ctas - 1u;
+    if (threadIdx.x == 0) {
+        uint32_t old;
+        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(fr.logits_done) : "memory");
+        s_last = old == fr.n_ctas - 1u;
+    }
     __syncthreads();
     if (!s_last) return;
-    __threadfence();
     route_permute_cta(S, fr.idx, fr.d, fr.offsets, fr.perm, fr.inv, fr.active, fr.plan, z, fr.wts);
-    __threadfence();
     __syncthreads();
     if (threadIdx.x == 0) asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(fr.route_ready), "r"(1u) : "memory");
 }
