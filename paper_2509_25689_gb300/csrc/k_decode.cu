@@ -231,6 +231,11 @@ __host__ __device__ __forceinline__ int stage_sb(int fmt, int ntok, int stage_by
 struct SlotCache {
     int32_t e[kMaxExperts + 1], first[kMaxExperts + 1], ntot[kMaxExperts + 1];
     int32_t pre_gu[kMaxExperts + 2], pre_dn[kMaxExperts + 2];
+    // the slot's tensors and formats (gate, up, down), copied from the expert
+    // table once: a kernel-parameter lookup with a run-time index goes
+    // through the constant cache, which the kernel's instructions share
+    const uint8_t* p[kMaxExperts + 1][3];
+    uint8_t fmt[kMaxExperts + 1][3];
 };
 
 // Stage geometry of one (kind, format, tokens per item), computed once per
@@ -1092,8 +1097,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     if (threadIdx.x == 0) s_fail = 0;
     {
         // Touch the expert table (a kernel parameter) once on this SM, so the
-        // per-item pointer lookups made after the routing result arrives hit
-        // the constant cache.
+        // slot table's lookups made when the routing result arrives hit the
+        // constant cache.
         uintptr_t v = 0;
         for (int i = threadIdx.x; i < 3 * (d.E + 1); i += kThreads) v |= reinterpret_cast<uintptr_t>(tab.p[i / 3][i % 3]);
         for (int i = threadIdx.x; i < d.E + 1; i += kThreads) v |= (uintptr_t)tab.fmt[i][0] << 8;
@@ -1117,6 +1122,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
     if (threadIdx.x == 0 && n_sh_items > 0) {
         sc.pre_gu[0] = 0; sc.pre_gu[1] = n_sh_items;
         sc.e[0] = d.E; sc.first[0] = 0; sc.ntot[0] = d.T;
+    }
+    if (threadIdx.x < 3 && d.has_shared) {
+        sc.p[0][threadIdx.x] = tab.p[d.E][threadIdx.x];
+        sc.fmt[0][threadIdx.x] = tab.fmt[d.E][threadIdx.x];
     }
     __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1199,6 +1208,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     sc.e[i] = e;
                     sc.first[i] = first;
                     sc.ntot[i] = ntot;
+                    // (the shared expert's slot 0 was filled at the start)
+                    if (i >= d.has_shared) {
+#pragma unroll
+                        for (int j = 0; j < 3; ++j) { sc.p[i][j] = tab.p[e][j]; sc.fmt[i][j] = tab.fmt[e][j]; }
+                    }
                 }
             }
 #pragma unroll
@@ -1254,8 +1268,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             const uint32_t pend = pending ? claim_issue() : 0u;
             if (item >= 0) {
                 decode_item(A, sc, s_perm, n_slots, n_gu, item, cur_gu, cur_dn, P);
-                fmt0 = tab.fmt[P.e][P.down ? 2 : 0];
-                fmt1 = tab.fmt[P.e][P.down ? 2 : 1];
+                fmt0 = sc.fmt[P.slot][P.down ? 2 : 0];
+                fmt1 = sc.fmt[P.slot][P.down ? 2 : 1];
                 const int span = P.ke - P.kb;
                 const int per0 = geo[P.down][fmt0 - 1][P.ntok - 1].per, per1 = geo[0][fmt1 - 1][P.ntok - 1].per;
                 P.nst0 = (span + per0 - 1) / per0;
@@ -1306,7 +1320,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     phase_j = pj;
                     fmt = tensor == 1 ? fmt1 : fmt0;
                     G = &geo[P.down][fmt - 1][P.ntok - 1];
-                    const uint8_t* tbase = tab.p[P.e][tensor >= 2 ? 2 : tensor];
+                    const uint8_t* tbase = sc.p[P.slot][tensor >= 2 ? 2 : tensor];
                     c_src = nullptr; c_stride = 0; c_dst = 0;
                     if (lane < G->npl) {
                         c_src = tbase + G->pl[lane] + (int64_t)(P.rb + (tensor == 3 ? 1 : 0)) * G->rbstr[lane];
@@ -1570,7 +1584,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                     // cached in shared memory (the first kMaxCachedAssign entries)
                     const float w = e_shared ? 1.0f : a < kMaxCachedAssign ? s_wts[a] : __ldcg(A.wts + a);
                     const float hv = v0 / (1.0f + expf(-v0)) * v1 * w;
-                    const int fam = families_of(tab.fmt[e_e][2]);
+                    const int fam = families_of(sc.fmt[e_slot][2]);
                     __half* hq = A.hq + (size_t)a * kFamSlots * A.nsbi * 256;
                     float* hs = A.hs + (size_t)a * A.nsbi * kStatFloats;
                     prep_block32(hv, e_rb, fam, hq, hs, A.nsbi);
