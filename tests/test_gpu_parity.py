@@ -362,18 +362,20 @@ def test_status_word_clean_after_forward_on_every_path(torch_cuda):
         assert torch.isfinite(out).all()
 
 
-def test_wait_give_up_reports_status_and_context_stays_usable(torch_cuda, orc):
+@pytest.mark.parametrize("T", [1, 3])
+def test_wait_give_up_reports_status_and_context_stays_usable(torch_cuda, orc, T):
     """The bounded-wait give-up path, made to run out on purpose: a test hook
     shortens every pipeline wait of the next decode call to 1 ms and has the
     gate/up producer post nothing for its first stage.  The consumers' wait
     on that stage ends, the kernels record it in the error word and exit
     (no copy left in flight), moe_quant_status returns MQ_EDEVICE with the
-    full-barrier bit, and the next call runs normally and matches the oracle."""
+    full-barrier bit, and the next call runs normally and matches the oracle.
+    T = 1 runs the one-token kernel, whose item-finishing warp then has to
+    leave its wait for items that never come; T = 3 the several-token one."""
     import torch
     mq = mq_lib()
-    spec = replace(SMALL_MIXED, tokens=3)
+    spec = replace(SMALL_MIXED, tokens=T)
     layer = DeviceLayer(spec, 4, fmts=SMALL_MIXED_FMTS)
-    T = 3
     x_bits = tokens(spec, 4)
     x = torch.from_numpy(x_bits.view(np.int16)).cuda()
     out = torch.empty((T, spec.hidden), device="cuda")
