@@ -157,11 +157,13 @@ constexpr int kNT = kConsumers >= 16 ? 1 : 2;       // 16-row MMA tiles per warp
 constexpr int kCols = kConsumers * kNT / 2;         // superblock columns the warps are spread over
 constexpr int kThreads = (kConsumers + 1) * 32;     // + one producer warp
 constexpr int kProducerWarp = kConsumers;
-// Ring of kNST slots (4 x 48 KB: Q3_K down stages are 37 KB, Q2_K gate/up
-// stages of 14 superblocks 47 KB, Q8_0 stages of 5 superblocks 44 KB)
+// Ring of kNST slots (one-token kernel 4 x 48 KB: Q3_K down stages are
+// 37 KB, Q2_K gate/up stages of 14 superblocks 47 KB, Q8_0 stages of 5
+// superblocks 44 KB; several-token kernel 4 x 46 KB, which leaves room for
+// its second item-end reduction buffer)
 constexpr int kNST = MQ_DECODE_SLOTS;
-constexpr int kRingBytes = 192 * 1024;
-constexpr int kSlotBytes = kRingBytes / kNST;
+__host__ __device__ constexpr int ring_bytes(int mt) { return mt == 1 ? 192 * 1024 : 184 * 1024; }
+__host__ __device__ constexpr int slot_bytes(int mt) { return ring_bytes(mt) / kNST; }
 constexpr int kStageSb = 16;                        // superblocks per stage (Q8_0: 8), fewer if over budget
 constexpr int kMaxCachedAssign = 1024;              // routed assignments cached in smem
 #ifndef MQ_SPLIT_SHARED
@@ -249,12 +251,12 @@ struct Geo {
 };
 static_assert(sizeof(Geo) == 88, "geometry record");
 
-__host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int fmt, int ntok) {
+__host__ __device__ inline void make_geo(Geo& G, const Dims& d, bool down, int fmt, int ntok, int slot_b) {
     const int nsb = down ? (d.I + 255) / 256 : (d.H + 255) / 256;
     const TensorLayout L = tensor_layout(fmt, down ? d.H : d.I, down ? d.I : d.H);
     const PlaneBytes pb = plane_bytes(fmt);
     const int bmul = block_len(fmt) == 32 ? 8 : 1;   // Q8_0 / BF16: 8 blocks of 32 per superblock
-    G.per = (int16_t)stage_sb(fmt, ntok, kSlotBytes);
+    G.per = (int16_t)stage_sb(fmt, ntok, slot_b);
     G.nst = (int16_t)((nsb + G.per - 1) / G.per);
     G.npl = (int16_t)pb.n;
     int at = 0;
@@ -1069,7 +1071,7 @@ template <int MT>
 __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant__ ExpertTab tab,
                                                           const __grid_constant__ DecodeArgs A) {
     extern __shared__ __align__(128) uint8_t smem[];
-    constexpr int kRedBufs = MT == 1 ? 2 : 1;          // item-end reduction buffers (smem budget)
+    constexpr int kRedBufs = 2;                         // item-end reduction buffers
     __shared__ SlotCache sc;
     __shared__ int32_t s_perm[kMaxCachedAssign];
     __shared__ float s_wts[kMaxCachedAssign];   // routing weights by assignment (the first kMaxCachedAssign)
@@ -1348,7 +1350,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
                 }
                 const int per = G->per;
                 const int s0 = P.kb + (pj - phase_j) * per, ks = min(per, P.ke - s0);
-                const uint32_t stage = ring + slot * kSlotBytes;
+                const uint32_t stage = ring + slot * slot_bytes(MT);
                 const uint32_t bytes = c_src ? (uint32_t)ks * c_stride : 0u;
                 uint32_t total = bytes;
 #pragma unroll
@@ -1420,7 +1422,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_kernel(const __grid_constant_
             }
             const Hdr& H = hdr[slot];
             if (H.item < 0) break;
-            const uint32_t stage = ring + slot * kSlotBytes;
+            const uint32_t stage = ring + slot * slot_bytes(MT);
             const int fmt = H.fmt, ks = H.ks, ntok = H.ntok;
             const bool dn = H.tensor >= 2;
             const Geo& GS = geo[dn ? 1 : 0][fmt - 1][ntok - 1];
@@ -1628,8 +1630,8 @@ __global__ void combine_kernel(Dims d, const float* __restrict__ pdn, float* __r
 }
 
 void decode_setup() {
-    cudaFuncSetAttribute(ffn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
-    cudaFuncSetAttribute(ffn_kernel<kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    cudaFuncSetAttribute(ffn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, ring_bytes(1));
+    cudaFuncSetAttribute(ffn_kernel<kDecodeTok>, cudaFuncAttributeMaxDynamicSharedMemorySize, ring_bytes(kDecodeTok));
 }
 
 void combine_setup() { prefer_max_shared(combine_kernel); }
@@ -1644,7 +1646,6 @@ size_t decode_counter_bytes(const Dims& d) {
 
 cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w, float* out, cudaStream_t s) {
     if (d.T == 0) return cudaSuccess;
-    const int smem = kRingBytes;
     const int num_sms = device_setup(kSetupDecode, decode_setup);
     if (num_sms <= 0) return cudaErrorInvalidDevice;
     DecodeArgs A;
@@ -1668,11 +1669,13 @@ cudaError_t launch_decode_mma(const Dims& d, const ExpertTab& tab, const Work& w
     A.fail_first_stage = 0;
     uint64_t test_ns = 0;
     if (take_wait_test(&test_ns)) { A.wait_ns = test_ns; A.fail_first_stage = 1; }
-    for (int dn = 0; dn < 2; ++dn)
-        for (int f = 1; f <= kNumFormats; ++f)
-            for (int n = 1; n <= kDecodeTok; ++n) make_geo(A.geo[dn][f - 1][n - 1], d, dn == 1, f, n);
     // one token: every item carries one, and the accumulators shrink to one token's
     const bool one = d.T == 1;
+    const int smem = ring_bytes(one ? 1 : kDecodeTok);
+    for (int dn = 0; dn < 2; ++dn)
+        for (int f = 1; f <= kNumFormats; ++f)
+            for (int n = 1; n <= kDecodeTok; ++n)
+                make_geo(A.geo[dn][f - 1][n - 1], d, dn == 1, f, n, slot_bytes(one ? 1 : kDecodeTok));
     prof_begin("ffn_mma", s);
     cudaError_t err = one ? launch_pdl(ffn_kernel<1>, dim3(num_sms), dim3(kThreads), smem, s, tab, A)
                           : launch_pdl(ffn_kernel<kDecodeTok>, dim3(num_sms), dim3(kThreads), smem, s, tab, A);
