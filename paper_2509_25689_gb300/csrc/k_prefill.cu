@@ -149,6 +149,12 @@ constexpr int kGOpsMax = MQ_GOPS_GU > MQ_GOPS_DN ? MQ_GOPS_GU : MQ_GOPS_DN;
 constexpr int kGPk = MQ_GPK;                   // packed-record stages
 constexpr int kGPkBytes = 37376;               // Q6_K + Q6_K half superblock of 128 rows: 2 x 18,688
 __host__ __device__ constexpr int g_smem(bool down) { return g_ops(down) * g_slot(down) + kGPk * kGPkBytes; }
+// a unit's tokens are the MMA's N (at most 256) and its TMEM columns (a power
+// of two); the dynamic shared memory leaves room for the kernel's static
+// arrays (about 7 KB) within the 227 KB of a CTA
+static_assert(kGNT >= 32 && kGNT <= 256 && (kGNT & (kGNT - 1)) == 0, "tokens per unit");
+static_assert(kGOpsMax >= 2 && kGOpsMax <= 4 && kGPk >= 2, "ring depths");
+static_assert(g_smem(false) <= 219 * 1024 && g_smem(true) <= 219 * 1024, "shared memory per CTA");
 
 // Activation rows of the warp-specialised GEMM in the order its units read
 // them: slot positions r (the permutation's order for the routed experts,
